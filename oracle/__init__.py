@@ -1,0 +1,12 @@
+"""CPU oracle of the A-PACK inner-LLM prune step (test infrastructure only).
+
+Only the tests, the smoke check and the CPU-baseline leg of the benchmark may
+import this package.  The CUDA library never calls it, and it never calls the
+CUDA library: the two share no code.  See ``apack_oracle.py``.
+"""
+
+from .apack_oracle import (  # noqa: F401
+    MOD_OTHER, MOD_AUDIO, MOD_VISUAL,
+    bf16_to_f64, relevance_scores, keep_count, step_keep_counts, select_keep,
+    compact_rows, new_cu_seqlens, prune_step, score_tolerance,
+)
