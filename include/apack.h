@@ -1,0 +1,180 @@
+/*
+ * apack.h -- C ABI of the A-PACK inner-LLM prune step on NVIDIA GB300 (sm_103a).
+ *
+ * A-PACK (Sec. 3.2, "Inner-LLM Query-Aware Compression"; Algorithm 1, the
+ * inner-LLM loop) prunes multimodal tokens inside the decoder: at a pruning
+ * layer it scores every cached audio and visual token by the attention it
+ * receives from the text query (Eq. inner_score), keeps the top fraction of
+ * them (Eq. inner) and drops the rest together with their key-value entries,
+ * so that later layers and decoding see a shorter sequence.
+ *
+ * Conventions shared by every entry point:
+ *  - Pointers are DEVICE memory unless the name ends in _h (HOST memory).
+ *  - The caller owns every buffer.  The library allocates nothing, keeps no
+ *    per-call state, never synchronises inside a step and never traps: every
+ *    call returns an apack_status.  All device work is enqueued on `stream`
+ *    (a cudaStream_t passed as void*; NULL = legacy default stream).
+ *  - bf16 data are passed as untyped pointers to 16-bit storage.
+ *  - A packed (ragged) batch of B sequences stores token t of sequence b at
+ *    row cu_seqlens[b] + t of every per-token array.
+ *  - Arguments are checked on the host before anything is enqueued
+ *    (APACK_EINVAL).  Problems only the device can see (modality counts that
+ *    disagree with the host counts, a bounded wait that gave up) are written
+ *    to an error word in the workspace and read with apack_device_error().
+ *  - Calls that share a workspace must be ordered (same stream, or joined).
+ */
+#ifndef APACK_H
+#define APACK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t apack_status;
+enum {
+  APACK_OK = 0,
+  APACK_EINVAL = 1,        /* bad argument (null, size, alignment, shape, ratio) */
+  APACK_ECUDA = 2,         /* a CUDA runtime or driver call failed */
+  APACK_EWORKSPACE = 3,    /* workspace too small (see apack_workspace_size) */
+  APACK_ETIMEOUT = 4,      /* device error word: a bounded wait gave up */
+  APACK_EDEVICE = 5,       /* device error word: device data disagree with host counts */
+  APACK_EUNSUPPORTED = 6   /* shape outside what this build supports (e.g. head_dim != 128) */
+};
+
+/* Per-token modality codes.  S, the set of prunable "cached multimodal
+   tokens" of Sec. 3.2, is every token coded AUDIO or VISUAL; OTHER tokens
+   (system prompt, text, the query itself) are never scored or dropped. */
+enum { APACK_MOD_OTHER = 0, APACK_MOD_AUDIO = 1, APACK_MOD_VISUAL = 2 };
+
+/* Selection segments.  PER_MODALITY takes the top-k separately for the audio
+   and the visual tokens of each sequence (two keep counts per sequence);
+   JOINT takes one top-k over all of S, the literal form of Eq. inner. */
+enum { APACK_SELECT_PER_MODALITY = 0, APACK_SELECT_JOINT = 1 };
+
+/* Maximum sizes of this build. */
+#define APACK_HEAD_DIM 128
+#define APACK_MAX_SEQS 4096
+
+/* The packed batch entering a pruning layer. */
+typedef struct apack_seqs {
+  int32_t num_seqs;             /* B, 1 .. APACK_MAX_SEQS */
+  const int32_t *cu_seqlens_h;  /* [B+1] token offsets, cu_seqlens_h[0] == 0, non-decreasing */
+  const int32_t *cu_qlens_h;    /* [B+1] offsets of each sequence's query rows in the packed Q */
+  const int32_t *n_audio_h;     /* [B] audio tokens per sequence (verified on the device) */
+  const int32_t *n_visual_h;    /* [B] visual tokens per sequence (verified on the device) */
+  const uint8_t *modality;      /* [T] APACK_MOD_* per token, T = cu_seqlens_h[B] */
+  int32_t num_q_heads;          /* Hq */
+  int32_t num_kv_heads;         /* Hkv; Hq % Hkv == 0, query head h reads key head h / (Hq/Hkv) */
+  int32_t head_dim;             /* D; must be APACK_HEAD_DIM */
+} apack_seqs;
+
+/* One group of per-token planes to compact (e.g. the K cache of layers l..L-1).
+   Plane p, token row t lives at  base + p*plane_stride + t*row_stride.
+   Rows of >= 16 bytes whose addresses and strides are 16-byte aligned take
+   the vectorised path; any other row size is copied with narrower accesses.
+   src and dst must not overlap unless src == dst with equal strides (in place). */
+typedef struct apack_plane {
+  const void *src;
+  void *dst;
+  int64_t src_plane_stride;     /* bytes between planes of src */
+  int64_t dst_plane_stride;     /* bytes between planes of dst */
+  int64_t src_row_stride;       /* bytes between token rows of src */
+  int64_t dst_row_stride;       /* bytes between token rows of dst */
+  int64_t row_bytes;            /* bytes copied per token row */
+  int32_t num_planes;
+  int32_t reserved;
+} apack_plane;
+
+/* Bytes of device workspace the calls below need for this batch (256-byte
+   aligned start required).  Depends on B, the query rows and head counts. */
+apack_status apack_workspace_size(const apack_seqs *seqs, size_t *bytes);
+
+/* Keep counts of Eq. inner, ceil((1-P)|S|), from keep ratios r = 1-P.
+   keep_ratio_h: [B][2] (audio, visual) in [0, 1]; with APACK_SELECT_JOINT
+   only [b][0] is used and applies to |S| = n_audio + n_visual.
+   The ratio is read on a 1e-6 grid: k = min(n, ceil(round(r*1e6) * n / 1e6))
+   in integer arithmetic, so that 0.55 * 100 keeps 55, not 56.
+   Outputs (host): keep_count_h [B][2] (JOINT: [b][1] = 0) and
+   new_cu_seqlens_h [B+1], the packed offsets after the step. */
+apack_status apack_keep_counts(const apack_seqs *seqs, const float *keep_ratio_h, int32_t select_mode,
+                               int32_t *keep_count_h, int32_t *new_cu_seqlens_h);
+
+/* Relevance scores of Eq. inner_score (Sec. 3.2), averaged over all Hq query
+   heads and all query rows of each sequence:
+     I_i = 1/(Hq * n_q) * sum_h sum_r  exp(q_{r,h}.k_{i,g(h)} / sqrt(D))
+                                      / sum_{j in S} exp(q_{r,h}.k_{j,g(h)} / sqrt(D))
+   for i in S of the sequence, and I_i = 0 for tokens outside S.
+   q: bf16 [sum n_q][Hq][D], contiguous (the query rows at the pruning layer).
+   k: bf16 keys of the pruning layer, token t at k + t*k_token_stride, laid
+      out [Hkv][D] within the row; k_token_stride a multiple of 16 bytes.
+   scores: fp32 [T].  Computed in fp32 from bf16 products on the tensor
+   cores; deterministic (fixed reduction order, no atomics). */
+apack_status apack_score(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
+                         float *scores, void *ws, size_t ws_bytes, void *stream);
+
+/* Top-k selection of Eq. inner per segment (see APACK_SELECT_*): keeps the
+   keep_count_h[b][m] highest scores of each segment, equal scores going to the
+   lower token index, plus every token outside S.
+   Outputs: keep_idx [T_out] (kept token indices in ascending order, i.e. the
+   original order; T_out = new_cu_seqlens_h[B] of apack_keep_counts),
+   modality_out [T_out] (nullable; the compacted modality mask),
+   dst_of_src [T] (nullable; output row of each token or -1),
+   new_cu_seqlens [B+1] (nullable; device copy of the new offsets).
+   scores must be finite and >= 0 (as apack_score produces). */
+apack_status apack_select(const apack_seqs *seqs, const float *scores, const int32_t *keep_count_h,
+                          int32_t select_mode, int32_t *keep_idx, uint8_t *modality_out,
+                          int32_t *dst_of_src, int32_t *new_cu_seqlens, void *ws, size_t ws_bytes,
+                          void *stream);
+
+/* KV-cache and hidden-state slicing (Sec. 3.2, last sentence; Algorithm 1,
+   "slice their KV-cache entries"): for every plane of every group,
+   dst row j = src row keep_idx[j], j < n_out, bit for bit.
+   planes_h: host array of num_groups descriptors.  Out of place only in this
+   build (src == dst returns APACK_EUNSUPPORTED). */
+apack_status apack_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes_h,
+                           int32_t num_groups, void *stream);
+
+/* One pruning step at layer `layer` of a num_layers-layer decoder
+   (Algorithm 1, one iteration of the inner-LLM loop): apack_score on the
+   layer's keys, apack_select, then compaction of the K and V caches of
+   layers [layer, num_layers), of the hidden states and of any extra planes.
+   k_cache / v_cache: bf16, slab 0 = layer `layer`, slab i at
+     + i*kv_layer_stride bytes, token t at + t*Hkv*D*2 bytes within a slab.
+   k_out / v_out: the same layout with kv_out_layer_stride (out of place).
+   hidden / hidden_out: bf16 [T][hidden_dim] / [T_out][hidden_dim] (hidden may be NULL).
+   keep_count_h: [B][2] counts (e.g. cumulative schedules); when NULL they
+   come from keep_ratio_h as in apack_keep_counts.
+   new_cu_seqlens_h (host, [B+1]) receives the new offsets before the call
+   returns (no device synchronisation needed).
+   scores (device [T] fp32) receives the relevance scores.
+   stage_events_h: NULL, or 4 cudaEvent_t recorded on `stream` before
+   scoring, before selection, before compaction and at the end. */
+apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num_layers,
+                              const void *q, const void *k_cache, const void *v_cache,
+                              int64_t kv_layer_stride, const void *hidden, int64_t hidden_dim,
+                              const float *keep_ratio_h, const int32_t *keep_count_h, int32_t select_mode,
+                              void *k_out, void *v_out, int64_t kv_out_layer_stride, void *hidden_out,
+                              const apack_plane *extra_planes_h, int32_t num_extra,
+                              uint8_t *modality_out, int32_t *keep_idx, int32_t *new_cu_seqlens_h,
+                              int32_t *new_cu_seqlens, float *scores, void *ws, size_t ws_bytes,
+                              void *const *stage_events_h, void *stream);
+
+/* Synchronises `stream`, then reads the device error word of `ws` into
+   *code_out (APACK_OK, APACK_ETIMEOUT or APACK_EDEVICE) and clears it when
+   `clear` is non-zero. */
+apack_status apack_device_error(const void *ws, void *stream, int32_t *code_out, int32_t clear);
+
+/* Number of kernels this library has launched in the calling process. */
+uint64_t apack_launch_count(void);
+
+/* Human-readable name of a status code (static string). */
+const char *apack_status_string(apack_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* APACK_H */

@@ -1,0 +1,232 @@
+"""Python binding of libapack, the GB300 (sm_103a) A-PACK inner-LLM prune step.
+
+Argument marshalling only: every computation runs in the CUDA kernels of
+``libapack.so`` behind the C ABI declared in ``include/apack.h``.  The
+functions keep the C names (``apack_score``, ``apack_select``,
+``apack_compact``, ``apack_prune_step``, ...).  Device buffers are passed as
+torch CUDA tensors (their data pointers) and streams as torch streams;
+PyTorch only provides memory and streams.
+
+Importing this package loads the library and raises if it has not been
+built (``__graft_entry__.build()`` or ``python -m paper_2608_08794_gb300._build``).
+There is no fallback.
+"""
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libapack.so")
+
+APACK_OK, APACK_EINVAL, APACK_ECUDA, APACK_EWORKSPACE, APACK_ETIMEOUT, APACK_EDEVICE, APACK_EUNSUPPORTED = range(7)
+APACK_MOD_OTHER, APACK_MOD_AUDIO, APACK_MOD_VISUAL = 0, 1, 2
+APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT = 0, 1
+APACK_HEAD_DIM = 128
+
+EXPORTED = ("apack_workspace_size", "apack_keep_counts", "apack_score", "apack_select", "apack_compact",
+            "apack_prune_step", "apack_device_error", "apack_launch_count", "apack_status_string")
+
+
+class ApackError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+class apack_seqs(ctypes.Structure):
+    _fields_ = [("num_seqs", ctypes.c_int32),
+                ("cu_seqlens_h", ctypes.POINTER(ctypes.c_int32)),
+                ("cu_qlens_h", ctypes.POINTER(ctypes.c_int32)),
+                ("n_audio_h", ctypes.POINTER(ctypes.c_int32)),
+                ("n_visual_h", ctypes.POINTER(ctypes.c_int32)),
+                ("modality", ctypes.c_void_p),
+                ("num_q_heads", ctypes.c_int32),
+                ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32)]
+
+
+class apack_plane(ctypes.Structure):
+    _fields_ = [("src", ctypes.c_void_p), ("dst", ctypes.c_void_p),
+                ("src_plane_stride", ctypes.c_int64), ("dst_plane_stride", ctypes.c_int64),
+                ("src_row_stride", ctypes.c_int64), ("dst_row_stride", ctypes.c_int64),
+                ("row_bytes", ctypes.c_int64), ("num_planes", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"libapack.so is not built ({LIB_PATH}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I32, I64, SZ, VP = ctypes.POINTER, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t, ctypes.c_void_p
+    PI32 = P(I32)
+    lib.apack_workspace_size.argtypes = [P(apack_seqs), P(SZ)]
+    lib.apack_keep_counts.argtypes = [P(apack_seqs), P(ctypes.c_float), I32, PI32, PI32]
+    lib.apack_score.argtypes = [P(apack_seqs), VP, VP, I64, VP, VP, SZ, VP]
+    lib.apack_select.argtypes = [P(apack_seqs), VP, PI32, I32, VP, VP, VP, VP, VP, SZ, VP]
+    lib.apack_compact.argtypes = [VP, I64, P(apack_plane), I32, VP]
+    lib.apack_prune_step.argtypes = [P(apack_seqs), I32, I32, VP, VP, VP, I64, VP, I64, P(ctypes.c_float), PI32,
+                                     I32, VP, VP, I64, VP, P(apack_plane), I32, VP, VP, PI32, VP, VP, VP, SZ,
+                                     P(VP), VP]
+    lib.apack_device_error.argtypes = [VP, VP, PI32, I32]
+    lib.apack_launch_count.argtypes = []
+    lib.apack_launch_count.restype = ctypes.c_uint64
+    lib.apack_status_string.argtypes = [I32]
+    lib.apack_status_string.restype = ctypes.c_char_p
+    for name in EXPORTED:
+        if name not in ("apack_launch_count", "apack_status_string"):
+            getattr(lib, name).restype = I32
+    return lib
+
+
+_lib = _load()
+
+
+def status_string(status):
+    return _lib.apack_status_string(int(status)).decode()
+
+
+def _check(status, where):
+    if status != APACK_OK:
+        raise ApackError(status, where)
+
+
+def _ptr(t):
+    """Device pointer of a torch tensor (or None -> NULL)."""
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _i32(a):
+    return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+
+
+class Seqs:
+    """A packed batch: host offsets and counts plus the device modality mask.
+
+    Keeps the host arrays alive for as long as the ``apack_seqs`` struct is used."""
+
+    def __init__(self, cu_seqlens, cu_qlens, n_audio, n_visual, modality, num_q_heads, num_kv_heads,
+                 head_dim=APACK_HEAD_DIM):
+        self.cu_seqlens = _i32(cu_seqlens)
+        self.cu_qlens = _i32(cu_qlens)
+        self.n_audio = _i32(n_audio)
+        self.n_visual = _i32(n_visual)
+        self.modality = modality
+        I32P = ctypes.POINTER(ctypes.c_int32)
+        self.struct = apack_seqs(
+            num_seqs=len(self.cu_seqlens) - 1,
+            cu_seqlens_h=self.cu_seqlens.ctypes.data_as(I32P),
+            cu_qlens_h=self.cu_qlens.ctypes.data_as(I32P),
+            n_audio_h=self.n_audio.ctypes.data_as(I32P),
+            n_visual_h=self.n_visual.ctypes.data_as(I32P),
+            modality=None if modality is None else modality.data_ptr(),
+            num_q_heads=num_q_heads, num_kv_heads=num_kv_heads, head_dim=head_dim)
+
+    @property
+    def num_seqs(self):
+        return len(self.cu_seqlens) - 1
+
+    @property
+    def total_tokens(self):
+        return int(self.cu_seqlens[-1])
+
+    def ref(self):
+        return ctypes.byref(self.struct)
+
+
+def apack_workspace_size(seqs):
+    n = ctypes.c_size_t(0)
+    _check(_lib.apack_workspace_size(seqs.ref(), ctypes.byref(n)), "apack_workspace_size")
+    return n.value
+
+
+def apack_keep_counts(seqs, keep_ratio, select_mode=APACK_SELECT_PER_MODALITY):
+    """Keep counts [B, 2] and new offsets [B+1] (host numpy) from keep ratios [B, 2]."""
+    r = np.ascontiguousarray(np.asarray(keep_ratio, dtype=np.float32).reshape(seqs.num_seqs, 2))
+    k = np.zeros((seqs.num_seqs, 2), np.int32)
+    cu = np.zeros(seqs.num_seqs + 1, np.int32)
+    I32P = ctypes.POINTER(ctypes.c_int32)
+    _check(_lib.apack_keep_counts(seqs.ref(), r.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), select_mode,
+                                  k.ctypes.data_as(I32P), cu.ctypes.data_as(I32P)), "apack_keep_counts")
+    return k, cu
+
+
+def apack_score(seqs, q, k, k_token_stride, scores, ws, stream=None):
+    _check(_lib.apack_score(seqs.ref(), _ptr(q), _ptr(k), int(k_token_stride), _ptr(scores), _ptr(ws),
+                            ws.numel() * ws.element_size(), _stream(stream)), "apack_score")
+
+
+def apack_select(seqs, scores, keep_count, keep_idx, ws, select_mode=APACK_SELECT_PER_MODALITY,
+                 modality_out=None, dst_of_src=None, new_cu_seqlens=None, stream=None):
+    kc = _i32(keep_count).reshape(-1)
+    _check(_lib.apack_select(seqs.ref(), _ptr(scores), kc.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
+                             select_mode, _ptr(keep_idx), _ptr(modality_out), _ptr(dst_of_src),
+                             _ptr(new_cu_seqlens), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)),
+           "apack_select")
+
+
+def make_plane(src, dst, row_bytes, num_planes=1, src_plane_stride=0, dst_plane_stride=0, src_row_stride=None,
+               dst_row_stride=None):
+    """Descriptor of a group of per-token planes (byte strides)."""
+    return apack_plane(src=src.data_ptr(), dst=dst.data_ptr(), src_plane_stride=src_plane_stride,
+                       dst_plane_stride=dst_plane_stride,
+                       src_row_stride=row_bytes if src_row_stride is None else src_row_stride,
+                       dst_row_stride=row_bytes if dst_row_stride is None else dst_row_stride,
+                       row_bytes=row_bytes, num_planes=num_planes, reserved=0)
+
+
+def apack_compact(keep_idx, n_out, planes, stream=None):
+    arr = (apack_plane * max(1, len(planes)))(*planes)
+    _check(_lib.apack_compact(_ptr(keep_idx), int(n_out), arr, len(planes), _stream(stream)), "apack_compact")
+
+
+def apack_prune_step(seqs, layer, num_layers, q, k_cache, v_cache, kv_layer_stride, hidden, hidden_dim,
+                     keep_ratio=None, keep_count=None, select_mode=APACK_SELECT_PER_MODALITY, k_out=None,
+                     v_out=None, kv_out_layer_stride=0, hidden_out=None, extra_planes=(), modality_out=None,
+                     keep_idx=None, new_cu_seqlens=None, scores=None, ws=None, stage_events=None, stream=None):
+    """One pruning step; returns the new packed offsets (host numpy [B+1])."""
+    B = seqs.num_seqs
+    I32P = ctypes.POINTER(ctypes.c_int32)
+    ratio = None
+    if keep_ratio is not None:
+        ratio = np.ascontiguousarray(np.asarray(keep_ratio, dtype=np.float32).reshape(B, 2))
+    kc = None if keep_count is None else _i32(keep_count).reshape(-1)
+    new_cu = np.zeros(B + 1, np.int32)
+    arr = (apack_plane * max(1, len(extra_planes)))(*extra_planes)
+    ev = None
+    if stage_events is not None:
+        ev = (ctypes.c_void_p * 4)(*[e.cuda_event if hasattr(e, "cuda_event") else e for e in stage_events])
+    st = _lib.apack_prune_step(
+        seqs.ref(), int(layer), int(num_layers), _ptr(q), _ptr(k_cache), _ptr(v_cache), int(kv_layer_stride),
+        _ptr(hidden), int(hidden_dim),
+        None if ratio is None else ratio.ctypes.data_as(ctypes.POINTER(ctypes.c_float)),
+        None if kc is None else kc.ctypes.data_as(I32P), select_mode, _ptr(k_out), _ptr(v_out),
+        int(kv_out_layer_stride), _ptr(hidden_out), arr, len(extra_planes), _ptr(modality_out), _ptr(keep_idx),
+        new_cu.ctypes.data_as(I32P), _ptr(new_cu_seqlens), _ptr(scores), _ptr(ws),
+        0 if ws is None else ws.numel() * ws.element_size(), ev, _stream(stream))
+    _check(st, "apack_prune_step")
+    return new_cu
+
+
+def apack_device_error(ws, stream=None, clear=True):
+    code = ctypes.c_int32(0)
+    _check(_lib.apack_device_error(_ptr(ws), _stream(stream), ctypes.byref(code), 1 if clear else 0),
+           "apack_device_error")
+    return code.value
+
+
+def apack_launch_count():
+    return int(_lib.apack_launch_count())
+
+
+def library_path():
+    return LIB_PATH

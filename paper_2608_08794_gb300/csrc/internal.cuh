@@ -1,0 +1,64 @@
+// internal.cuh -- declarations shared by the translation units of libapack.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "apack.h"
+
+namespace apack {
+
+// Sequences handled by one kernel launch; larger batches take several launches.
+constexpr int kSeqsPerLaunch = 64;
+// Wall-clock limit of every device-side wait.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+// Key splits of the row-statistics pass (upper bound, sizes the workspace).
+constexpr int kMaxSplits = 32;
+
+// Device error word at offset 0 of the workspace.
+struct DeviceError {
+  int32_t code;     // APACK_OK, APACK_ETIMEOUT, APACK_EDEVICE (first error wins)
+  int32_t where;    // kernel-specific location code
+  int32_t info[2];
+};
+
+__device__ __forceinline__ void raise_device_error(DeviceError *e, int32_t code, int32_t where, int32_t a = 0,
+                                                   int32_t b = 0) {
+  if (atomicCAS(&e->code, 0, code) == 0) {
+    e->where = where;
+    e->info[0] = a;
+    e->info[1] = b;
+  }
+}
+
+// Workspace carve-up (offsets in bytes from the 256-byte aligned start).
+struct WsLayout {
+  size_t err_off;     // DeviceError
+  size_t part_off;    // float2 [kMaxSplits][sum n_q][Hq]: per-split (max, sum) in log2 units
+  size_t lse_off;     // float [chunks][256]: log2 normalisers per query-row chunk, +inf padding
+  size_t total;
+  int64_t lse_chunks;
+};
+
+// Query tokens per MMA tile: rows of a tile are (token, head-in-group) pairs.
+__host__ __device__ inline int rows_tile1(int group) { return 128 / group; }   // row-stats pass (M = 128)
+__host__ __device__ inline int rows_tile2(int group) { return 256 / group; }   // column pass (N = 256)
+
+WsLayout workspace_layout(const apack_seqs *seqs);
+int device_sm_count();
+void count_launches(uint64_t n);
+apack_status check_cuda(cudaError_t e);
+
+apack_status validate_seqs(const apack_seqs *seqs, int64_t *total_tokens, int64_t *total_qrows);
+
+apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
+                       float *scores, void *ws, cudaStream_t stream);
+apack_status run_select(const apack_seqs *seqs, const float *scores, const int32_t *keep_count_h, int32_t mode,
+                        int32_t *keep_idx, uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu_seqlens,
+                        void *ws, cudaStream_t stream);
+apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes, int32_t num_groups,
+                         cudaStream_t stream);
+
+}  // namespace apack

@@ -1,0 +1,128 @@
+"""Host-side driver of a progressive pruning schedule (Algorithm 1, the loop
+over pruning layers l >= L_mid; Sec. 3.2: pruning repeats at later layers on
+the already shortened sequence).
+
+Each step calls ``apack_prune_step`` once.  Step i prunes at layer l_i and
+compacts the K/V slabs of layers [l_i, L) plus the hidden states; step i+1
+reads its layer's keys from slab (l_{i+1} - l_i) of step i's output.  Two
+output buffers alternate (ping-pong), so the input cache of step 0 is never
+written and the schedule can be replayed on the same inputs.
+
+Only buffer management and argument marshalling happen here.
+"""
+
+import numpy as np
+import torch
+
+from . import (Seqs, apack_prune_step, apack_workspace_size, APACK_HEAD_DIM, APACK_SELECT_PER_MODALITY)
+
+
+class ProgressivePrune:
+    def __init__(self, cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, num_kv_heads, num_layers, hidden_dim,
+                 prune_layers, keep_counts, device="cuda", select_mode=APACK_SELECT_PER_MODALITY,
+                 with_hidden=True):
+        """keep_counts[i]: int array [B, 2] of the tokens each segment keeps after step i."""
+        self.dev = torch.device(device)
+        self.cu0 = np.asarray(cu_seqlens, np.int32)
+        self.cuq = np.asarray(cu_qlens, np.int32)
+        self.na0 = np.asarray(n_audio, np.int32)
+        self.nv0 = np.asarray(n_visual, np.int32)
+        self.hq, self.hkv, self.L, self.H = num_q_heads, num_kv_heads, num_layers, hidden_dim
+        self.layers = list(prune_layers)
+        self.counts = [np.asarray(k, np.int32).reshape(-1, 2) for k in keep_counts]
+        self.mode = select_mode
+        self.row = num_kv_heads * APACK_HEAD_DIM * 2
+        self.T0 = int(self.cu0[-1])
+        self.B = len(self.cu0) - 1
+        other = np.diff(self.cu0) - self.na0 - self.nv0
+        self.t_out = [int((other + k[:, 0] + k[:, 1]).sum()) for k in self.counts]
+        dev, T0, Lc0 = self.dev, self.T0, num_layers - self.layers[0]
+        # inputs (filled by the caller): K/V of layers [l_0, L), hidden, modality, Q per step
+        self.k_in = torch.empty((Lc0, T0, num_kv_heads, APACK_HEAD_DIM), dtype=torch.bfloat16, device=dev)
+        self.v_in = torch.empty_like(self.k_in)
+        self.hidden_in = torch.empty((T0, hidden_dim), dtype=torch.bfloat16, device=dev) if with_hidden else None
+        self.modality_in = torch.empty(T0, dtype=torch.uint8, device=dev)
+        nq = int(self.cuq[-1])
+        self.q = [torch.empty((nq, num_q_heads, APACK_HEAD_DIM), dtype=torch.bfloat16, device=dev)
+                  for _ in self.layers]
+        # outputs, sized for the largest step
+        t1 = self.t_out[0]
+        self.k_out = [torch.empty(Lc0 * t1 * self.row // 2, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+        self.v_out = [torch.empty_like(self.k_out[0]) for _ in range(2)]
+        self.h_out = [torch.empty((t1, hidden_dim), dtype=torch.bfloat16, device=dev) if with_hidden else None
+                      for _ in range(2)]
+        self.mod_out = [torch.empty(t1, dtype=torch.uint8, device=dev) for _ in range(2)]
+        self.keep_idx = [torch.empty(max(1, t), dtype=torch.int32, device=dev) for t in self.t_out]
+        self.scores = torch.empty(max(1, T0), dtype=torch.float32, device=dev)
+        self._seqs = []
+        ws_bytes = 0
+        for i in range(len(self.layers)):
+            s = self._step_seqs(i)
+            ws_bytes = max(ws_bytes, apack_workspace_size(s))
+        self.ws = torch.zeros(ws_bytes + 256, dtype=torch.uint8, device=dev)
+        off = (-self.ws.data_ptr()) % 256
+        self.ws = self.ws[off:off + ws_bytes]
+        self.new_cu = []
+
+    def _step_seqs(self, i):
+        if i < len(self._seqs):
+            return self._seqs[i]
+        if i == 0:
+            cu, na, nv, mod = self.cu0, self.na0, self.nv0, self.modality_in
+        else:
+            other = np.diff(self.cu0) - self.na0 - self.nv0
+            k = self.counts[i - 1]
+            cu = np.concatenate([[0], np.cumsum(other + k[:, 0] + k[:, 1])]).astype(np.int32)
+            na, nv = k[:, 0], k[:, 1]
+            mod = self.mod_out[(i - 1) % 2]
+        s = Seqs(cu, self.cuq, na, nv, mod, self.hq, self.hkv)
+        self._seqs.append(s)
+        return s
+
+    def step_args(self, i):
+        """(seqs, k_in, v_in, in_layer_stride, hidden_in) entering step i; K/V as flat bf16 views."""
+        if i == 0:
+            return (self._step_seqs(0), self.k_in.view(-1), self.v_in.view(-1), self.T0 * self.row, self.hidden_in)
+        prev = (i - 1) % 2
+        t_prev = self.t_out[i - 1]
+        skip = self.layers[i] - self.layers[i - 1]
+        off = skip * t_prev * self.row // 2          # bf16 elements
+        k = self.k_out[prev][off:]
+        v = self.v_out[prev][off:]
+        return (self._step_seqs(i), k, v, t_prev * self.row, self.h_out[prev])
+
+    def run(self, events=None, stream=None):
+        """Runs every step; events[i] = 4 CUDA events per step or None."""
+        self.new_cu = [None] * len(self.layers)
+        for i in range(len(self.layers)):
+            self.run_step(i, None if events is None else events[i], stream)
+
+    def run_step(self, i, events=None, stream=None):
+        if len(self.new_cu) != len(self.layers):
+            self.new_cu = [None] * len(self.layers)
+        seqs, k, v, stride, h = self.step_args(i)
+        o = i % 2
+        t_out = self.t_out[i]
+        self.new_cu[i] = apack_prune_step(
+            seqs, self.layers[i], self.L, self.q[i], k, v, stride, h, self.H, keep_count=self.counts[i],
+            select_mode=self.mode, k_out=self.k_out[o], v_out=self.v_out[o], kv_out_layer_stride=t_out * self.row,
+            hidden_out=self.h_out[o], modality_out=self.mod_out[o], keep_idx=self.keep_idx[i],
+            scores=self.scores, ws=self.ws, stage_events=events, stream=stream)
+        return self.new_cu[i]
+
+    def output_kv(self, i):
+        """Views of step i's compacted K and V: [L - l_i, t_out_i, Hkv, D]."""
+        o = i % 2
+        n = (self.L - self.layers[i]) * self.t_out[i] * self.row // 2
+        shape = (self.L - self.layers[i], self.t_out[i], self.hkv, APACK_HEAD_DIM)
+        return self.k_out[o][:n].view(shape), self.v_out[o][:n].view(shape)
+
+    def output_hidden(self, i):
+        return None if self.h_out[i % 2] is None else self.h_out[i % 2][:self.t_out[i]]
+
+    def mm_tokens_per_step(self):
+        """|S| entering each step (the unit of the throughput metric)."""
+        out = [int(self.na0.sum() + self.nv0.sum())]
+        for k in self.counts[:-1]:
+            out.append(int(k.sum()))
+        return out

@@ -1,0 +1,250 @@
+"""Kernel-level parity of the CUDA path against the oracle, through the C ABI.
+
+Sizes span several tiles and ragged tails: 256-key blocks and 128-key tiles
+of the scoring passes, 126-row (7 heads x 18 tokens) query tiles, 8-CTA
+clusters of the selection, 512-byte pieces of the gather.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from parity import check_scores, check_keep
+from synth.gen import f32_to_bf16_bits
+
+pytestmark = pytest.mark.gpu
+
+D = 128
+
+
+@pytest.fixture(scope="module")
+def ap():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2608_08794_gb300 as ap
+    return ap
+
+
+def dev(a):
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint16:
+        a = a.view(np.int16)
+    return torch.from_numpy(a).cuda()
+
+
+def aligned_ws(ap, seqs):
+    n = ap.apack_workspace_size(seqs)
+    t = torch.zeros(n + 256, dtype=torch.uint8, device="cuda")
+    off = (-t.data_ptr()) % 256
+    return t[off:off + n]
+
+
+def bf16(x):
+    return f32_to_bf16_bits(np.asarray(x, np.float32))
+
+
+def random_batch(rng, lens, nqs, hq, hkv, p_other=0.05, scale_k=1.0, scale_q=1.0):
+    mods = []
+    for L in lens:
+        m = rng.choice([1, 2], L, p=[0.2, 0.8]).astype(np.uint8)
+        m[rng.random(L) < p_other] = 0
+        mods.append(m)
+    mod = np.concatenate(mods) if mods else np.zeros(0, np.uint8)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    cuq = np.concatenate([[0], np.cumsum(nqs)]).astype(np.int32)
+    T, NQ = int(cu[-1]), int(cuq[-1])
+    k = bf16(rng.standard_normal((T, hkv, D)) * scale_k)
+    q = bf16(rng.standard_normal((max(NQ, 1), hq, D)) * scale_q)[:NQ]
+    na = [int((mod[cu[s]:cu[s + 1]] == 1).sum()) for s in range(len(lens))]
+    nv = [int((mod[cu[s]:cu[s + 1]] == 2).sum()) for s in range(len(lens))]
+    return mod, cu, cuq, k, q, na, nv
+
+
+def gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv):
+    mod_d = dev(mod)
+    seqs = ap.Seqs(cu, cuq, na, nv, mod_d, hq, hkv)
+    ws = aligned_ws(ap, seqs)
+    T = int(cu[-1])
+    scores = torch.full((max(T, 1),), float("nan"), dtype=torch.float32, device="cuda")
+    q_d = dev(q) if q.size else torch.zeros(16, dtype=torch.int16, device="cuda")
+    ap.apack_score(seqs, q_d, dev(k), hkv * D * 2, scores, ws)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(ws) == ap.APACK_OK
+    return scores[:T].cpu().numpy()
+
+
+SHAPES = [
+    # lens, n_q per seq, Hq, Hkv
+    ([1000], [32], 28, 4),                  # one sequence, 4 key blocks + tail, two query tiles
+    ([300, 77, 1290], [5, 1, 40], 28, 4),   # ragged batch, last-query-only sequence
+    ([700], [64], 16, 2),                   # 3B heads: 8 per group, exact 128/256-row tiles
+    ([513], [3], 4, 4),                     # MHA (group 1)
+    ([129, 257, 1], [7, 19, 2], 12, 2),     # tails of one key past a tile
+    ([0, 40, 60], [2, 0, 3], 28, 4),        # empty sequence and a sequence without query rows
+]
+
+
+@pytest.mark.parametrize("lens,nqs,hq,hkv", SHAPES)
+def test_scores_match_oracle(ap, lens, nqs, hq, hkv):
+    rng = np.random.default_rng(sum(lens) + hq)
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, lens, nqs, hq, hkv)
+    got = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv)
+    ref = oracle.relevance_scores(q, k, cu, cuq, mod, hq, hkv)
+    check_scores(got, ref, strict_rel=2e-3)
+    for s in range(len(lens)):      # closed form: scores of a sequence sum to 1 when it has S and queries
+        S = ((mod[cu[s]:cu[s + 1]] == 1) | (mod[cu[s]:cu[s + 1]] == 2)).sum()
+        tot = got[cu[s]:cu[s + 1]].astype(np.float64).sum()
+        assert tot == pytest.approx(1.0 if S and nqs[s] else 0.0, abs=1e-4)
+
+
+def test_scores_large_logits_and_sequence_without_S(ap):
+    rng = np.random.default_rng(11)
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, [900, 50], [9, 4], 28, 4, scale_k=3.0, scale_q=3.0)
+    mod[900:] = 0
+    nv[1] = na[1] = 0
+    got = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, 28, 4)
+    ref = oracle.relevance_scores(q, k, cu, cuq, mod, 28, 4)
+    check_scores(got, ref)
+    assert np.all(got[900:] == 0)
+
+
+def test_scores_identical_keys_are_uniform(ap):
+    mod = np.array([0] * 16 + [1, 2, 2, 2] * 300 + [0] * 8, np.uint8)
+    T = mod.size
+    rng = np.random.default_rng(3)
+    k = np.repeat(bf16(rng.standard_normal((1, 4, D))), T, axis=0)
+    q = bf16(rng.standard_normal((8, 28, D)))
+    got = gpu_scores(ap, mod, np.array([0, T]), np.array([0, 8]), k, q, [300], [900], 28, 4)
+    np.testing.assert_allclose(got[mod != 0], 1.0 / 1200, rtol=2e-5)
+
+
+def test_scores_are_deterministic(ap):
+    rng = np.random.default_rng(5)
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, [5000, 3000], [64, 17], 28, 4)
+    a = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, 28, 4)
+    b = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, 28, 4)
+    assert a.tobytes() == b.tobytes()
+
+
+# ------------------------------------------------------------------------------ selection
+
+def gpu_select(ap, scores, mod, cu, counts, na, nv, mode):
+    mod_d = dev(mod)
+    seqs = ap.Seqs(cu, np.zeros(len(cu), np.int32), na, nv, mod_d, 28, 4)
+    ws = aligned_ws(ap, seqs)
+    T = int(cu[-1])
+    other = np.diff(cu) - np.asarray(na) - np.asarray(nv)
+    counts = np.asarray(counts, np.int32).reshape(-1, 2)
+    n_out = int((other + counts[:, 0] + counts[:, 1]).sum())
+    keep = torch.full((max(n_out, 1),), -7, dtype=torch.int32, device="cuda")
+    mod_o = torch.zeros(max(n_out, 1), dtype=torch.uint8, device="cuda")
+    d2s = torch.full((max(T, 1),), -7, dtype=torch.int32, device="cuda")
+    ncu = torch.zeros(len(cu), dtype=torch.int32, device="cuda")
+    ap.apack_select(seqs, dev(scores.astype(np.float32)), counts, keep, ws, select_mode=mode, modality_out=mod_o,
+                    dst_of_src=d2s, new_cu_seqlens=ncu)
+    torch.cuda.synchronize()
+    err = ap.apack_device_error(ws)
+    return (keep[:n_out].cpu().numpy(), mod_o[:n_out].cpu().numpy(), d2s[:T].cpu().numpy(), ncu.cpu().numpy(),
+            err)
+
+
+SEL_CASES = [
+    ([2000], "random"), ([1298], "ties"), ([50000, 30, 7000, 0, 1], "random"),
+    ([20000], "allequal"), ([100000], "coarse"), ([3, 5, 7, 9, 11, 13, 15, 17, 19, 21] * 7, "coarse"),
+]
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("lens,kind", SEL_CASES)
+def test_select_matches_oracle_exactly(ap, lens, kind, mode):
+    rng = np.random.default_rng(len(lens) * 7 + sum(lens) + mode)
+    mods = [rng.choice([0, 1, 2], L, p=[0.05, 0.2, 0.75]).astype(np.uint8) for L in lens]
+    mod = np.concatenate(mods)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = mod.size
+    if kind == "random":
+        sc = rng.random(T).astype(np.float32) * 1e-3
+    elif kind == "ties":
+        sc = (rng.integers(0, 20, T) / 64.0).astype(np.float32)
+    elif kind == "coarse":
+        sc = (rng.integers(0, 3000, T) * 1e-7).astype(np.float32)
+    else:
+        sc = np.full(T, 1.0 / 3.0, np.float32)
+    sc[(mod != 1) & (mod != 2)] = 0
+    na = [int((m == 1).sum()) for m in mods]
+    nv = [int((m == 2).sum()) for m in mods]
+    counts = []
+    for b, (a, v) in enumerate(zip(na, nv)):      # k = 0, k = n and in between
+        if mode == 1:
+            n = a + v
+            counts.append(([n // 3, 0, n, (2 * n) // 3][b % 4], 0))
+        else:
+            counts.append(([a // 2, 0, a, (a * 7) // 10][b % 4], [(v * 3) // 10, v, 0, v // 4][b % 4]))
+    keep, mod_o, d2s, ncu, err = gpu_select(ap, sc, mod, cu, counts, na, nv, mode)
+    assert err == ap.APACK_OK
+    ref = oracle.select_keep(sc, mod, cu, counts, joint=(mode == 1))
+    np.testing.assert_array_equal(keep, ref)
+    np.testing.assert_array_equal(mod_o, mod[ref])
+    exp_d2s = np.full(T, -1, np.int32)
+    exp_d2s[ref] = np.arange(ref.size)
+    np.testing.assert_array_equal(d2s, exp_d2s)
+    np.testing.assert_array_equal(ncu, oracle.new_cu_seqlens(ref, cu))
+
+
+def test_select_reports_count_mismatch_without_faulting(ap):
+    rng = np.random.default_rng(2)
+    mod = rng.choice([0, 1, 2], 5000).astype(np.uint8)
+    cu = np.array([0, 5000], np.int32)
+    na, nv = int((mod == 1).sum()), int((mod == 2).sum())
+    sc = rng.random(5000).astype(np.float32)
+    keep, _, _, _, err = gpu_select(ap, sc, mod, cu, [(10, 10)], [na - 1], [nv + 1], 0)
+    assert err == ap.APACK_EDEVICE
+    assert np.all(keep >= -7) and np.all(keep < 5000)
+
+
+# ------------------------------------------------------------------------------ compaction
+
+@pytest.mark.parametrize("row_bytes,planes", [(1024, 3), (512, 2), (7168, 1), (4096, 1), (16, 2), (12, 1),
+                                              (1, 1), (272, 2)])
+def test_compact_is_bitexact(ap, row_bytes, planes):
+    rng = np.random.default_rng(row_bytes)
+    T = 3001
+    src = rng.integers(0, 256, (planes, T, row_bytes), dtype=np.uint8)
+    keep = np.sort(rng.choice(T, 1237, replace=False)).astype(np.int32)
+    s = dev(src)
+    d = torch.zeros((planes, keep.size, row_bytes), dtype=torch.uint8, device="cuda")
+    p = ap.make_plane(s, d, row_bytes, planes, src_plane_stride=T * row_bytes,
+                      dst_plane_stride=keep.size * row_bytes)
+    ap.apack_compact(dev(keep), keep.size, [p])
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(d.cpu().numpy(), src[:, keep, :])
+
+
+def test_compact_many_groups_and_strided_rows(ap):
+    rng = np.random.default_rng(9)
+    T = 2000
+    keep = np.sort(rng.choice(T, 901, replace=False)).astype(np.int32)
+    kd = dev(keep)
+    groups, outs, refs = [], [], []
+    for g, rb in enumerate([1024, 2048, 512, 48]):
+        src = rng.integers(0, 256, (2, T, rb + 64), dtype=np.uint8)   # row stride > row bytes
+        s = dev(src)
+        d = torch.zeros((2, keep.size, rb), dtype=torch.uint8, device="cuda")
+        groups.append(ap.make_plane(s, d, rb, 2, src_plane_stride=T * (rb + 64), dst_plane_stride=keep.size * rb,
+                                    src_row_stride=rb + 64))
+        outs.append((s, d))
+        refs.append(src[:, keep, :rb])
+    ap.apack_compact(kd, keep.size, groups)
+    torch.cuda.synchronize()
+    for (s, d), r in zip(outs, refs):
+        np.testing.assert_array_equal(d.cpu().numpy(), r)
+
+
+def test_device_fill_matches_host_generator(ap):
+    from synth.device import fill_normal_bf16
+    from synth.gen import normal_bf16_bits
+    t = torch.empty(1 << 20, dtype=torch.int16, device="cuda")
+    fill_normal_bf16(t, 3, 2004, start=12345)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(t.cpu().numpy().view(np.uint16), normal_bf16_bits(3, 2004, 12345, 1 << 20))

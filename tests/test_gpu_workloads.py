@@ -1,0 +1,104 @@
+"""End-to-end parity of apack_prune_step on the five audio-video workloads
+(full sizes, the launch configuration the benchmark times), step by step
+through progressive schedules.
+
+Each step is checked against the oracle on the GPU's own previous-step
+result, so that a legitimate near-tie reordering in one step does not
+cascade: scores within 1e-5 + 2e-3|ref|, kept indices identical up to
+tokens within that tolerance of the k-th score, compacted K/V/hidden rows
+bit-exact given the GPU's indices (sampled layers), modality and offsets
+exact, planted tokens kept.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from parity import check_scores, check_keep
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ap():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2608_08794_gb300 as ap
+    return ap
+
+
+def host_u16(t):
+    return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+@pytest.mark.parametrize("name", ["tiny", "3b_60s", "7b_2min", "7b_10min", "7b_ragged16"])
+def test_workload_parity(ap, name):
+    from paper_2608_08794_gb300.schedule import ProgressivePrune
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+    from synth.inputs import key_slab, planted_tokens, base_counts
+
+    wl = workload(name)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod0 = wl.modality()
+    mod_d = torch.from_numpy(mod0).cuda()
+    s0 = ap.Seqs(cu0, cuq, na, nv, mod_d, wl.num_q_heads, wl.num_kv_heads)
+    counts = []
+    for i in range(len(wl.prune_layers)):
+        k_gpu, _ = ap.apack_keep_counts(s0, np.array(wl.ratios[i], np.float32))
+        k_ref = oracle.step_keep_counts(wl.ratios[i], base_counts(wl))
+        assert k_gpu.tolist() == [list(x) for x in k_ref]
+        counts.append(k_gpu)
+    pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                          wl.prune_layers, counts)
+    qs = fill_progressive_inputs(pp, wl)
+
+    composite = np.arange(wl.total_tokens)
+    mod_cur, cu_cur = mod0, cu0
+    l0 = wl.prune_layers[0]
+    exempt_total = 0
+    for i, layer in enumerate(wl.prune_layers):
+        seqs, k_in, v_in, in_stride, h_in = pp.step_args(i)
+        new_cu = pp.run_step(i)
+        torch.cuda.synchronize()
+        assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+        T_in, t_out = int(cu_cur[-1]), pp.t_out[i]
+        # scores
+        k_host = key_slab(wl, layer, qs[i])[composite]
+        ref_scores = oracle.relevance_scores(qs[i], k_host, cu_cur, cuq, mod_cur, wl.num_q_heads, wl.num_kv_heads)
+        got = pp.scores[:T_in].cpu().numpy()
+        check_scores(got, ref_scores)
+        # selection
+        ref_keep = oracle.select_keep(ref_scores, mod_cur, cu_cur, [tuple(c) for c in counts[i]])
+        keep = pp.keep_idx[i][:t_out].cpu().numpy().astype(np.int64)
+        exempt_total += check_keep(keep, ref_keep, ref_scores, mod_cur, cu_cur)
+        # the GPU's own selection is exact on its own fp32 scores
+        np.testing.assert_array_equal(keep, oracle.select_keep(got, mod_cur, cu_cur, [tuple(c) for c in counts[i]]))
+        np.testing.assert_array_equal(new_cu, oracle.new_cu_seqlens(keep, cu_cur))
+        np.testing.assert_array_equal(pp.mod_out[i % 2][:t_out].cpu().numpy(), mod_cur[keep])
+        # compaction, bit-exact given the GPU's indices, on sampled layers
+        k_out, v_out = pp.output_kv(i)
+        n_l = wl.num_layers - layer
+        row_elems = wl.num_kv_heads * wl.head_dim
+        keep_t = torch.from_numpy(keep).cuda()
+        for j in sorted({0, n_l // 2, n_l - 1}):
+            src_k = k_in[j * T_in * row_elems:(j + 1) * T_in * row_elems].view(T_in, row_elems)
+            src_v = v_in[j * T_in * row_elems:(j + 1) * T_in * row_elems].view(T_in, row_elems)
+            assert torch.equal(k_out[j].reshape(t_out, row_elems).view(torch.int16),
+                               src_k.index_select(0, keep_t).view(torch.int16))
+            assert torch.equal(v_out[j].reshape(t_out, row_elems).view(torch.int16),
+                               src_v.index_select(0, keep_t).view(torch.int16))
+        if i == 0:
+            # slab 0 of the first input is the planted key cache the host generator defines
+            np.testing.assert_array_equal(host_u16(k_out[0]).reshape(t_out, -1), k_host.reshape(T_in, -1)[keep])
+        h_out = pp.output_hidden(i)
+        assert torch.equal(h_out.view(torch.int16), h_in[:T_in].index_select(0, keep_t).view(torch.int16))
+        composite = composite[keep]
+        mod_cur = mod_cur[keep]
+        cu_cur = new_cu
+    tok, _ = planted_tokens(wl)
+    assert np.isin(tok, composite).all(), "a planted token was dropped"
+    print(f"{name}: tie-exempt tokens {exempt_total}")
