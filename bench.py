@@ -1,0 +1,414 @@
+"""Benchmark of the A-PACK inner-LLM prune step on GB300.
+
+One benchmark step is one pass of the whole hot path over the workload: the
+progressive schedule of the 7B-shaped 10-minute audio-video sequence
+(135,272 tokens, 15,000 audio + 120,000 visual, 256 query rows, Hq 28 /
+Hkv 4, pruning at layers 4, 12 and 20 of 28), i.e. three apack_prune_step
+calls, each scoring, selecting and compacting K/V of all later layers and
+the hidden states.  The metric is multimodal tokens entering the prune steps
+per second (sum over steps of |S| / time).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Multi-GPU (torchrun): every rank runs its own copy of the workload (the step
+shards by independent sequences; there is no data-path collective), the
+barrier and max-over-ranks timing use torch.distributed, value = units of
+all ranks / time (weak scaling).  ``--impl reference`` times the CPU oracle
+on a bounded sample of the same workload (rank 0 only).
+"""
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "prune-step multimodal tokens/s; KV-compaction HBM GB/s vs peak (7B-shaped)"
+UNIT = "multimodal tokens/s"
+WORKLOAD = "7b_10min"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default=WORKLOAD)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--e2e-steps", type=int, default=None)
+    return p.parse_args()
+
+
+# ----------------------------------------------------------------------------- helpers
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d.get("hbm_gbs", FALLBACK_HBM_GBS)), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def profiled_traffic(kernel_src):
+    """DRAM bytes per launch of the compaction kernel from the committed ncu
+    summary, if it was taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "gather_wide_traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    src = open(os.path.join(ROOT, "paper_2608_08794_gb300", "csrc", kernel_src), "rb").read()
+    if d.get("source_sha256") != hashlib.sha256(src).hexdigest():
+        return None
+    return d
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 100 ms."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.samples = []
+        self.proc = None
+        self.marks = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), line.strip()))
+
+    def mark(self, on):
+        self.marks.append((time.time(), on))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        spans, t0 = [], None
+        for t, on in self.marks:
+            if on:
+                t0 = t
+            elif t0 is not None:
+                spans.append((t0, t))
+                t0 = None
+        mhz, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for t, line in self.samples:
+            if not any(a - 0.05 <= t <= b + 0.05 for a, b in spans):
+                continue
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                mhz.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not mhz:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": 0}
+        mhz.sort()
+        return {"sm_mhz": mhz[len(mhz) // 2], "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(mhz)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle leg
+
+ORACLE_SNIPPET = r"""
+import json, sys, time
+sys.path.insert(0, {root!r})
+import numpy as np
+import oracle
+from synth import workload
+from synth.configs import scaled_copy
+from synth.inputs import query_rows, key_slab, value_slab, plain_key_slab, hidden_states, base_counts
+wl = scaled_copy(workload({name!r}), {dur})
+cu, cuq, mod = wl.cu_seqlens(), wl.cu_qlens(), wl.modality()
+L, l0 = wl.num_layers, wl.prune_layers[0]
+qs = [query_rows(wl, l) for l in wl.prune_layers]
+ks = [key_slab(wl, l, q) for l, q in zip(wl.prune_layers, qs)]
+# bulk K/V planes: one drawn layer repeated over the compacted layers (values do not change the copy cost)
+kv = [np.repeat(plain_key_slab(wl, l0)[None], L - l0, axis=0), np.repeat(value_slab(wl, l0)[None], L - l0, axis=0)]
+hid = hidden_states(wl)
+counts = [oracle.step_keep_counts(r, base_counts(wl)) for r in wl.ratios]
+def one():
+    comp = np.arange(wl.total_tokens); c, m = cu, mod
+    kk, vv, hh = kv[0], kv[1], hid
+    mm = 0
+    for i, layer in enumerate(wl.prune_layers):
+        mm += int(((m == 1) | (m == 2)).sum())
+        j = layer - l0 if i == 0 else layer - wl.prune_layers[i - 1]
+        out = oracle.prune_step(qs[i], ks[i][comp], c, cuq, m, wl.num_q_heads, wl.num_kv_heads, counts[i],
+                                planes=[kk[j:].transpose(1, 0, 2, 3), vv[j:].transpose(1, 0, 2, 3), hh])
+        keep = out["keep_idx"]
+        kk = out["planes"][0].transpose(1, 0, 2, 3); vv = out["planes"][1].transpose(1, 0, 2, 3); hh = out["planes"][2]
+        comp, c, m = comp[keep], out["cu_seqlens"], out["modality"]
+    return mm
+reps = {reps}
+times, mm = [], 0
+for r in range(reps):
+    t0 = time.perf_counter(); mm = one(); times.append(time.perf_counter() - t0)
+print(json.dumps(dict(times=times, mm=mm, tokens=wl.total_tokens, dur={dur})))
+"""
+
+
+def run_oracle(name, dur, reps):
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = ORACLE_SNIPPET.format(root=ROOT, name=name, dur=dur, reps=reps)
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env)
+    if r.returncode != 0:
+        raise RuntimeError(r.stderr[-2000:])
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def cpu_sample_duration(name, budget_s, max_dur=120):
+    """Clip length (even seconds) whose oracle schedule takes about budget_s."""
+    probe = run_oracle(name, 10, 1)
+    per_s = probe["times"][0] / 10.0
+    dur = int(max(2, min(max_dur, budget_s / max(per_s, 1e-6))))
+    return max(2, dur - dur % 2)
+
+
+def cpu_baseline(name, budget_s=15.0):
+    dur = cpu_sample_duration(name, budget_s)
+    d = run_oracle(name, dur, 1)
+    v = d["mm"] / d["times"][0]
+    return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"first {dur} s of the {name} sequence ({d['tokens']} tokens), same heads, query rows and "
+                      f"3-step schedule, single-threaded numpy fp64 oracle, {d['times'][0]:.1f} s"}
+
+
+def reference_arm(args, rank, world):
+    if rank != 0:
+        return
+    per_step = min(10.0, 120.0 / max(1, args.steps + args.warmup))
+    dur = cpu_sample_duration(args.workload, per_step)
+    d = run_oracle(args.workload, dur, args.warmup + args.steps)
+    times = d["times"][args.warmup:]
+    t = sum(times)
+    v = d["mm"] * len(times) / t
+    sample = (f"first {dur} s of the {args.workload} sequence ({d['tokens']} tokens) per step, same heads, query "
+              f"rows and 3-step schedule, single-threaded numpy fp64 oracle")
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * t / len(times), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "sample_seconds": dur},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- GPU leg
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        reference_arm(args, rank, world)
+        return
+
+    import numpy as np
+    import torch
+    import paper_2608_08794_gb300 as ap
+    from paper_2608_08794_gb300.schedule import ProgressivePrune
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    wl = workload(args.workload)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod_tmp = torch.from_numpy(wl.modality()).cuda()
+    s0 = ap.Seqs(cu0, cuq, na, nv, mod_tmp, wl.num_q_heads, wl.num_kv_heads)
+    counts = [ap.apack_keep_counts(s0, np.array(r, np.float32))[0] for r in wl.ratios]
+    pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                          wl.prune_layers, counts)
+    fill_progressive_inputs(pp, wl)
+    mm_per_iter = sum(pp.mm_tokens_per_step())
+    nsteps = len(wl.prune_layers)
+    stream = torch.cuda.current_stream()
+
+    # algorithmic bytes of the compaction launch of each prune step
+    row = wl.num_kv_heads * wl.head_dim * 2
+    comp_bytes = [2 * t * (2 * (wl.num_layers - l) * row + wl.hidden * 2) + 4 * t
+                  for t, l in zip(pp.t_out, wl.prune_layers)]
+
+    for _ in range(args.warmup):
+        pp.run(stream=stream)
+    torch.cuda.synchronize()
+
+    # timed region: K steps, stage events on the launching stream
+    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(nsteps)]
+          for _ in range(args.steps)]
+    for per_iter in ev:       # torch creates events on first record; the C ABI records raw handles
+        for per_step in per_iter:
+            for e in per_step:
+                e.record(stream)
+    torch.cuda.synchronize()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local) if rank == 0 else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    launches0 = ap.apack_launch_count()
+    barrier()
+    if clocks:
+        clocks.mark(True)
+    t_start.record(stream)
+    for k in range(args.steps):
+        pp.run(events=ev[k], stream=stream)
+    t_end.record(stream)
+    barrier()
+    if clocks:
+        clocks.mark(False)
+    launches = ap.apack_launch_count() - launches0
+    ms = t_start.elapsed_time(t_end)
+    if dist is not None:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    stage_ms = np.zeros((nsteps, 3))
+    for k in range(args.steps):
+        for i in range(nsteps):
+            for s in range(3):
+                stage_ms[i, s] += ev[k][i][s].elapsed_time(ev[k][i][s + 1])
+    stage_ms /= args.steps
+
+    # end to end through the C ABI with host buffers: H2D of the step's inputs
+    # from pinned memory, the three prune steps, D2H of the result
+    e2e_steps = args.e2e_steps or max(3, min(args.steps, 20))
+    h_k = torch.empty(pp.k_in.shape, dtype=pp.k_in.dtype, pin_memory=True)
+    h_v = torch.empty_like(h_k, pin_memory=True)
+    h_h = torch.empty(pp.hidden_in.shape, dtype=pp.hidden_in.dtype, pin_memory=True)
+    h_m = torch.empty(pp.modality_in.shape, dtype=torch.uint8, pin_memory=True)
+    h_q = [torch.empty(q.shape, dtype=q.dtype, pin_memory=True) for q in pp.q]
+    h_k.copy_(pp.k_in); h_v.copy_(pp.v_in); h_h.copy_(pp.hidden_in); h_m.copy_(pp.modality_in)
+    for a, b in zip(h_q, pp.q):
+        a.copy_(b)
+    last = nsteps - 1
+    ko, vo = pp.output_kv(last)
+    ho = pp.output_hidden(last)
+    o_k = torch.empty(ko.shape, dtype=ko.dtype, pin_memory=True)
+    o_v = torch.empty_like(o_k, pin_memory=True)
+    o_h = torch.empty(ho.shape, dtype=ho.dtype, pin_memory=True)
+    o_i = [torch.empty(int(t), dtype=torch.int32, pin_memory=True) for t in pp.t_out]
+    h2d = sum(x.numel() * x.element_size() for x in [h_k, h_v, h_h, h_m] + h_q)
+    d2h = sum(x.numel() * x.element_size() for x in [o_k, o_v, o_h] + o_i)
+
+    def e2e_step():
+        pp.k_in.copy_(h_k, non_blocking=True); pp.v_in.copy_(h_v, non_blocking=True)
+        pp.hidden_in.copy_(h_h, non_blocking=True); pp.modality_in.copy_(h_m, non_blocking=True)
+        for a, b in zip(pp.q, h_q):
+            a.copy_(b, non_blocking=True)
+        pp.run(stream=stream)
+        o_k.copy_(ko, non_blocking=True); o_v.copy_(vo, non_blocking=True); o_h.copy_(ho, non_blocking=True)
+        for i, t in enumerate(pp.t_out):
+            o_i[i].copy_(pp.keep_idx[i][:t], non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    barrier()
+    if clocks:
+        clocks.mark(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    barrier()
+    if clocks:
+        clocks.mark(False)
+        clocks.stop()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    if dist is not None:
+        t = torch.tensor([e2e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+
+    if rank == 0:
+        per_step_ms = ms / args.steps
+        value = world * mm_per_iter / (per_step_ms / 1e3)
+        peak, peak_kind = measured_peaks()
+        comp_ms = stage_ms[:, 2]
+        achieved = sum(comp_bytes) / (comp_ms.sum() / 1e3) / 1e9
+        prof = profiled_traffic("compact.cu")
+        traffic = None
+        if prof is not None:
+            traffic = prof.get("dram_bytes_per_launch")
+        score_ms, select_ms = stage_ms[:, 0].sum(), stage_ms[:, 1].sum()
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": per_step_ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": args.workload, "tokens": wl.total_tokens, "mm_tokens": wl.total_mm,
+                       "query_rows": int(cuq[-1]), "heads": f"{wl.num_q_heads}q/{wl.num_kv_heads}kv",
+                       "hidden": wl.hidden, "num_layers": wl.num_layers, "prune_layers": wl.prune_layers,
+                       "tokens_after_steps": pp.t_out, "mm_tokens_per_iter": mm_per_iter,
+                       "l2": "inputs larger than L2 (K/V of the compacted layers: %.1f GB)" %
+                             (2 * pp.k_in.numel() * 2 / 1e9),
+                       "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
+            "gpu_launches": int(launches),
+            "roofline": {"bound": "hbm", "kernel": "gather_wide_kernel (compaction)", "achieved": achieved,
+                         "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": traffic, "peak_source": peak_kind,
+                         "algorithmic_bytes_per_launch": comp_bytes,
+                         "avg_launch_ms": [float(x) for x in comp_ms]},
+            "stages_ms_per_iter": {"score": float(score_ms), "select": float(select_ms),
+                                   "compact": float(comp_ms.sum())},
+            "e2e": {"value": world * mm_per_iter / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+                    "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps},
+            "clocks": clocks.summary() if clocks else None,
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            try:
+                line["cpu_baseline"] = cpu_baseline(args.workload)
+            except Exception as exc:  # report, do not hide
+                line["cpu_baseline"] = {"value": None, "error": str(exc)[-300:]}
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -204,7 +204,10 @@ def apack_prune_step(seqs, layer, num_layers, q, k_cache, v_cache, kv_layer_stri
     arr = (apack_plane * max(1, len(extra_planes)))(*extra_planes)
     ev = None
     if stage_events is not None:
-        ev = (ctypes.c_void_p * 4)(*[e.cuda_event if hasattr(e, "cuda_event") else e for e in stage_events])
+        handles = [e.cuda_event if hasattr(e, "cuda_event") else e for e in stage_events]
+        if len(handles) != 4 or not all(handles):
+            raise ValueError("stage_events: four created CUDA events (record a torch event once to create it)")
+        ev = (ctypes.c_void_p * 4)(*handles)
     st = _lib.apack_prune_step(
         seqs.ref(), int(layer), int(num_layers), _ptr(q), _ptr(k_cache), _ptr(v_cache), int(kv_layer_stride),
         _ptr(hidden), int(hidden_dim),
