@@ -53,11 +53,11 @@ WsLayout workspace_layout(const apack_seqs *s) {
   WsLayout L{};
   const int64_t NQ = s->cu_qlens_h[s->num_seqs];
   const int G = s->num_q_heads / s->num_kv_heads;
-  const int r2 = rows_tile2(G);
+  const int r1 = rows_tile1(G);
   int64_t chunks = 0;
   for (int b = 0; b < s->num_seqs; ++b) {
     const int64_t nq = s->cu_qlens_h[b + 1] - s->cu_qlens_h[b];
-    chunks += static_cast<int64_t>(s->num_kv_heads) * ((nq + r2 - 1) / r2);
+    chunks += static_cast<int64_t>(s->num_kv_heads) * ((nq + r1 - 1) / r1);
   }
   auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
   L.err_off = 0;
@@ -65,7 +65,7 @@ WsLayout workspace_layout(const apack_seqs *s) {
   const size_t part_bytes = static_cast<size_t>(kMaxSplits) * NQ * s->num_q_heads * sizeof(float2);
   L.lse_off = up(L.part_off + part_bytes);
   L.lse_chunks = chunks;
-  L.total = up(L.lse_off + static_cast<size_t>(chunks) * 256 * sizeof(float));
+  L.total = up(L.lse_off + static_cast<size_t>(chunks) * 128 * sizeof(float));
   return L;
 }
 

@@ -37,14 +37,14 @@ __device__ __forceinline__ void raise_device_error(DeviceError *e, int32_t code,
 struct WsLayout {
   size_t err_off;     // DeviceError
   size_t part_off;    // float2 [kMaxSplits][sum n_q][Hq]: per-split (max, sum) in log2 units
-  size_t lse_off;     // float [chunks][256]: log2 normalisers per query-row chunk, +inf padding
+  size_t lse_off;     // float [chunks][128]: negated log2 normalisers per 128-row query chunk, -inf padding
   size_t total;
   int64_t lse_chunks;
 };
 
 // Query tokens per MMA tile: rows of a tile are (token, head-in-group) pairs.
-__host__ __device__ inline int rows_tile1(int group) { return 128 / group; }   // row-stats pass (M = 128)
-__host__ __device__ inline int rows_tile2(int group) { return 256 / group; }   // column pass (N = 256)
+__host__ __device__ inline int rows_tile1(int group) { return 128 / group; }   // one 128-row tile
+__host__ __device__ inline int rows_tile2(int group) { return 256 / group; }   // a pair of tiles (256 rows)
 
 WsLayout workspace_layout(const apack_seqs *seqs);
 int device_sm_count();

@@ -162,6 +162,14 @@ def _build() -> dict:
         ratios=[[(0.7, 0.4)], [(0.5, 0.25)], [(0.3, 0.15)]],
         plants=[[Plant(1, 750, 1.0), Plant(2, 6000, 1.0),
                  Plant(1, 15, 3.0), Plant(2, 120, 3.0)]])
+    # 4 on one layer: the 10-minute sequence pruned once at the last layer (one
+    # compacted K/V layer); same scoring and selection work as the first step of
+    # 7b_10min with a device footprint of about 2 GB (profiling captures).
+    w["7b_10min_1l"] = Workload(
+        name="7b_10min_1l", seed=3, **_qwen7b(), seqs=[s4], prune_layers=[27],
+        ratios=[[(0.7, 0.4)]],
+        plants=[[Plant(1, 750, 1.0), Plant(2, 6000, 1.0),
+                 Plant(1, 15, 3.0), Plant(2, 120, 3.0)]])
     # 5: ragged batch of 16 7B-shaped sequences, prune at layer 8.
     seqs5, r5 = _ragged_seqs(4, 16)
     w["7b_ragged16"] = Workload(
