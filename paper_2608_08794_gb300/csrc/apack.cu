@@ -52,20 +52,24 @@ apack_status validate_seqs(const apack_seqs *s, int64_t *total_tokens, int64_t *
 WsLayout workspace_layout(const apack_seqs *s) {
   WsLayout L{};
   const int64_t NQ = s->cu_qlens_h[s->num_seqs];
+  const int64_t T = s->cu_seqlens_h[s->num_seqs];
   const int G = s->num_q_heads / s->num_kv_heads;
-  const int r1 = rows_tile1(G);
-  int64_t chunks = 0;
+  int64_t chunks = 0, qp_rows = 0;
   for (int b = 0; b < s->num_seqs; ++b) {
-    const int64_t nq = s->cu_qlens_h[b + 1] - s->cu_qlens_h[b];
-    chunks += static_cast<int64_t>(s->num_kv_heads) * ((nq + r1 - 1) / r1);
+    const int64_t rows = static_cast<int64_t>(G) * (s->cu_qlens_h[b + 1] - s->cu_qlens_h[b]);
+    chunks += static_cast<int64_t>(s->num_kv_heads) * ((rows + 127) / 128);
+    qp_rows += static_cast<int64_t>(s->num_kv_heads) * ((rows + 255) / 256) * 256;
   }
-  auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
+  auto up = [](size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); };
   L.err_off = 0;
-  L.part_off = 256;
+  L.part_off = 1024;
   const size_t part_bytes = static_cast<size_t>(kMaxSplits) * NQ * s->num_q_heads * sizeof(float2);
   L.lse_off = up(L.part_off + part_bytes);
   L.lse_chunks = chunks;
-  L.total = up(L.lse_off + static_cast<size_t>(chunks) * 128 * sizeof(float));
+  L.qp_off = up(L.lse_off + static_cast<size_t>(chunks) * 128 * sizeof(float));
+  L.qp_rows = qp_rows;
+  L.gsum_off = up(L.qp_off + static_cast<size_t>(qp_rows) * 256);
+  L.total = up(L.gsum_off + static_cast<size_t>(s->num_kv_heads) * T * sizeof(float));
   return L;
 }
 

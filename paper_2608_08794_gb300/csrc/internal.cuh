@@ -38,13 +38,13 @@ struct WsLayout {
   size_t err_off;     // DeviceError
   size_t part_off;    // float2 [kMaxSplits][sum n_q][Hq]: per-split (max, sum) in log2 units
   size_t lse_off;     // float [chunks][128]: negated log2 normalisers per 128-row query chunk, -inf padding
+  size_t qp_off;      // bf16 [qp_rows][128]: query rows repacked per KV head group, 256-row padded
+  size_t gsum_off;    // float [Hkv][T]: per head group key sums of the column pass
   size_t total;
   int64_t lse_chunks;
+  int64_t qp_rows;
 };
 
-// Query tokens per MMA tile: rows of a tile are (token, head-in-group) pairs.
-__host__ __device__ inline int rows_tile1(int group) { return 128 / group; }   // one 128-row tile
-__host__ __device__ inline int rows_tile2(int group) { return 256 / group; }   // a pair of tiles (256 rows)
 
 WsLayout workspace_layout(const apack_seqs *seqs);
 int device_sm_count();
