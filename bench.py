@@ -61,7 +61,7 @@ def measured_peaks():
 def profiled_traffic(kernel_src):
     """DRAM bytes per launch of the compaction kernel from the committed ncu
     summary, if it was taken on the current kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", "gather_wide_traffic.json")
+    path = os.path.join(ROOT, "profiles", "gather_tma_traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
@@ -389,7 +389,7 @@ def main():
                              (2 * pp.k_in.numel() * 2 / 1e9),
                        "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
             "gpu_launches": int(launches),
-            "roofline": {"bound": "hbm", "kernel": "gather_wide_kernel (compaction)", "achieved": achieved,
+            "roofline": {"bound": "hbm", "kernel": "gather_tma_kernel (compaction)", "achieved": achieved,
                          "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                          "traffic": traffic, "peak_source": peak_kind,
                          "algorithmic_bytes_per_launch": comp_bytes,

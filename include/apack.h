@@ -133,9 +133,11 @@ apack_status apack_select(const apack_seqs *seqs, const float *scores, const int
    "slice their KV-cache entries"): for every plane of every group,
    dst row j = src row keep_idx[j], j < n_out, bit for bit.
    planes_h: host array of num_groups descriptors.  Out of place only in this
-   build (src == dst returns APACK_EUNSUPPORTED). */
+   build (src == dst returns APACK_EUNSUPPORTED).
+   ws: NULL, or a 256-byte aligned workspace (e.g. the one of apack_score)
+   whose error word receives APACK_ETIMEOUT if a bounded wait gives up. */
 apack_status apack_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes_h,
-                           int32_t num_groups, void *stream);
+                           int32_t num_groups, void *ws, void *stream);
 
 /* One pruning step at layer `layer` of a num_layers-layer decoder
    (Algorithm 1, one iteration of the inner-LLM loop): apack_score on the

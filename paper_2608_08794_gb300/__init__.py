@@ -64,7 +64,7 @@ def _load():
     lib.apack_keep_counts.argtypes = [P(apack_seqs), P(ctypes.c_float), I32, PI32, PI32]
     lib.apack_score.argtypes = [P(apack_seqs), VP, VP, I64, VP, VP, SZ, VP]
     lib.apack_select.argtypes = [P(apack_seqs), VP, PI32, I32, VP, VP, VP, VP, VP, SZ, VP]
-    lib.apack_compact.argtypes = [VP, I64, P(apack_plane), I32, VP]
+    lib.apack_compact.argtypes = [VP, I64, P(apack_plane), I32, VP, VP]
     lib.apack_prune_step.argtypes = [P(apack_seqs), I32, I32, VP, VP, VP, I64, VP, I64, P(ctypes.c_float), PI32,
                                      I32, VP, VP, I64, VP, P(apack_plane), I32, VP, VP, PI32, VP, VP, VP, SZ,
                                      P(VP), VP]
@@ -184,9 +184,10 @@ def make_plane(src, dst, row_bytes, num_planes=1, src_plane_stride=0, dst_plane_
                        row_bytes=row_bytes, num_planes=num_planes, reserved=0)
 
 
-def apack_compact(keep_idx, n_out, planes, stream=None):
+def apack_compact(keep_idx, n_out, planes, ws=None, stream=None):
     arr = (apack_plane * max(1, len(planes)))(*planes)
-    _check(_lib.apack_compact(_ptr(keep_idx), int(n_out), arr, len(planes), _stream(stream)), "apack_compact")
+    _check(_lib.apack_compact(_ptr(keep_idx), int(n_out), arr, len(planes), _ptr(ws), _stream(stream)),
+           "apack_compact")
 
 
 def apack_prune_step(seqs, layer, num_layers, q, k_cache, v_cache, kv_layer_stride, hidden, hidden_dim,

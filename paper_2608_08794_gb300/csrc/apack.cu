@@ -180,8 +180,10 @@ apack_status apack_select(const apack_seqs *seqs, const float *scores, const int
 }
 
 apack_status apack_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes_h, int32_t num_groups,
-                           void *stream) {
-  return run_compact(keep_idx, n_out, planes_h, num_groups, static_cast<cudaStream_t>(stream));
+                           void *ws, void *stream) {
+  if (ws && (reinterpret_cast<uintptr_t>(ws) & 255)) return APACK_EINVAL;
+  return run_compact(keep_idx, n_out, planes_h, num_groups, static_cast<DeviceError *>(ws),
+                     static_cast<cudaStream_t>(stream));
 }
 
 apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num_layers, const void *q,
@@ -244,7 +246,8 @@ apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num
     planes.push_back(hp);
   }
   for (int i = 0; i < num_extra; ++i) planes.push_back(extra_planes_h[i]);
-  st = run_compact(keep_idx, n_out, planes.data(), static_cast<int32_t>(planes.size()), s);
+  st = run_compact(keep_idx, n_out, planes.data(), static_cast<int32_t>(planes.size()),
+                   reinterpret_cast<DeviceError *>(static_cast<uint8_t *>(ws) + workspace_layout(seqs).err_off), s);
   if (st != APACK_OK) return st;
   mark(3);
   return APACK_OK;

@@ -1,83 +1,129 @@
 // compact.cu -- KV-cache and hidden-state slicing of Sec. 3.2 (Algorithm 1, "slice their
 // KV-cache entries"): dst row j = src row keep_idx[j] for every plane.
 //
-// HBM-bound: every byte is read once and written once.  The wide kernel moves
-// rows in 512-byte pieces (one 16-byte vector per lane of a warp), with
-// kUnroll pieces in flight per warp before any store; loads bypass L1 and
-// stores are marked streaming so that the copy does not evict the L2 working
-// set.  Rows that are not 16-byte multiples (or misaligned) take the narrow
-// kernel, one thread per row.
+// HBM-bound: every byte is read once and written once.
+//  - TMA kernel (rows of 16-byte multiples up to 32 KB, 16-byte aligned): one
+//    warp per CTA streams kept rows into a ring of 32 KB shared-memory slots
+//    with cp.async.bulk (one row per lane, completion on the slot's mbarrier)
+//    and writes each slot back with a single bulk store when the output rows
+//    are contiguous (one per row otherwise).  Several slots stay in flight per
+//    CTA, so a handful of threads keep the whole HBM pipe busy.
+//  - Rows that are not 16-byte multiples (or misaligned) take the narrow
+//    kernel, one thread per row.
 #include "internal.cuh"
+#include "ptx.cuh"
 
 namespace apack {
 
 namespace {
 
 constexpr int kMaxGroups = 16;
-constexpr int kWideThreads = 256;
-constexpr int kUnroll = 4;
+constexpr int kSlots = 3;                       // slots per CTA (two CTAs per SM)
+constexpr uint32_t kSlotBytes = 32768;
+constexpr uint32_t kTmaSmem = kSlots * kSlotBytes;
 
-struct WideGroup {
+struct TmaGroup {
   const uint8_t *src;
   uint8_t *dst;
   int64_t sps, dps, srs, drs;   // plane and row strides in bytes
-  uint32_t vecs;                // 16-byte vectors per row
-  uint32_t pieces;              // 512-byte pieces per row = ceil(vecs / 32)
-  uint32_t n_planes;
-  uint32_t item_begin;          // first piece index of this group
+  uint32_t row_bytes;
+  uint32_t rows_per_slot;
+  uint32_t chunks_per_plane;    // ceil(n_out / rows_per_slot)
+  uint32_t item_begin;          // first slot-sized item of this group
+  uint32_t contiguous;          // output rows are back to back (one bulk store per slot)
+  uint32_t pad;
 };
 
-struct WidePlan {
+struct TmaPlan {
   int32_t ngroups;
   uint32_t total_items;
   uint32_t n_out;
-  WideGroup g[kMaxGroups];
+  TmaGroup g[kMaxGroups];
 };
 
-__device__ __forceinline__ uint4 ld_stream(const void *p) {
-  uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
+struct Item {
+  const TmaGroup *grp;
+  uint32_t plane, r0, nrows;
+};
+
+__device__ __forceinline__ Item decode_item(const TmaPlan &p, uint32_t item) {
+  int gi = 0;
+  while (gi + 1 < p.ngroups && p.g[gi + 1].item_begin <= item) ++gi;
+  const TmaGroup &G = p.g[gi];
+  const uint32_t local = item - G.item_begin;
+  Item it;
+  it.grp = &G;
+  it.plane = local / G.chunks_per_plane;
+  it.r0 = (local - it.plane * G.chunks_per_plane) * G.rows_per_slot;
+  it.nrows = min(G.rows_per_slot, p.n_out - it.r0);
+  return it;
 }
 
-__device__ __forceinline__ void st_stream(void *p, uint4 v) {
-  asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-               : "memory");
-}
-
-__global__ void __launch_bounds__(kWideThreads)
-    gather_wide_kernel(const __grid_constant__ WidePlan plan, const int32_t *__restrict__ keep_idx) {
-  const int lane = threadIdx.x & 31;
-  const uint32_t warp = (blockIdx.x * kWideThreads + threadIdx.x) >> 5;
-  const uint32_t nwarps = (gridDim.x * kWideThreads) >> 5;
-  for (uint32_t batch = warp; batch * kUnroll < plan.total_items; batch += nwarps) {
-    uint4 v[kUnroll];
-    uint8_t *dptr[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      dptr[u] = nullptr;
-      const uint32_t item = batch * kUnroll + u;
-      if (item >= plan.total_items) continue;
-      int gi = 0;
-      while (gi + 1 < plan.ngroups && plan.g[gi + 1].item_begin <= item) ++gi;
-      const WideGroup &G = plan.g[gi];
-      const uint32_t local = item - G.item_begin;
-      const uint32_t rowplane = local / G.pieces;
-      const uint32_t piece = local - rowplane * G.pieces;
-      const uint32_t plane = rowplane / plan.n_out;
-      const uint32_t row = rowplane - plane * plan.n_out;
-      const uint32_t vec = piece * 32 + lane;
-      if (vec >= G.vecs) continue;
-      const int64_t src_row = keep_idx[row];
-      v[u] = ld_stream(G.src + plane * G.sps + src_row * G.srs + vec * 16ull);
-      dptr[u] = G.dst + plane * G.dps + static_cast<int64_t>(row) * G.drs + vec * 16ull;
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u)
-      if (dptr[u]) st_stream(dptr[u], v[u]);
+// Loads the kept rows of one item into a slot (all lanes take part).
+__device__ __forceinline__ void load_item(const Item &it, uint8_t *slot, uint64_t *bar,
+                                          const int32_t *__restrict__ keep_idx, int lane) {
+  const TmaGroup &G = *it.grp;
+  if (lane == 0) mbar_arrive_expect_tx(bar, it.nrows * G.row_bytes);
+  __syncwarp();
+  const uint8_t *src = G.src + static_cast<int64_t>(it.plane) * G.sps;
+  for (uint32_t r = lane; r < it.nrows; r += 32) {
+    const int64_t srow = keep_idx[it.r0 + r];
+    bulk_load(slot + r * G.row_bytes, src + srow * G.srs, G.row_bytes, bar);
   }
+}
+
+// Stores a full slot to the output rows of its item; every lane commits its group.
+__device__ __forceinline__ void store_item(const Item &it, const uint8_t *slot, int lane) {
+  const TmaGroup &G = *it.grp;
+  uint8_t *dst = G.dst + static_cast<int64_t>(it.plane) * G.dps + static_cast<int64_t>(it.r0) * G.drs;
+  if (G.contiguous) {
+    if (lane == 0) bulk_store(dst, slot, it.nrows * G.row_bytes);
+  } else {
+    for (uint32_t r = lane; r < it.nrows; r += 32) bulk_store(dst + r * G.drs, slot + r * G.row_bytes, G.row_bytes);
+  }
+  bulk_commit();
+}
+
+__global__ void __launch_bounds__(32) gather_tma_kernel(const __grid_constant__ TmaPlan plan,
+                                                        const int32_t *__restrict__ keep_idx, DeviceError *err) {
+  extern __shared__ __align__(1024) uint8_t slots[];
+  __shared__ __align__(8) uint64_t full[kSlots];
+  const int lane = threadIdx.x;
+  if (lane == 0) {
+    for (int i = 0; i < kSlots; ++i) mbar_init(&full[i], 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  // this CTA's items: blockIdx.x, blockIdx.x + gridDim.x, ...
+  const uint32_t first = blockIdx.x, stride = gridDim.x;
+  const uint32_t n_mine = first < plan.total_items ? (plan.total_items - first + stride - 1) / stride : 0;
+  for (uint32_t j = 0; j < n_mine && j < kSlots; ++j)
+    load_item(decode_item(plan, first + j * stride), slots + j * kSlotBytes, &full[j], keep_idx, lane);
+  bool ok = true;
+  uint32_t j = 0;
+  for (; j < n_mine; ++j) {
+    const int slot = j % kSlots;
+    const Item it = decode_item(plan, first + j * stride);
+    if (!mbar_wait(&full[slot], (j / kSlots) & 1u, kWaitLimitNs)) {
+      if (lane == 0 && err) raise_device_error(err, APACK_ETIMEOUT, 41);
+      ok = false;
+      break;
+    }
+    fence_proxy_async_smem();
+    store_item(it, slots + slot * kSlotBytes, lane);
+    // refill the slot whose store was issued one item ago, once that store has read it
+    if (j >= 1 && j - 1 + kSlots < n_mine) {
+      bulk_wait_read<1>();
+      const uint32_t k = j - 1 + kSlots;
+      const int ks = k % kSlots;
+      load_item(decode_item(plan, first + k * stride), slots + ks * kSlotBytes, &full[ks], keep_idx, lane);
+    }
+  }
+  if (!ok) {
+    // loads of items j .. j+kSlots-1 may still be in flight: wait for them (bounded)
+    for (uint32_t k = j; k < n_mine && k < j + kSlots; ++k) mbar_wait(&full[k % kSlots], (k / kSlots) & 1u, kWaitLimitNs / 4);
+  }
+  bulk_wait_all();
 }
 
 // One thread per (plane, row); copies with the widest access the row allows.
@@ -132,14 +178,16 @@ bool ranges_overlap(const apack_plane &p, int64_t n_rows_src, int64_t n_out) {
 }  // namespace
 
 apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes, int32_t num_groups,
-                         cudaStream_t stream) {
+                         DeviceError *err, cudaStream_t stream) {
   if (n_out < 0 || num_groups < 0 || (num_groups > 0 && !planes)) return APACK_EINVAL;
   if (n_out == 0 || num_groups == 0) return APACK_OK;
   if (!keep_idx || n_out > INT32_MAX) return APACK_EINVAL;
-  WidePlan wp{};
-  wp.n_out = static_cast<uint32_t>(n_out);
+  // validate and plan every group before anything touches the device
+  TmaPlan tp{};
+  tp.n_out = static_cast<uint32_t>(n_out);
   uint64_t items = 0;
-  const int sms = device_sm_count();
+  int narrow[kMaxGroups * 4];
+  int n_narrow = 0;
   for (int i = 0; i < num_groups; ++i) {
     const apack_plane &p = planes[i];
     if (p.num_planes < 0 || p.row_bytes < 0) return APACK_EINVAL;
@@ -149,40 +197,49 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
       return APACK_EINVAL;
     if (p.src == p.dst) return APACK_EUNSUPPORTED;   // in-place compaction is not offered by this build
     if (ranges_overlap(p, n_out, n_out)) return APACK_EINVAL;
-    const int unit = widest_unit(p);
-    if (unit == 16 && p.row_bytes >= 256) {
-      if (wp.ngroups == kMaxGroups) return APACK_EINVAL;
-      WideGroup &g = wp.g[wp.ngroups++];
+    if (widest_unit(p) == 16 && p.row_bytes <= static_cast<int64_t>(kSlotBytes)) {
+      if (tp.ngroups == kMaxGroups) return APACK_EINVAL;
+      TmaGroup &g = tp.g[tp.ngroups++];
       g.src = static_cast<const uint8_t *>(p.src);
       g.dst = static_cast<uint8_t *>(p.dst);
       g.sps = p.src_plane_stride;
       g.dps = p.dst_plane_stride;
       g.srs = p.src_row_stride;
       g.drs = p.dst_row_stride;
-      g.vecs = static_cast<uint32_t>(p.row_bytes / 16);
-      g.pieces = (g.vecs + 31) / 32;
-      g.n_planes = static_cast<uint32_t>(p.num_planes);
+      g.row_bytes = static_cast<uint32_t>(p.row_bytes);
+      g.rows_per_slot = kSlotBytes / g.row_bytes;
+      g.chunks_per_plane = static_cast<uint32_t>((n_out + g.rows_per_slot - 1) / g.rows_per_slot);
       g.item_begin = static_cast<uint32_t>(items);
-      items += static_cast<uint64_t>(g.pieces) * p.num_planes * static_cast<uint64_t>(n_out);
+      g.contiguous = p.dst_row_stride == p.row_bytes;
+      items += static_cast<uint64_t>(g.chunks_per_plane) * p.num_planes;
       if (items > 0x7FFFFFFFull) return APACK_EINVAL;
     } else {
-      const int64_t n = static_cast<int64_t>(p.num_planes) * n_out;
-      const int threads = 256;
-      gather_narrow_kernel<<<static_cast<unsigned>((n + threads - 1) / threads), threads, 0, stream>>>(
-          static_cast<const uint8_t *>(p.src), static_cast<uint8_t *>(p.dst), p.src_plane_stride,
-          p.dst_plane_stride, p.src_row_stride, p.dst_row_stride, p.row_bytes, unit, p.num_planes, n_out, keep_idx);
-      count_launches(1);
-      if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+      if (n_narrow == kMaxGroups * 4) return APACK_EINVAL;
+      narrow[n_narrow++] = i;
     }
   }
-  if (wp.ngroups > 0) {
-    wp.total_items = static_cast<uint32_t>(items);
-    const uint64_t batches = (items + kUnroll - 1) / kUnroll;
-    const uint64_t warps_per_block = kWideThreads / 32;
-    uint64_t blocks = (batches + warps_per_block - 1) / warps_per_block;
-    const uint64_t cap = static_cast<uint64_t>(sms) * 8;   // 8 resident blocks of 256 threads per SM
-    if (blocks > cap) blocks = cap;
-    gather_wide_kernel<<<static_cast<unsigned>(blocks), kWideThreads, 0, stream>>>(wp, keep_idx);
+  for (int k = 0; k < n_narrow; ++k) {
+    const apack_plane &p = planes[narrow[k]];
+    const int64_t n = static_cast<int64_t>(p.num_planes) * n_out;
+    const int threads = 256;
+    gather_narrow_kernel<<<static_cast<unsigned>((n + threads - 1) / threads), threads, 0, stream>>>(
+        static_cast<const uint8_t *>(p.src), static_cast<uint8_t *>(p.dst), p.src_plane_stride, p.dst_plane_stride,
+        p.src_row_stride, p.dst_row_stride, p.row_bytes, widest_unit(p), p.num_planes, n_out, keep_idx);
+    count_launches(1);
+    if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+  }
+  if (tp.ngroups > 0) {
+    static bool attr_done = false;
+    if (!attr_done) {
+      if (check_cuda(cudaFuncSetAttribute(gather_tma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          kTmaSmem)) != APACK_OK)
+        return APACK_ECUDA;
+      attr_done = true;
+    }
+    tp.total_items = static_cast<uint32_t>(items);
+    uint64_t blocks = static_cast<uint64_t>(device_sm_count()) * 2;   // two CTAs of kSlots slots per SM
+    if (blocks > items) blocks = items;
+    gather_tma_kernel<<<static_cast<unsigned>(blocks), 32, kTmaSmem, stream>>>(tp, keep_idx, err);
     count_launches(1);
     if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
   }

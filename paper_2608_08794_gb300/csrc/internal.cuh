@@ -59,6 +59,6 @@ apack_status run_select(const apack_seqs *seqs, const float *scores, const int32
                         int32_t *keep_idx, uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu_seqlens,
                         void *ws, cudaStream_t stream);
 apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes, int32_t num_groups,
-                         cudaStream_t stream);
+                         DeviceError *err, cudaStream_t stream);
 
 }  // namespace apack

@@ -248,3 +248,20 @@ def test_device_fill_matches_host_generator(ap):
     fill_normal_bf16(t, 3, 2004, start=12345)
     torch.cuda.synchronize()
     np.testing.assert_array_equal(t.cpu().numpy().view(np.uint16), normal_bf16_bits(3, 2004, 12345, 1 << 20))
+
+
+def test_compact_strided_destination_rows(ap):
+    # output rows with a larger stride than the row: the copy stores row by row
+    rng = np.random.default_rng(10)
+    T, rb, pad = 1500, 1024, 512
+    keep = np.sort(rng.choice(T, 700, replace=False)).astype(np.int32)
+    src = rng.integers(0, 256, (3, T, rb), dtype=np.uint8)
+    s = dev(src)
+    d = torch.zeros((3, keep.size, rb + pad), dtype=torch.uint8, device="cuda")
+    p = ap.make_plane(s, d, rb, 3, src_plane_stride=T * rb, dst_plane_stride=keep.size * (rb + pad),
+                      dst_row_stride=rb + pad)
+    ap.apack_compact(dev(keep), keep.size, [p])
+    torch.cuda.synchronize()
+    out = d.cpu().numpy()
+    np.testing.assert_array_equal(out[:, :, :rb], src[:, keep, :])
+    assert not out[:, :, rb:].any()
