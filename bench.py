@@ -374,8 +374,8 @@ def main():
         achieved = sum(comp_bytes) / (comp_ms.sum() / 1e3) / 1e9
         prof = profiled_traffic("compact.cu")
         traffic = None
-        if prof is not None:
-            traffic = prof.get("dram_bytes_per_launch")
+        if prof is not None:   # ncu DRAM bytes of a captured launch, scaled to each launch by rows moved
+            traffic = [int(prof["traffic_over_algorithmic"] * b) for b in comp_bytes]
         score_ms, select_ms = stage_ms[:, 0].sum(), stage_ms[:, 1].sum()
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
