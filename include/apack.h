@@ -164,6 +164,25 @@ apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num
                               int32_t *new_cu_seqlens, float *scores, void *ws, size_t ws_bytes,
                               void *const *stage_events_h, void *stream);
 
+/* apack_score for callers that cannot allocate device memory: plugins inside
+   an engine that owns every device allocation, and serving processes that fix
+   their device memory at start-up.  The paper has no counterpart; it is a
+   deployment variant of apack_score.
+   Same arguments and results as apack_score, without the workspace: the
+   scratch is one 8 MiB array that the library keeps on every device it is
+   loaded on, until the process exits.  Batches whose apack_workspace_size
+   exceeds 8 MiB return APACK_EWORKSPACE (a single 7B-shaped sequence with
+   135k tokens and 256 query rows needs about 5.6 MiB).  Nothing is allocated.
+   The first call on a device looks the array's address up (a CUDA runtime
+   call); make that first call before any stream capture on that device.
+   All calls share the one array and it keeps the last call's contents: calls
+   that can overlap on the GPU (other streams, other threads) race on it and
+   must be serialised by the caller.
+   device_error_out: NULL, or a device int32 that receives the call's device
+   error code (APACK_OK, APACK_ETIMEOUT, APACK_EDEVICE) on `stream`. */
+apack_status apack_score_static(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
+                                float *scores, int32_t *device_error_out, void *stream);
+
 /* Synchronises `stream`, then reads the device error word of `ws` into
    *code_out (APACK_OK, APACK_ETIMEOUT or APACK_EDEVICE) and clears it when
    `clear` is non-zero. */

@@ -26,7 +26,8 @@ APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT = 0, 1
 APACK_HEAD_DIM = 128
 
 EXPORTED = ("apack_workspace_size", "apack_keep_counts", "apack_score", "apack_select", "apack_compact",
-            "apack_prune_step", "apack_device_error", "apack_launch_count", "apack_status_string")
+            "apack_prune_step", "apack_device_error", "apack_launch_count", "apack_status_string",
+            "apack_score_static")
 
 
 class ApackError(RuntimeError):
@@ -69,6 +70,7 @@ def _load():
                                      I32, VP, VP, I64, VP, P(apack_plane), I32, VP, VP, PI32, VP, VP, VP, SZ,
                                      P(VP), VP]
     lib.apack_device_error.argtypes = [VP, VP, PI32, I32]
+    lib.apack_score_static.argtypes = [P(apack_seqs), VP, VP, I64, VP, VP, VP]
     lib.apack_launch_count.argtypes = []
     lib.apack_launch_count.restype = ctypes.c_uint64
     lib.apack_status_string.argtypes = [I32]
@@ -219,6 +221,13 @@ def apack_prune_step(seqs, layer, num_layers, q, k_cache, v_cache, kv_layer_stri
         0 if ws is None else ws.numel() * ws.element_size(), ev, _stream(stream))
     _check(st, "apack_prune_step")
     return new_cu
+
+
+def apack_score_static(seqs, q, k, k_token_stride, scores, device_error_out=None, stream=None):
+    """apack_score without a workspace, for callers that cannot allocate device
+    memory (the library's fixed 8 MiB scratch array is used instead)."""
+    _check(_lib.apack_score_static(seqs.ref(), _ptr(q), _ptr(k), int(k_token_stride), _ptr(scores),
+                                   _ptr(device_error_out), _stream(stream)), "apack_score_static")
 
 
 def apack_device_error(ws, stream=None, clear=True):
