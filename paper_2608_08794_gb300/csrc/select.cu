@@ -11,10 +11,15 @@
 //     The result per segment is a threshold bit pattern T and a quota q: keep
 //     every score > T and the first q scores == T in token order (ties go to
 //     the lower index).
-//  2. Counts per CTA (other tokens, > T, == T) are exchanged through DSMEM so
-//     that each CTA knows its output offset and how many ties precede it.
-//  3. Each CTA walks its slice in token order with block-wide scans and writes
-//     keep_idx (ascending), the compacted modality and dst_of_src.
+//  2. Counts per warp run and per CTA (other tokens, > T, == T) are exchanged
+//     through DSMEM so that each warp knows its output offset and how many
+//     ties precede it.  Histogram atomics are aggregated per warp and bin.
+//  3. Each warp walks its contiguous run of the slice in token order (ballot
+//     prefix counts give the positions) and writes keep_idx (ascending), the
+//     compacted modality and dst_of_src.
+// A CTA's slice (scores as bit patterns and modality codes) is read from global
+// memory once into shared memory when it fits (slices up to kMaxCached tokens);
+// all passes then run on the shared copy.
 #include <cstdio>
 
 #include "internal.cuh"
@@ -25,10 +30,10 @@ namespace apack {
 namespace {
 
 constexpr int kCluster = 8;
-constexpr int kThreads = 512;
+constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;
-constexpr int kItems = 8;                       // contiguous tokens per thread per tile
-constexpr int kTile = kThreads * kItems;
+constexpr int kMaxCached = 40960;               // tokens per CTA slice cached in shared memory (200 KB)
+constexpr size_t kCacheBytes = static_cast<size_t>(kMaxCached) * 5;
 
 struct SelSeq {
   int32_t t0, len;
@@ -42,6 +47,7 @@ struct SelectPlan {
   int32_t nsegs;               // 2 per modality, 1 joint
   int32_t write_cu0;           // write new_cu_seqlens[0] = 0 (first launch of a batch)
   int32_t seq_base;            // index of seq[0] in the batch
+  int32_t cache_tokens;        // slice tokens the dynamic shared memory holds (0: no cache)
   SelSeq seq[kSeqsPerLaunch];
 };
 
@@ -51,51 +57,43 @@ __device__ __forceinline__ int seg_of(uint8_t m, int nsegs) {
   return -1;
 }
 
-// Exclusive block scan of one uint32 per thread; returns the exclusive prefix
-// and writes the block total to *total.  Uses `scratch` [kWarps + 1].
-__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t *scratch, uint32_t *total) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t incl = v;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const uint32_t n = __shfl_up_sync(0xffffffffu, incl, off);
-    if (lane >= off) incl += n;
+// One token of the slice, from the shared-memory copy when there is one.
+struct Tok {
+  uint32_t bits;
+  int seg;
+  uint8_t mod;
+  bool in;
+};
+
+__device__ __forceinline__ Tok load_tok(const float *__restrict__ scores, const uint8_t *__restrict__ modality,
+                                        const uint32_t *c_bits, const uint8_t *c_mod, int lo, int i, int end,
+                                        int nsegs) {
+  Tok t;
+  t.in = i < end;
+  if (c_bits) {
+    t.bits = t.in ? c_bits[i - lo] : 0u;
+    t.mod = t.in ? c_mod[i - lo] : static_cast<uint8_t>(0xFF);
+  } else {
+    t.bits = t.in ? __float_as_uint(scores[i]) : 0u;
+    t.mod = t.in ? modality[i] : static_cast<uint8_t>(0xFF);
   }
-  if (lane == 31) scratch[warp] = incl;
-  __syncthreads();
-  if (warp == 0) {
-    uint32_t w = lane < kWarps ? scratch[lane] : 0u;
-    uint32_t wi = w;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t n = __shfl_up_sync(0xffffffffu, wi, off);
-      if (lane >= off) wi += n;
-    }
-    if (lane < kWarps) scratch[lane] = wi - w;       // exclusive warp offsets
-    if (lane == kWarps - 1) scratch[kWarps] = wi;    // block total
-  }
-  __syncthreads();
-  const uint32_t res = scratch[warp] + incl - v;
-  *total = scratch[kWarps];
-  __syncthreads();
-  return res;
+  t.seg = seg_of(t.mod, nsegs);
+  return t;
 }
 
-// Loads the kItems contiguous tokens of this thread in the tile at `base`
-// (segment -1 and bits 0 past `hi` or outside S).  All loads are issued
-// before any is used.
-__device__ __forceinline__ void load_items(const float *__restrict__ scores, const uint8_t *__restrict__ modality,
-                                           int base, int hi, int nsegs, int (&seg)[kItems],
-                                           uint32_t (&bits)[kItems], uint8_t (&mod)[kItems]) {
-  const int i0 = base + threadIdx.x * kItems;
-#pragma unroll
-  for (int j = 0; j < kItems; ++j) {
-    const bool in = i0 + j < hi;
-    mod[j] = in ? modality[i0 + j] : static_cast<uint8_t>(0xFF);
-    bits[j] = in ? __float_as_uint(scores[i0 + j]) : 0u;
+// Adds one count per lane with bin >= 0.  When every counted lane of the warp
+// has the same bin (the usual case for the high digits, where neighbouring
+// scores share them) a single atomic carries the whole warp.
+__device__ __forceinline__ void add_bin(uint32_t *h, int bin, int lane) {
+  const uint32_t valid = __ballot_sync(0xffffffffu, bin >= 0);
+  if (valid == 0u) return;
+  const int first = __shfl_sync(0xffffffffu, bin, __ffs(valid) - 1);
+  const uint32_t same = __ballot_sync(0xffffffffu, bin == first);
+  if (same == valid) {
+    if (lane == 0) atomicAdd(&h[first], static_cast<uint32_t>(__popc(valid)));
+  } else if (bin >= 0) {
+    atomicAdd(&h[bin], 1u);
   }
-#pragma unroll
-  for (int j = 0; j < kItems; ++j) seg[j] = seg_of(mod[j], nsegs);
 }
 
 __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
@@ -104,19 +102,40 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
                   uint8_t *__restrict__ modality_out, int32_t *__restrict__ dst_of_src,
                   int32_t *__restrict__ new_cu, DeviceError *err) {
   __shared__ uint32_t hist[2][2][256];
+  __shared__ uint32_t tot[2][256];            // cluster-wide histogram of the current pass
+  __shared__ uint32_t rcnt[kCluster][5];      // per-CTA counts of the cluster
   __shared__ uint32_t st_prefix[2], st_mask[2], st_krem[2], st_total[2];
-  __shared__ uint32_t cnt[5];                 // other, gt0, gt1, eq0, eq1 (read by the cluster)
-  __shared__ uint32_t scratch[kWarps + 1];
-  __shared__ int32_t info[6];                 // kept_before, eq_before0, eq_before1, eq_mode0, eq_mode1
+  __shared__ uint32_t wcnt[kWarps][5];        // per warp chunk: other, gt0, gt1, eq0, eq1
+  __shared__ uint32_t cnt[5];                 // per CTA (read by the cluster)
+  __shared__ uint32_t wbase[kWarps], weqb[kWarps][2];
+  extern __shared__ __align__(16) uint8_t cache_raw[];
 
   const SelSeq &sq = plan.seq[blockIdx.y];
   const uint32_t crank = cluster_ctarank();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t lt_mask = (1u << lane) - 1u;
   const int nsegs = plan.nsegs;
   const int chunk = (sq.len + kCluster - 1) / kCluster;
   const int lo = sq.t0 + min(sq.len, static_cast<int>(crank) * chunk);
   const int hi = sq.t0 + min(sq.len, static_cast<int>(crank + 1) * chunk);
+  // each warp owns a contiguous run of the slice (a multiple of 32 tokens)
+  const int cw = ((hi - lo) + kWarps * 32 - 1) / (kWarps * 32) * 32;
+  const int wlo = min(hi, lo + warp * cw), whi = min(hi, wlo + cw);
 
+  // shared copy of the slice: bits [n] then modality [n]
+  const uint32_t *c_bits = nullptr;
+  const uint8_t *c_mod = nullptr;
+  const int n = hi - lo;
+  if (n <= plan.cache_tokens) {
+    uint32_t *wb = reinterpret_cast<uint32_t *>(cache_raw);
+    uint8_t *wm = cache_raw + static_cast<size_t>(plan.cache_tokens) * 4;
+    for (int x = tid; x < n; x += kThreads) {
+      wb[x] = __float_as_uint(scores[lo + x]);
+      wm[x] = modality[lo + x];
+    }
+    c_bits = wb;
+    c_mod = wm;
+  }
   for (int j = tid; j < 2 * 2 * 256; j += kThreads) (&hist[0][0][0])[j] = 0u;
   if (tid < 2) {
     st_prefix[tid] = 0u;
@@ -132,39 +151,48 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
     const int hb = d & 1;
     const int shift = 24 - 8 * d;
     const uint32_t p0 = st_prefix[0], p1 = st_prefix[1], m0 = st_mask[0], m1 = st_mask[1];
-    for (int base = lo; base < hi; base += kTile) {
-      int sg[kItems];
-      uint32_t bt[kItems];
-      uint8_t md[kItems];
-      load_items(scores, modality, base, hi, nsegs, sg, bt, md);
-#pragma unroll
-      for (int j = 0; j < kItems; ++j) {
-        if (sg[j] < 0) continue;
-        const uint32_t pm = sg[j] ? p1 : p0, mm = sg[j] ? m1 : m0;
-        if ((bt[j] & mm) == pm) atomicAdd(&hist[hb][sg[j]][(bt[j] >> shift) & 255u], 1u);
-      }
+    // two 32-token rounds per iteration (independent chains)
+    for (int b = wlo; b < whi; b += 64) {
+      const Tok t0 = load_tok(scores, modality, c_bits, c_mod, lo, b + lane, whi, nsegs);
+      const Tok t1 = load_tok(scores, modality, c_bits, c_mod, lo, b + 32 + lane, whi, nsegs);
+      int bin0 = -1, bin1 = -1;
+      if (t0.seg >= 0 && (t0.bits & (t0.seg ? m1 : m0)) == (t0.seg ? p1 : p0))
+        bin0 = t0.seg * 256 + static_cast<int>((t0.bits >> shift) & 255u);
+      if (t1.seg >= 0 && (t1.bits & (t1.seg ? m1 : m0)) == (t1.seg ? p1 : p0))
+        bin1 = t1.seg * 256 + static_cast<int>((t1.bits >> shift) & 255u);
+      add_bin(&hist[hb][0][0], bin0, lane);
+      add_bin(&hist[hb][0][0], bin1, lane);
     }
     __syncthreads();
     cluster_sync();
     for (int j = tid; j < 2 * 256; j += kThreads) (&hist[hb ^ 1][0][0])[j] = 0u;
+    // cluster-wide histogram: thread (seg, bin) adds the bin of every CTA, its
+    // kCluster remote loads issued back to back
+    for (int j = tid; j < nsegs * 256; j += kThreads) {
+      uint32_t v[kCluster];
+#pragma unroll
+      for (int r = 0; r < kCluster; ++r) v[r] = ld_shared_cluster_u32(map_shared_rank(&(&hist[hb][0][0])[j], r));
+      uint32_t sum = 0;
+#pragma unroll
+      for (int r = 0; r < kCluster; ++r) sum += v[r];
+      (&tot[0][0])[j] = sum;
+    }
+    __syncthreads();
     if (warp < nsegs) {
       const int seg = warp;
       uint32_t c[8];
       uint32_t lsum = 0;
 #pragma unroll
       for (int b = 0; b < 8; ++b) {
-        uint32_t v = 0;
-        for (int r = 0; r < kCluster; ++r)
-          v += ld_shared_cluster_u32(map_shared_rank(&hist[hb][seg][lane * 8 + b], r));
-        c[b] = v;
-        lsum += v;
+        c[b] = tot[seg][lane * 8 + b];
+        lsum += c[b];
       }
       // inclusive suffix sum over lanes (higher lanes hold higher digits)
       uint32_t suf = lsum;
 #pragma unroll
       for (int off = 1; off < 32; off <<= 1) {
-        const uint32_t n = __shfl_down_sync(0xffffffffu, suf, off);
-        if (lane + off < 32) suf += n;
+        const uint32_t nb = __shfl_down_sync(0xffffffffu, suf, off);
+        if (lane + off < 32) suf += nb;
       }
       const uint32_t above_lane = suf - lsum;
       const uint32_t total = __shfl_sync(0xffffffffu, suf, 0);
@@ -207,40 +235,43 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
     quota[s] = none ? 0u : st_krem[s];
   }
 
-  // ---- 2. per-CTA counts, exchanged through the cluster
+  // ---- 2. counts per warp run, per CTA, exchanged through the cluster
   {
-    uint32_t other = 0, gt0 = 0, gt1 = 0, eq0 = 0, eq1 = 0;
-    for (int base = lo; base < hi; base += kTile) {
-      int sg[kItems];
-      uint32_t bt[kItems];
-      uint8_t md[kItems];
-      load_items(scores, modality, base, hi, nsegs, sg, bt, md);
-#pragma unroll
-      for (int j = 0; j < kItems; ++j) {
-        if (base + tid * kItems + j >= hi) break;
-        if (sg[j] < 0) { ++other; continue; }
-        const uint32_t t = sg[j] ? T[1] : T[0];
-        if (bt[j] > t) { if (sg[j]) ++gt1; else ++gt0; }
-        else if (bt[j] == t) { if (sg[j]) ++eq1; else ++eq0; }
-      }
+    uint32_t c_other = 0, c_gt0 = 0, c_gt1 = 0, c_eq0 = 0, c_eq1 = 0;
+    for (int b = wlo; b < whi; b += 32) {
+      const Tok t = load_tok(scores, modality, c_bits, c_mod, lo, b + lane, whi, nsegs);
+      const uint32_t tt = t.seg > 0 ? T[1] : T[0];
+      c_other += __popc(__ballot_sync(0xffffffffu, t.in && t.seg < 0));
+      c_gt0 += __popc(__ballot_sync(0xffffffffu, t.seg == 0 && t.bits > tt));
+      c_gt1 += __popc(__ballot_sync(0xffffffffu, t.seg == 1 && t.bits > tt));
+      c_eq0 += __popc(__ballot_sync(0xffffffffu, t.seg == 0 && t.bits == tt));
+      c_eq1 += __popc(__ballot_sync(0xffffffffu, t.seg == 1 && t.bits == tt));
     }
-    uint32_t tot;
-    // five reductions through the scan helper (exclusive value unused)
-    block_exclusive_scan(other, scratch, &tot); if (tid == 0) cnt[0] = tot;
-    block_exclusive_scan(gt0, scratch, &tot);   if (tid == 0) cnt[1] = tot;
-    block_exclusive_scan(gt1, scratch, &tot);   if (tid == 0) cnt[2] = tot;
-    block_exclusive_scan(eq0, scratch, &tot);   if (tid == 0) cnt[3] = tot;
-    block_exclusive_scan(eq1, scratch, &tot);   if (tid == 0) cnt[4] = tot;
+    if (lane == 0) {
+      wcnt[warp][0] = c_other;
+      wcnt[warp][1] = c_gt0;
+      wcnt[warp][2] = c_gt1;
+      wcnt[warp][3] = c_eq0;
+      wcnt[warp][4] = c_eq1;
+    }
+  }
+  __syncthreads();
+  if (tid < 5) {
+    uint32_t v = 0;
+    for (int w = 0; w < kWarps; ++w) v += wcnt[w][tid];
+    cnt[tid] = v;
   }
   __syncthreads();
   cluster_sync();
+  if (tid < kCluster * 5) rcnt[tid / 5][tid % 5] = ld_shared_cluster_u32(map_shared_rank(&cnt[tid % 5], tid / 5));
+  __syncthreads();
   if (tid == 0) {
-    uint32_t kept_before = 0, eqb[2] = {0, 0}, kept_all = 0, seg_dev[2] = {0, 0};
-    // Walk the CTAs in order: ties are granted to CTAs until the quota runs out.
-    uint32_t eq_prefix[2] = {0, 0};
+    // Walk the CTAs of the cluster, then the warps of this CTA, in token order:
+    // ties are granted until the quota runs out.
+    uint32_t kept_before = 0, kept_all = 0, seg_dev[2] = {0, 0};
+    uint32_t eq_prefix[2] = {0, 0}, eqb[2] = {0, 0};
     for (int r = 0; r < kCluster; ++r) {
-      uint32_t c[5];
-      for (int j = 0; j < 5; ++j) c[j] = ld_shared_cluster_u32(map_shared_rank(&cnt[j], r));
+      const uint32_t *c = rcnt[r];
       uint32_t kept = c[0] + c[1] + c[2];
       for (int s = 0; s < 2; ++s) {
         const uint32_t ties = c[3 + s];
@@ -253,16 +284,18 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
       if (r < static_cast<int>(crank)) kept_before += kept;
       kept_all += kept;
     }
-    info[0] = static_cast<int32_t>(kept_before);
-    for (int s = 0; s < 2; ++s) {
-      info[1 + s] = static_cast<int32_t>(eqb[s]);
-      // tie mode of this CTA: 0 = drop all its ties, 1 = keep all, 2 = rank them
-      const uint32_t my_ties = cnt[3 + s];
-      int mode;
-      if (eqb[s] >= quota[s]) mode = 0;
-      else if (eqb[s] + my_ties <= quota[s]) mode = 1;
-      else mode = 2;
-      info[3 + s] = mode;
+    uint32_t run = kept_before;
+    for (int w = 0; w < kWarps; ++w) {
+      wbase[w] = run;
+      uint32_t kept = wcnt[w][0] + wcnt[w][1] + wcnt[w][2];
+      for (int s = 0; s < 2; ++s) {
+        weqb[w][s] = eqb[s];
+        const uint32_t ties = wcnt[w][3 + s];
+        const uint32_t avail = quota[s] > eqb[s] ? quota[s] - eqb[s] : 0u;
+        kept += ties < avail ? ties : avail;
+        eqb[s] += ties;
+      }
+      run += kept;
     }
     if (crank == 0) {
       // Device-side consistency with the host counts.
@@ -280,65 +313,36 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
   __syncthreads();
   cluster_sync();   // all remote reads of cnt[] are done before any CTA may exit
 
-  // ---- 3. ordered write of the kept tokens of this slice
-  uint32_t run_keep = static_cast<uint32_t>(info[0]);
-  uint32_t run_eq[2] = {static_cast<uint32_t>(info[1]), static_cast<uint32_t>(info[2])};
-  const int mode0 = info[3], mode1 = info[4];
-  const bool need_rank = (mode0 == 2) || (mode1 == 2);
-  for (int base = lo; base < hi; base += kTile) {
-    int sg[kItems];
-    uint32_t bt[kItems];
-    uint8_t md[kItems];
-    load_items(scores, modality, base, hi, nsegs, sg, bt, md);
-    const int i0 = base + tid * kItems;
-    bool keep[kItems], eq[kItems];
-#pragma unroll
-    for (int j = 0; j < kItems; ++j) {
-      const bool valid = i0 + j < hi;
-      const uint32_t t = sg[j] > 0 ? T[1] : T[0];
-      eq[j] = valid && sg[j] >= 0 && bt[j] == t;
-      keep[j] = valid && (sg[j] < 0 || bt[j] > t || (eq[j] && (sg[j] ? mode1 : mode0) == 1));
+  // ---- 3. ordered writes: each warp walks its run in token order
+  uint32_t pos = wbase[warp];
+  uint32_t er0 = weqb[warp][0], er1 = weqb[warp][1];
+  for (int b = wlo; b < whi; b += 32) {
+    const int i = b + lane;
+    const Tok t = load_tok(scores, modality, c_bits, c_mod, lo, i, whi, nsegs);
+    const uint32_t tt = t.seg > 0 ? T[1] : T[0];
+    const bool eq = t.seg >= 0 && t.bits == tt;
+    const uint32_t em0 = __ballot_sync(0xffffffffu, eq && t.seg == 0);
+    const uint32_t em1 = __ballot_sync(0xffffffffu, eq && t.seg == 1);
+    bool keep = t.in && (t.seg < 0 || t.bits > tt);
+    if (eq) {
+      const uint32_t rank = t.seg ? er1 + __popc(em1 & lt_mask) : er0 + __popc(em0 & lt_mask);
+      keep = rank < (t.seg ? quota[1] : quota[0]);
     }
-    if (need_rank) {
-      // ties ranked in token order: per-thread counts (packed: low 16 bits
-      // segment 0, high 16 bits segment 1), then a block scan
-      uint32_t e = 0;
-#pragma unroll
-      for (int j = 0; j < kItems; ++j)
-        if (eq[j]) e += sg[j] ? (1u << 16) : 1u;
-      uint32_t etot;
-      uint32_t ex = block_exclusive_scan(e, scratch, &etot);
-      uint32_t r0 = run_eq[0] + (ex & 0xFFFFu), r1 = run_eq[1] + (ex >> 16);
-#pragma unroll
-      for (int j = 0; j < kItems; ++j) {
-        if (!eq[j]) continue;
-        const int md2 = sg[j] ? mode1 : mode0;
-        uint32_t &r = sg[j] ? r1 : r0;
-        if (md2 == 2) keep[j] = r < (sg[j] ? quota[1] : quota[0]);
-        ++r;
-      }
-      run_eq[0] += etot & 0xFFFFu;
-      run_eq[1] += etot >> 16;
-    }
-    uint32_t nk = 0;
-#pragma unroll
-    for (int j = 0; j < kItems; ++j) nk += keep[j] ? 1u : 0u;
-    uint32_t ktot;
-    uint32_t pos = run_keep + block_exclusive_scan(nk, scratch, &ktot);
-#pragma unroll
-    for (int j = 0; j < kItems; ++j) {
-      if (i0 + j >= hi) break;
-      if (keep[j] && pos < static_cast<uint32_t>(sq.out_len)) {
-        const int o = sq.out_base + static_cast<int>(pos);
-        keep_idx[o] = i0 + j;
-        if (modality_out) modality_out[o] = md[j];
-        if (dst_of_src) dst_of_src[i0 + j] = o;
+    const uint32_t km = __ballot_sync(0xffffffffu, keep);
+    const uint32_t p = pos + __popc(km & lt_mask);
+    if (t.in) {
+      if (keep && p < static_cast<uint32_t>(sq.out_len)) {
+        const int o = sq.out_base + static_cast<int>(p);
+        keep_idx[o] = i;
+        if (modality_out) modality_out[o] = t.mod;
+        if (dst_of_src) dst_of_src[i] = o;
       } else if (dst_of_src) {
-        dst_of_src[i0 + j] = -1;
+        dst_of_src[i] = -1;
       }
-      if (keep[j]) ++pos;
     }
-    run_keep += ktot;
+    pos += __popc(km);
+    er0 += __popc(em0);
+    er1 += __popc(em1);
   }
 }
 
@@ -396,9 +400,25 @@ apack_status run_select(const apack_seqs *seqs, const float *scores, const int32
       q.out_base = out_base;
       out_base += q.out_len;
     }
+    // cache each CTA's slice in shared memory when the longest slice of the launch fits
+    int max_len = 0;
+    for (int i = 0; i < ns; ++i) max_len = P.seq[i].len > max_len ? P.seq[i].len : max_len;
+    const int slice = (max_len + kCluster - 1) / kCluster;
+    size_t smem = 0;
+    if (slice <= kMaxCached) {
+      P.cache_tokens = slice;
+      smem = static_cast<size_t>(slice) * 5;
+    }
+    static bool attr_done = false;
+    if (!attr_done) {
+      if (check_cuda(cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          static_cast<int>(kCacheBytes))) != APACK_OK)
+        return APACK_ECUDA;
+      attr_done = true;
+    }
     dim3 grid(kCluster, ns, 1);
-    select_kernel<<<grid, kThreads, 0, stream>>>(P, scores, seqs->modality, keep_idx, modality_out, dst_of_src,
-                                                 new_cu_seqlens, err);
+    select_kernel<<<grid, kThreads, smem, stream>>>(P, scores, seqs->modality, keep_idx, modality_out, dst_of_src,
+                                                    new_cu_seqlens, err);
     count_launches(1);
     if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
   }

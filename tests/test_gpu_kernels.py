@@ -152,6 +152,7 @@ def gpu_select(ap, scores, mod, cu, counts, na, nv, mode):
 SEL_CASES = [
     ([2000], "random"), ([1298], "ties"), ([50000, 30, 7000, 0, 1], "random"),
     ([20000], "allequal"), ([100000], "coarse"), ([3, 5, 7, 9, 11, 13, 15, 17, 19, 21] * 7, "coarse"),
+    ([400000], "coarse"),   # slices beyond the shared-memory cache: passes read global memory
 ]
 
 
