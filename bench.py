@@ -49,6 +49,21 @@ def parse():
 
 # ----------------------------------------------------------------------------- helpers
 
+def max_over_ranks(x, dist, device):
+    """The largest value of x over all ranks (x itself without a process group)."""
+    if dist is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_value(units_per_rank, world, ms_per_iter):
+    """Units of all ranks per second, each rank running its own replica."""
+    return world * units_per_rank / (ms_per_iter / 1e3)
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -303,11 +318,7 @@ def main():
     if clocks:
         clocks.mark(False)
     launches = ap.apack_launch_count() - launches0
-    ms = t_start.elapsed_time(t_end)
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(t_start.elapsed_time(t_end), dist, "cuda")
     stage_ms = np.zeros((nsteps, 3))
     for k in range(args.steps):
         for i in range(nsteps):
@@ -360,15 +371,11 @@ def main():
     if clocks:
         clocks.mark(False)
         clocks.stop()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
-    if dist is not None:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dist, "cuda")
 
     if rank == 0:
         per_step_ms = ms / args.steps
-        value = world * mm_per_iter / (per_step_ms / 1e3)
+        value = whole_job_value(mm_per_iter, world, per_step_ms)
         peak, peak_kind = measured_peaks()
         comp_ms = stage_ms[:, 2]
         achieved = sum(comp_bytes) / (comp_ms.sum() / 1e3) / 1e9
@@ -396,7 +403,7 @@ def main():
                          "avg_launch_ms": [float(x) for x in comp_ms]},
             "stages_ms_per_iter": {"score": float(score_ms), "select": float(select_ms),
                                    "compact": float(comp_ms.sum())},
-            "e2e": {"value": world * mm_per_iter / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+            "e2e": {"value": whole_job_value(mm_per_iter, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps},
             "clocks": clocks.summary() if clocks else None,
         }
