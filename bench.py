@@ -173,7 +173,13 @@ ks = [key_slab(wl, l, q) for l, q in zip(wl.prune_layers, qs)]
 # bulk K/V planes: one drawn layer repeated over the compacted layers (values do not change the copy cost)
 kv = [np.repeat(plain_key_slab(wl, l0)[None], L - l0, axis=0), np.repeat(value_slab(wl, l0)[None], L - l0, axis=0)]
 hid = hidden_states(wl)
-counts = [oracle.step_keep_counts(r, base_counts(wl)) for r in wl.ratios]
+if wl.joint_step_keep is None:
+    counts = [oracle.step_keep_counts(r, base_counts(wl)) for r in wl.ratios]
+else:
+    counts, nS = [], [a + v for a, v in base_counts(wl)]
+    for _ in wl.prune_layers:
+        nS = [oracle.keep_count(wl.joint_step_keep, x) for x in nS]
+        counts.append([(x, 0) for x in nS])
 def one():
     comp = np.arange(wl.total_tokens); c, m = cu, mod
     kk, vv, hh = kv[0], kv[1], hid
@@ -182,7 +188,8 @@ def one():
         mm += int(((m == 1) | (m == 2)).sum())
         j = layer - l0 if i == 0 else layer - wl.prune_layers[i - 1]
         out = oracle.prune_step(qs[i], ks[i][comp], c, cuq, m, wl.num_q_heads, wl.num_kv_heads, counts[i],
-                                planes=[kk[j:].transpose(1, 0, 2, 3), vv[j:].transpose(1, 0, 2, 3), hh])
+                                planes=[kk[j:].transpose(1, 0, 2, 3), vv[j:].transpose(1, 0, 2, 3), hh],
+                                joint=wl.joint_step_keep is not None)
         keep = out["keep_idx"]
         kk = out["planes"][0].transpose(1, 0, 2, 3); vv = out["planes"][1].transpose(1, 0, 2, 3); hh = out["planes"][2]
         comp, c, m = comp[keep], out["cu_seqlens"], out["modality"]
@@ -255,7 +262,7 @@ def main():
     import numpy as np
     import torch
     import paper_2608_08794_gb300 as ap
-    from paper_2608_08794_gb300.schedule import ProgressivePrune
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
     from synth import workload
     from synth.device import fill_progressive_inputs
 
@@ -275,10 +282,10 @@ def main():
     na = np.array([s.n_audio for s in wl.seqs], np.int32)
     nv = np.array([s.n_visual for s in wl.seqs], np.int32)
     mod_tmp = torch.from_numpy(wl.modality()).cuda()
-    s0 = ap.Seqs(cu0, cuq, na, nv, mod_tmp, wl.num_q_heads, wl.num_kv_heads)
-    counts = [ap.apack_keep_counts(s0, np.array(r, np.float32))[0] for r in wl.ratios]
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_tmp,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
     pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
-                          wl.prune_layers, counts)
+                          wl.prune_layers, counts, select_mode=mode)
     fill_progressive_inputs(pp, wl)
     mm_per_iter = sum(pp.mm_tokens_per_step())
     nsteps = len(wl.prune_layers)

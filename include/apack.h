@@ -64,7 +64,9 @@ typedef struct apack_seqs {
   const int32_t *cu_seqlens_h;  /* [B+1] token offsets, cu_seqlens_h[0] == 0, non-decreasing */
   const int32_t *cu_qlens_h;    /* [B+1] offsets of each sequence's query rows in the packed Q */
   const int32_t *n_audio_h;     /* [B] audio tokens per sequence (verified on the device) */
-  const int32_t *n_visual_h;    /* [B] visual tokens per sequence (verified on the device) */
+  const int32_t *n_visual_h;    /* [B] visual tokens per sequence (verified on the device);
+                                   with APACK_SELECT_JOINT only n_audio_h + n_visual_h = |S| is
+                                   used, so a caller that knows only |S| may pass (|S|, 0) */
   const uint8_t *modality;      /* [T] APACK_MOD_* per token, T = cu_seqlens_h[B] */
   int32_t num_q_heads;          /* Hq */
   int32_t num_kv_heads;         /* Hkv; Hq % Hkv == 0, query head h reads key head h / (Hq/Hkv) */

@@ -62,6 +62,16 @@ WsLayout workspace_layout(const apack_seqs *s) {
   }
   auto up = [](size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); };
   L.err_off = 0;
+  if (narrow_score_applies(s)) {
+    size_t lf = 0, pf = 0, ef = 0;
+    narrow_layout(s, &lf, &pf, &ef);
+    L.narrow = true;
+    L.nlog_off = 1024;
+    L.npart_off = up(L.nlog_off + lf * sizeof(float));
+    L.nlse_off = up(L.npart_off + pf * sizeof(float2));
+    L.total = up(L.nlse_off + ef * sizeof(float));
+    return L;
+  }
   L.part_off = 1024;
   const size_t part_bytes = static_cast<size_t>(kMaxSplits) * NQ * s->num_q_heads * sizeof(float2);
   L.lse_off = up(L.part_off + part_bytes);

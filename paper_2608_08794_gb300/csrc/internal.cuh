@@ -12,6 +12,9 @@ namespace apack {
 
 // Sequences handled by one kernel launch; larger batches take several launches.
 constexpr int kSeqsPerLaunch = 64;
+// Narrow scoring path: at most this many query rows per KV head group, and in all.
+constexpr int kNarrowGroupRows = 32;
+constexpr int kNarrowRows = 256;
 // Wall-clock limit of every device-side wait.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 // Key splits of the row-statistics pass (upper bound, sizes the workspace).
@@ -40,6 +43,11 @@ struct WsLayout {
   size_t lse_off;     // float [chunks][128]: negated log2 normalisers per 128-row query chunk, -inf padding
   size_t qp_off;      // bf16 [qp_rows][128]: query rows repacked per KV head group, 256-row padded
   size_t gsum_off;    // float [Hkv][T]: per head group key sums of the column pass
+  // few query rows per head group (narrow path, used instead of the four above):
+  bool narrow;
+  size_t nlog_off;    // float [sum over sequences of Hq n_q len]: log2-domain logits
+  size_t npart_off;   // float2 [sum of Hq n_q ctas]: per-CTA row (max, sum of exp2)
+  size_t nlse_off;    // float [sum of Hq n_q]: log2 normalisers
   size_t total;
   int64_t lse_chunks;
   int64_t qp_rows;
@@ -55,6 +63,10 @@ apack_status validate_seqs(const apack_seqs *seqs, int64_t *total_tokens, int64_
 
 apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
                        float *scores, void *ws, cudaStream_t stream);
+bool narrow_score_applies(const apack_seqs *seqs);
+void narrow_layout(const apack_seqs *seqs, size_t *logit_floats, size_t *part_float2s, size_t *lse_floats);
+apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
+                              float *scores, void *ws, cudaStream_t stream);
 apack_status run_select(const apack_seqs *seqs, const float *scores, const int32_t *keep_count_h, int32_t mode,
                         int32_t *keep_idx, uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu_seqlens,
                         void *ws, cudaStream_t stream);

@@ -734,6 +734,8 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
   const int hq = seqs->num_q_heads, hkv = seqs->num_kv_heads, G = hq / hkv;
   if (hkv > 256) return APACK_EUNSUPPORTED;
   if (T == 0) return APACK_OK;
+  // few query rows per head group (e.g. the last query token only): K-read-bound CUDA-core path
+  if (narrow_score_applies(seqs)) return run_score_narrow(seqs, q, k, k_token_stride, scores, ws, stream);
   const WsLayout L = workspace_layout(seqs);
   uint8_t *wsb = static_cast<uint8_t *>(ws);
   DeviceError *err = reinterpret_cast<DeviceError *>(wsb + L.err_off);

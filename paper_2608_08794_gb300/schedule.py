@@ -14,7 +14,31 @@ Only buffer management and argument marshalling happen here.
 import numpy as np
 import torch
 
-from . import (Seqs, apack_prune_step, apack_workspace_size, APACK_HEAD_DIM, APACK_SELECT_PER_MODALITY)
+from . import (Seqs, apack_prune_step, apack_workspace_size, apack_keep_counts, APACK_HEAD_DIM,
+               APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT)
+
+
+def schedule_keep_counts(cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, num_kv_heads, modality,
+                         steps, cumulative_ratios=None, joint_step_keep=None):
+    """Keep counts [B, 2] of every step of a schedule, from the library's rule
+    (ceil((1-P)|S|) of Eq. inner, apack_keep_counts), and the selection mode.
+
+    cumulative_ratios[i][b] = (audio, visual) keep ratios of step i, applied to
+    the counts entering step 0 (per-modality selection); or joint_step_keep =
+    the fraction of the current |S| each step keeps (the paper's joint form)."""
+    na = np.asarray(n_audio, np.int32)
+    nv = np.asarray(n_visual, np.int32)
+    if joint_step_keep is None:
+        s0 = Seqs(cu_seqlens, cu_qlens, na, nv, modality, num_q_heads, num_kv_heads)
+        counts = [apack_keep_counts(s0, np.asarray(r, np.float32))[0] for r in cumulative_ratios]
+        return counts, APACK_SELECT_PER_MODALITY
+    counts, n = [], na + nv
+    for _ in range(steps):
+        s = Seqs(cu_seqlens, cu_qlens, n, np.zeros_like(n), modality, num_q_heads, num_kv_heads)
+        k, _ = apack_keep_counts(s, np.full((len(n), 2), joint_step_keep, np.float32), APACK_SELECT_JOINT)
+        counts.append(k)
+        n = k[:, 0].copy()
+    return counts, APACK_SELECT_JOINT
 
 
 class ProgressivePrune:

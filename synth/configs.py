@@ -84,6 +84,9 @@ class Workload:
     # counts entering the first step
     ratios: List[List[Tuple[float, float]]]
     plants: List[List[Plant]] = field(default_factory=list)  # per sequence
+    # joint selection over S with a per-step keep fraction of the current |S|
+    # (the paper's form); when set, `ratios` is unused
+    joint_step_keep: float = None
 
     @property
     def num_seqs(self) -> int:
@@ -170,6 +173,15 @@ def _build() -> dict:
         ratios=[[(0.7, 0.4)]],
         plants=[[Plant(1, 750, 1.0), Plant(2, 6000, 1.0),
                  Plant(1, 15, 3.0), Plant(2, 120, 3.0)]])
+    # The paper's own inner-LLM setting on the 10-minute sequence: the last query
+    # token only, one top-k over all of S, pruning at every layer from L_mid = 14
+    # (depth / 2) to 27 with P = 15% of the current |S| per layer (25% tier).
+    s4q = SeqLayout(duration_s=600, fps=2, tpf=100, n_q=1)
+    w["7b_10min_paper"] = Workload(
+        name="7b_10min_paper", seed=5, **_qwen7b(), seqs=[s4q], prune_layers=list(range(14, 28)),
+        ratios=[], joint_step_keep=0.85,
+        plants=[[Plant(1, 750, 1.0), Plant(2, 6000, 1.0),
+                 Plant(1, 15, 3.0), Plant(2, 120, 3.0)]])
     # 5: ragged batch of 16 7B-shaped sequences, prune at layer 8.
     seqs5, r5 = _ragged_seqs(4, 16)
     w["7b_ragged16"] = Workload(
@@ -201,4 +213,4 @@ def scaled_copy(wl: Workload, duration_s: int, n_q: int = None, name: str = None
     return Workload(name=name or f"{wl.name}@{duration_s}s", seed=wl.seed, num_layers=wl.num_layers,
                     num_q_heads=wl.num_q_heads, num_kv_heads=wl.num_kv_heads, head_dim=wl.head_dim,
                     hidden=wl.hidden, seqs=[s], prune_layers=list(wl.prune_layers),
-                    ratios=[[r[0]] for r in wl.ratios], plants=[plants])
+                    ratios=[[r[0]] for r in wl.ratios], plants=[plants], joint_step_keep=wl.joint_step_keep)

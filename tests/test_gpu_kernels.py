@@ -82,7 +82,28 @@ SHAPES = [
     ([513], [3], 4, 4),                     # MHA (group 1)
     ([129, 257, 1], [7, 19, 2], 12, 2),     # tails of one key past a tile
     ([0, 40, 60], [2, 0, 3], 28, 4),        # empty sequence and a sequence without query rows
+    ([0, 40, 600], [2, 0, 30], 28, 4),      # the same on the tensor-core path (210 rows per group)
 ]
+
+# At most 32 query rows per KV head group take the K-read-bound CUDA-core path
+# (the paper scores with the last query token only: G = 7 rows per group).
+NARROW_SHAPES = [
+    ([1000], [1], 28, 4),
+    ([3000, 700, 1, 0, 90], [1, 4, 2, 1, 0], 28, 4),
+    ([5000], [2], 16, 2),                   # 16 rows per group
+    ([2049], [4], 8, 1),                    # 32 rows in one group
+]
+
+
+@pytest.mark.parametrize("lens,nqs,hq,hkv", NARROW_SHAPES)
+def test_narrow_path_scores_match_oracle(ap, lens, nqs, hq, hkv):
+    rng = np.random.default_rng(sum(lens) * 3 + hq)
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, lens, nqs, hq, hkv, scale_k=1.5)
+    got = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv)
+    ref = oracle.relevance_scores(q, k, cu, cuq, mod, hq, hkv)
+    check_scores(got, ref, strict_rel=2e-3)
+    again = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv)
+    assert got.tobytes() == again.tobytes()
 
 
 @pytest.mark.parametrize("lens,nqs,hq,hkv", SHAPES)

@@ -32,12 +32,26 @@ def host_u16(t):
     return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
 
 
-@pytest.mark.parametrize("name", ["tiny", "3b_60s", "7b_2min", "7b_10min", "7b_ragged16"])
+def oracle_counts(wl):
+    """The oracle's keep counts per step and the joint flag."""
+    from synth.inputs import base_counts
+    if wl.joint_step_keep is None:
+        return [oracle.step_keep_counts(r, base_counts(wl)) for r in wl.ratios], False
+    n = [a + v for a, v in base_counts(wl)]
+    out = []
+    for _ in wl.prune_layers:
+        k = [oracle.keep_count(wl.joint_step_keep, x) for x in n]
+        out.append([(x, 0) for x in k])
+        n = k
+    return out, True
+
+
+@pytest.mark.parametrize("name", ["tiny", "3b_60s", "7b_2min", "7b_10min", "7b_ragged16", "7b_10min_paper"])
 def test_workload_parity(ap, name):
-    from paper_2608_08794_gb300.schedule import ProgressivePrune
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
     from synth import workload
     from synth.device import fill_progressive_inputs
-    from synth.inputs import key_slab, planted_tokens, base_counts
+    from synth.inputs import key_slab, planted_tokens
 
     wl = workload(name)
     cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
@@ -45,15 +59,12 @@ def test_workload_parity(ap, name):
     nv = np.array([s.n_visual for s in wl.seqs], np.int32)
     mod0 = wl.modality()
     mod_d = torch.from_numpy(mod0).cuda()
-    s0 = ap.Seqs(cu0, cuq, na, nv, mod_d, wl.num_q_heads, wl.num_kv_heads)
-    counts = []
-    for i in range(len(wl.prune_layers)):
-        k_gpu, _ = ap.apack_keep_counts(s0, np.array(wl.ratios[i], np.float32))
-        k_ref = oracle.step_keep_counts(wl.ratios[i], base_counts(wl))
-        assert k_gpu.tolist() == [list(x) for x in k_ref]
-        counts.append(k_gpu)
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_d,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
+    ref_counts, joint = oracle_counts(wl)
+    assert [c.tolist() for c in counts] == [[list(x) for x in r] for r in ref_counts]
     pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
-                          wl.prune_layers, counts)
+                          wl.prune_layers, counts, select_mode=mode)
     qs = fill_progressive_inputs(pp, wl)
 
     composite = np.arange(wl.total_tokens)
@@ -72,11 +83,12 @@ def test_workload_parity(ap, name):
         got = pp.scores[:T_in].cpu().numpy()
         check_scores(got, ref_scores)
         # selection
-        ref_keep = oracle.select_keep(ref_scores, mod_cur, cu_cur, [tuple(c) for c in counts[i]])
+        ref_keep = oracle.select_keep(ref_scores, mod_cur, cu_cur, [tuple(c) for c in counts[i]], joint=joint)
         keep = pp.keep_idx[i][:t_out].cpu().numpy().astype(np.int64)
-        exempt_total += check_keep(keep, ref_keep, ref_scores, mod_cur, cu_cur)
+        exempt_total += check_keep(keep, ref_keep, ref_scores, mod_cur, cu_cur, joint=joint)
         # the GPU's own selection is exact on its own fp32 scores
-        np.testing.assert_array_equal(keep, oracle.select_keep(got, mod_cur, cu_cur, [tuple(c) for c in counts[i]]))
+        np.testing.assert_array_equal(keep, oracle.select_keep(got, mod_cur, cu_cur, [tuple(c) for c in counts[i]],
+                                                               joint=joint))
         np.testing.assert_array_equal(new_cu, oracle.new_cu_seqlens(keep, cu_cur))
         np.testing.assert_array_equal(pp.mod_out[i % 2][:t_out].cpu().numpy(), mod_cur[keep])
         # compaction, bit-exact given the GPU's indices, on sampled layers

@@ -43,4 +43,6 @@ def test_workload_layouts():
     for s, (ra, rv) in zip(r.seqs, r.ratios[0]):
         assert 30 <= s.duration_s <= 300 and s.duration_s % 2 == 0 and 16 <= s.n_q <= 256
         assert 0.2 <= ra <= 0.6 and 0.2 <= rv <= 0.6
-    assert len(WORKLOADS) == 6 and WORKLOADS['7b_10min_1l'].total_tokens == 135272
+    assert len(WORKLOADS) == 7 and WORKLOADS['7b_10min_1l'].total_tokens == 135272
+    p = WORKLOADS['7b_10min_paper']
+    assert p.prune_layers == list(range(14, 28)) and p.seqs[0].n_q == 1 and p.joint_step_keep == 0.85
