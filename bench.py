@@ -155,6 +155,20 @@ class ClockSampler:
         return {"sm_mhz": mhz[len(mhz) // 2], "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(mhz)}
 
 
+def schedule_context(wl, pp):
+    """Analytic prefill-FLOPs ratio of the benchmarked inner-LLM schedule
+    (App. G, single sequence; the pre-LLM stage is not part of this path)."""
+    from paper_2608_08794_gb300 import flops as F
+    if wl.num_seqs != 1:
+        return None
+    model = F.QWEN25_OMNI_7B if wl.hidden == 3584 else F.QWEN25_OMNI_3B
+    if wl.num_layers != model.layers:
+        return None
+    sched = F.layer_schedule(wl.total_tokens, list(zip(wl.prune_layers, pp.t_out)), model)
+    return {"inner_llm_prefill_flops_ratio": F.flops_ratio(sched, wl.total_tokens, model),
+            "note": "App. G accounting of this schedule; the paper's 78% also includes pre-LLM compression"}
+
+
 # ----------------------------------------------------------------------------- CPU oracle leg
 
 ORACLE_SNIPPET = r"""
@@ -413,6 +427,7 @@ def main():
             "e2e": {"value": whole_job_value(mm_per_iter, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps},
             "clocks": clocks.summary() if clocks else None,
+            "context": schedule_context(wl, pp),
         }
         if world == 1 and not args.no_cpu_baseline:
             try:
