@@ -5,6 +5,7 @@ import this package.  The CUDA library never calls it, and it never calls the
 CUDA library: the two share no code.  See ``apack_oracle.py``.
 """
 
+from .prellm_oracle import frame_embeddings, window_cka, gate, frame_alignment  # noqa: F401
 from .apack_oracle import (  # noqa: F401
     MOD_OTHER, MOD_AUDIO, MOD_VISUAL,
     bf16_to_f64, relevance_scores, keep_count, step_keep_counts, select_keep,
