@@ -185,6 +185,28 @@ apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num
 apack_status apack_score_static(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
                                 float *scores, int32_t *device_error_out, void *stream);
 
+/* Pre-LLM frame alignment (Sec. 3.1, "Coarse pass" and "Gated fine pass";
+   Eq. cka and Eq. gate; Algorithm 1, its first pre-LLM steps).  Per video frame f:
+     v_f = mean of the frame's visual tokens; a_f = mean of the audio tokens
+           resampled onto the frame axis (audio token j belongs to frame
+           floor(j * n_frames / n_audio));
+     c_f = ||V_f^T A_f||_F^2 / (||A_f^T A_f||_F ||V_f^T V_f||_F), linear CKA of the
+           mean-centred window rows f - window/2 .. f + window/2 (cut to the clip;
+           0 for a window whose centred rows vanish);
+     s_f = c_f if mean(c) >= tau, else (1 - beta) c_f + beta (1 - dn_f), with
+           dn_f = the min-max normalised ||v_f - a_f|| over the clip.
+   visual: bf16 [n_frames * tokens_per_frame][dim], frame f's tokens at rows
+   f*tokens_per_frame ..; audio: bf16 [n_audio][dim]; dim a multiple of 8,
+   n_audio >= n_frames >= 1, window odd in 1..7 (the paper uses 3, tau = 0.78,
+   beta = 0.90).  Outputs (device, fp32): c_out [F], s_out [F], dnorm_out [F]
+   (nullable), cbar_out [1] (nullable).  fp32 accumulation, fixed reduction
+   order (deterministic).  ws: 256-byte aligned, apack_frame_alignment_workspace_size. */
+apack_status apack_frame_alignment_workspace_size(int32_t n_frames, int64_t dim, size_t *bytes);
+apack_status apack_frame_alignment(const void *visual, const void *audio, int32_t n_frames,
+                                   int32_t tokens_per_frame, int32_t n_audio, int64_t dim, int32_t window,
+                                   float tau, float beta, float *c_out, float *s_out, float *dnorm_out,
+                                   float *cbar_out, void *ws, size_t ws_bytes, void *stream);
+
 /* Synchronises `stream`, then reads the device error word of `ws` into
    *code_out (APACK_OK, APACK_ETIMEOUT or APACK_EDEVICE) and clears it when
    `clear` is non-zero. */

@@ -27,7 +27,7 @@ APACK_HEAD_DIM = 128
 
 EXPORTED = ("apack_workspace_size", "apack_keep_counts", "apack_score", "apack_select", "apack_compact",
             "apack_prune_step", "apack_device_error", "apack_launch_count", "apack_status_string",
-            "apack_score_static")
+            "apack_score_static", "apack_frame_alignment_workspace_size", "apack_frame_alignment")
 
 
 class ApackError(RuntimeError):
@@ -71,6 +71,9 @@ def _load():
                                      P(VP), VP]
     lib.apack_device_error.argtypes = [VP, VP, PI32, I32]
     lib.apack_score_static.argtypes = [P(apack_seqs), VP, VP, I64, VP, VP, VP]
+    lib.apack_frame_alignment_workspace_size.argtypes = [I32, I64, P(SZ)]
+    lib.apack_frame_alignment.argtypes = [VP, VP, I32, I32, I32, I64, I32, ctypes.c_float, ctypes.c_float, VP, VP,
+                                          VP, VP, VP, SZ, VP]
     lib.apack_launch_count.argtypes = []
     lib.apack_launch_count.restype = ctypes.c_uint64
     lib.apack_status_string.argtypes = [I32]
@@ -228,6 +231,22 @@ def apack_score_static(seqs, q, k, k_token_stride, scores, device_error_out=None
     memory (the library's fixed 8 MiB scratch array is used instead)."""
     _check(_lib.apack_score_static(seqs.ref(), _ptr(q), _ptr(k), int(k_token_stride), _ptr(scores),
                                    _ptr(device_error_out), _stream(stream)), "apack_score_static")
+
+
+def apack_frame_alignment_workspace_size(n_frames, dim):
+    n = ctypes.c_size_t(0)
+    _check(_lib.apack_frame_alignment_workspace_size(int(n_frames), int(dim), ctypes.byref(n)),
+           "apack_frame_alignment_workspace_size")
+    return n.value
+
+
+def apack_frame_alignment(visual, audio, n_frames, tokens_per_frame, n_audio, dim, c_out, s_out, ws, window=3,
+                          tau=0.78, beta=0.90, dnorm_out=None, cbar_out=None, stream=None):
+    """Pre-LLM windowed CKA c_f and gated score s_f per frame (Sec. 3.1)."""
+    _check(_lib.apack_frame_alignment(_ptr(visual), _ptr(audio), int(n_frames), int(tokens_per_frame), int(n_audio),
+                                      int(dim), int(window), float(tau), float(beta), _ptr(c_out), _ptr(s_out),
+                                      _ptr(dnorm_out), _ptr(cbar_out), _ptr(ws), ws.numel() * ws.element_size(),
+                                      _stream(stream)), "apack_frame_alignment")
 
 
 def apack_device_error(ws, stream=None, clear=True):
