@@ -262,6 +262,94 @@ def reference_arm(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+PRELLM_SNIPPET = r"""
+import json, sys, time
+sys.path.insert(0, {root!r})
+import oracle
+from synth.gen import normal_bf16_bits, TID_VIS_EMB, TID_AUD_EMB
+F, tpf, na, dim = {F}, {tpf}, {na}, {dim}
+vis = normal_bf16_bits({seed}, TID_VIS_EMB, 0, F * tpf * dim).reshape(F * tpf, dim)
+aud = normal_bf16_bits({seed}, TID_AUD_EMB, 0, na * dim).reshape(na, dim)
+t0 = time.perf_counter()
+oracle.frame_alignment(vis, aud, F, tpf)
+print(json.dumps(dict(seconds=time.perf_counter() - t0)))
+"""
+
+
+def prellm_shape(wl):
+    """Frames, visual tokens per frame, audio tokens and feature size of the
+    pre-LLM alignment of the workload's first sequence."""
+    s = wl.seqs[0]
+    return s.fps * s.duration_s, s.tpf, s.n_audio, wl.hidden
+
+
+def prellm_cpu_baseline(wl, frames=24):
+    F, tpf, na, dim = prellm_shape(wl)
+    fs = min(F, frames)
+    nas = max(fs, na * fs // F)
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = PRELLM_SNIPPET.format(root=ROOT, F=fs, tpf=tpf, na=nas, dim=dim, seed=wl.seed)
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env)
+    if r.returncode != 0:
+        raise RuntimeError(r.stderr[-2000:])
+    sec = json.loads(r.stdout.strip().splitlines()[-1])["seconds"]
+    return {"value": fs / sec, "unit": "frames/s", "cores": 1, "kind": "oracle",
+            "sample": f"{fs} frames x {tpf} visual tokens, {nas} audio tokens, d={dim}; single-threaded numpy "
+                      f"fp64 oracle (literal d x d products), {sec:.1f} s"}
+
+
+def prellm_measure(ap, wl, steps, warmup, stream, dist):
+    """Pre-LLM frame alignment (Sec. 3.1, Eq. cka and Eq. gate) of the
+    workload's clip: pooled frame embeddings, windowed CKA and the gate, one
+    apack_frame_alignment call per step.  The bf16 encoder tokens are read
+    once and exceed L2, so no flush is needed between calls."""
+    import torch
+    from synth.gen import TID_VIS_EMB, TID_AUD_EMB
+    from synth.device import fill_normal_bf16
+    F, tpf, na, dim = prellm_shape(wl)
+    vis = torch.empty(F * tpf, dim, dtype=torch.bfloat16, device="cuda")
+    aud = torch.empty(na, dim, dtype=torch.bfloat16, device="cuda")
+    fill_normal_bf16(vis, wl.seed, TID_VIS_EMB, stream=stream)
+    fill_normal_bf16(aud, wl.seed, TID_AUD_EMB, stream=stream)
+    ws = torch.empty(ap.apack_frame_alignment_workspace_size(F, dim), dtype=torch.uint8, device="cuda")
+    c = torch.empty(F, dtype=torch.float32, device="cuda")
+    sc = torch.empty_like(c)
+
+    def call():
+        ap.apack_frame_alignment(vis, aud, F, tpf, na, dim, c, sc, ws, stream=stream)
+
+    for _ in range(max(3, warmup)):
+        call()
+    torch.cuda.synchronize()
+    k = max(3, min(steps, 50))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n0 = ap.apack_launch_count()
+    e0.record(stream)
+    for _ in range(k):
+        call()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    launches = ap.apack_launch_count() - n0
+    ms = max_over_ranks(e0.elapsed_time(e1) / k, dist, "cuda")
+    token_bytes = (F * tpf + na) * dim * 2
+    frame_bytes = 2 * F * dim * 4
+    alg = token_bytes + frame_bytes
+    achieved = alg / (ms / 1e3) / 1e9
+    peak, peak_kind = measured_peaks()
+    del vis, aud, ws
+    return {"metric": "frames aligned per second", "value": F / (ms / 1e3), "unit": "frames/s",
+            "ms_per_clip": ms, "steps": k, "gpu_launches": int(launches),
+            "config": {"workload": f"{wl.name} clip: {F} frames x {tpf} visual tokens, {na} audio tokens, d={dim}",
+                       "window": 3, "tau": 0.78, "beta": 0.90,
+                       "l2": "inputs larger than L2 (%.2f GB of bf16 encoder tokens)" % (token_bytes / 1e9)},
+            "roofline": {"bound": "hbm", "kernel": "apack_frame_alignment call (frame_pool_kernel + "
+                                                   "frame_cka_kernel + frame_gate_kernel)",
+                         "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": None, "peak_source": peak_kind,
+                         "algorithmic_bytes_per_launch": alg,
+                         "note": "bf16 tokens read once + fp32 frame embeddings written once, over the whole call"}}
+
+
 # ----------------------------------------------------------------------------- GPU leg
 
 def main():
@@ -394,6 +482,9 @@ def main():
         clocks.stop()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dist, "cuda")
 
+    # the pre-LLM stage of the same clip, timed on its own after the prune steps
+    prellm = prellm_measure(ap, wl, args.steps, args.warmup, stream, dist)
+
     if rank == 0:
         per_step_ms = ms / args.steps
         value = whole_job_value(mm_per_iter, world, per_step_ms)
@@ -429,11 +520,16 @@ def main():
             "clocks": clocks.summary() if clocks else None,
             "context": schedule_context(wl, pp),
         }
+        line["prellm_alignment"] = prellm
         if world == 1 and not args.no_cpu_baseline:
             try:
                 line["cpu_baseline"] = cpu_baseline(args.workload)
             except Exception as exc:  # report, do not hide
                 line["cpu_baseline"] = {"value": None, "error": str(exc)[-300:]}
+            try:
+                prellm["cpu_baseline"] = prellm_cpu_baseline(wl)
+            except Exception as exc:
+                prellm["cpu_baseline"] = {"value": None, "error": str(exc)[-300:]}
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()

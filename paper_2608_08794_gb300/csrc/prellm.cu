@@ -10,9 +10,12 @@
 //                the feature dimension, which gives Eq. cka exactly since
 //                ||V^T A||_F^2 = <K_A, K_V>_F and ||A^T A||_F = ||K_A||_F; also the
 //                direct distance d_f = ||v_f - a_f||.
-//  gate kernel:  one CTA: c-bar, min/max of d, the min-max normalised distance and the
-//                gated score s_f of Eq. gate (blend when c-bar < tau).
-// All reductions run in a fixed order: results are deterministic.
+//  gate:         the last CTA of the CKA kernel to finish (a counter in the workspace,
+//                zeroed by the pool kernel) computes c-bar, min/max of d, the min-max
+//                normalised distance and the gated score s_f of Eq. gate (blend when
+//                c-bar < tau) over the whole clip.
+// All reductions run in a fixed order: results are deterministic.  Two launches per call.
+#include <algorithm>
 #include <cmath>
 
 #include "internal.cuh"
@@ -21,11 +24,9 @@ namespace apack {
 
 namespace {
 
-constexpr int kPoolThreads = 256;      // 8 features per thread: 2048 features per CTA
+constexpr int kPoolMaxThreads = 512;   // 8 features per thread: up to 4096 features per CTA
 constexpr int kCkaThreads = 256;
 constexpr int kMaxWindow = 7;
-constexpr int kGram = kMaxWindow * (kMaxWindow + 1) / 2;   // upper triangle of a w x w Gram
-constexpr int kGateThreads = 1024;
 
 __device__ __forceinline__ void add_bf16x8(const uint4 &v, float (&acc)[8]) {
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -36,17 +37,19 @@ __device__ __forceinline__ void add_bf16x8(const uint4 &v, float (&acc)[8]) {
   }
 }
 
-__global__ void __launch_bounds__(kPoolThreads)
+__global__ void __launch_bounds__(kPoolMaxThreads, 2)
     frame_pool_kernel(const uint4 *__restrict__ visual, const uint4 *__restrict__ audio, int n_frames, int tpf,
-                      int n_audio, int64_t dim, float *__restrict__ v_out, float *__restrict__ a_out) {
+                      int n_audio, int64_t dim, float *__restrict__ v_out, float *__restrict__ a_out,
+                      unsigned int *done) {
   const int f = blockIdx.x;
-  const int64_t fi = (static_cast<int64_t>(blockIdx.y) * kPoolThreads + threadIdx.x) * 8;
+  if (f == 0 && blockIdx.y == 0 && threadIdx.x == 0) *done = 0u;   // CTA counter of the CKA kernel
+  const int64_t fi = (static_cast<int64_t>(blockIdx.y) * blockDim.x + threadIdx.x) * 8;
   if (fi >= dim) return;
   const int64_t vec_per_row = dim / 8;
   const int64_t col = fi / 8;
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   const int64_t r0 = static_cast<int64_t>(f) * tpf;
-#pragma unroll 4
+#pragma unroll 8
   for (int t = 0; t < tpf; ++t) add_bf16x8(__ldg(visual + (r0 + t) * vec_per_row + col), acc);
   const float inv_v = 1.f / static_cast<float>(tpf);
 #pragma unroll
@@ -56,115 +59,130 @@ __global__ void __launch_bounds__(kPoolThreads)
   const int64_t j1 = (static_cast<int64_t>(f + 1) * n_audio + n_frames - 1) / n_frames;
 #pragma unroll
   for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-#pragma unroll 4
+#pragma unroll 8
   for (int64_t j = j0; j < j1; ++j) add_bf16x8(__ldg(audio + j * vec_per_row + col), acc);
   const float inv_a = 1.f / static_cast<float>(j1 - j0);
 #pragma unroll
   for (int i = 0; i < 8; ++i) a_out[static_cast<int64_t>(f) * dim + fi + i] = acc[i] * inv_a;
 }
 
+// Per-frame windowed CKA (Eq. cka) and direct distance; the last CTA to finish also
+// runs the gate (Eq. gate) over all frames.  W is the window size (odd, <= kMaxWindow);
+// windows cut by the clip's ends hold w < W rows and the missing rows are zeros that
+// never enter a Gram entry with i or j >= w.
+template <int W>
 __global__ void __launch_bounds__(kCkaThreads)
-    frame_cka_kernel(const float *__restrict__ v, const float *__restrict__ a, int n_frames, int64_t dim, int window,
-                     float *__restrict__ c_out, float *__restrict__ d_out) {
-  __shared__ float red[kCkaThreads / 32][2 * kGram + 1];
+    frame_cka_gate_kernel(const float *__restrict__ v, const float *__restrict__ a, int n_frames, int64_t dim,
+                          float tau, float beta, unsigned int *done, float *__restrict__ c_out,
+                          float *__restrict__ d_out, float *__restrict__ s_out, float *__restrict__ dn_out,
+                          float *__restrict__ cbar_out) {
+  constexpr int kG = W * (W + 1) / 2;
+  constexpr int kN = 2 * kG + 1;
+  constexpr int kWarps = kCkaThreads / 32;
+  __shared__ float red[kWarps][kN];
+  __shared__ float tot[kN];
+  __shared__ bool last;
   const int f = blockIdx.x;
-  const int half = window / 2;
-  const int lo = max(0, f - half), hi = min(n_frames, f + half + 1);
+  const int lo = max(0, f - W / 2), hi = min(n_frames, f + W / 2 + 1);
   const int w = hi - lo;
   const int center = f - lo;
-  float ga[kGram], gv[kGram], dist = 0.f;
+  const float inv_w = 1.f / static_cast<float>(w);
+  float ga[kG], gv[kG], dist = 0.f;
 #pragma unroll
-  for (int i = 0; i < kGram; ++i) ga[i] = gv[i] = 0.f;
+  for (int i = 0; i < kG; ++i) ga[i] = gv[i] = 0.f;
   for (int64_t x = threadIdx.x; x < dim; x += kCkaThreads) {
-    float av[kMaxWindow], vv[kMaxWindow], am = 0.f, vm = 0.f;
+    float av[W], vv[W], am = 0.f, vm = 0.f, dd = 0.f;
 #pragma unroll
-    for (int r = 0; r < kMaxWindow; ++r) {
+    for (int r = 0; r < W; ++r) {
       av[r] = r < w ? a[static_cast<int64_t>(lo + r) * dim + x] : 0.f;
       vv[r] = r < w ? v[static_cast<int64_t>(lo + r) * dim + x] : 0.f;
       am += av[r];
       vm += vv[r];
+      if (r == center) dd = vv[r] - av[r];
     }
-    {
-      const float dd = vv[center] - av[center];
-      dist = fmaf(dd, dd, dist);
-    }
-    am /= static_cast<float>(w);
-    vm /= static_cast<float>(w);
+    dist = fmaf(dd, dd, dist);
+    am *= inv_w;
+    vm *= inv_w;
 #pragma unroll
-    for (int r = 0; r < kMaxWindow; ++r) {
+    for (int r = 0; r < W; ++r) {
       av[r] = r < w ? av[r] - am : 0.f;
       vv[r] = r < w ? vv[r] - vm : 0.f;
     }
     int k = 0;
 #pragma unroll
-    for (int i = 0; i < kMaxWindow; ++i)
+    for (int i = 0; i < W; ++i)
 #pragma unroll
-      for (int j = i; j < kMaxWindow; ++j, ++k) {
+      for (int j = i; j < W; ++j, ++k) {
         ga[k] = fmaf(av[i], av[j], ga[k]);
         gv[k] = fmaf(vv[i], vv[j], gv[k]);
       }
   }
-  // block reduction of the 2 * kGram + 1 sums (warp tree, then warps in order)
+  // fixed-order block reduction: warp trees, then one thread per sum over the warps in order
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
-  for (int i = 0; i < kGram; ++i) {
+  for (int i = 0; i < kG; ++i) {
+#pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       ga[i] += __shfl_xor_sync(0xffffffffu, ga[i], o);
       gv[i] += __shfl_xor_sync(0xffffffffu, gv[i], o);
     }
   }
+#pragma unroll
   for (int o = 16; o > 0; o >>= 1) dist += __shfl_xor_sync(0xffffffffu, dist, o);
   if (lane == 0) {
 #pragma unroll
-    for (int i = 0; i < kGram; ++i) {
+    for (int i = 0; i < kG; ++i) {
       red[warp][i] = ga[i];
-      red[warp][kGram + i] = gv[i];
+      red[warp][kG + i] = gv[i];
     }
-    red[warp][2 * kGram] = dist;
+    red[warp][2 * kG] = dist;
+  }
+  __syncthreads();
+  if (threadIdx.x < kN) {
+    float t = 0.f;
+#pragma unroll
+    for (int wp = 0; wp < kWarps; ++wp) t += red[wp][threadIdx.x];
+    tot[threadIdx.x] = t;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    double sa[kGram], sv[kGram], sd = 0.0;
-    for (int i = 0; i < kGram; ++i) {
-      sa[i] = sv[i] = 0.0;
-      for (int wp = 0; wp < kCkaThreads / 32; ++wp) {
-        sa[i] += red[wp][i];
-        sv[i] += red[wp][kGram + i];
-      }
-    }
-    for (int wp = 0; wp < kCkaThreads / 32; ++wp) sd += red[wp][2 * kGram];
-    // <K_A, K_V>_F, ||K_A||_F^2, ||K_V||_F^2 from the upper triangles
-    double dot = 0.0, na = 0.0, nv = 0.0;
+    // <K_A, K_V>_F, ||K_A||_F^2 and ||K_V||_F^2 from the upper triangles (off-diagonal entries twice)
+    float dot = 0.f, na = 0.f, nv = 0.f;
     int k = 0;
-    for (int i = 0; i < kMaxWindow; ++i)
-      for (int j = i; j < kMaxWindow; ++j, ++k) {
-        if (i >= w || j >= w) continue;
-        const double m = (i == j) ? 1.0 : 2.0;
-        dot += m * sa[k] * sv[k];
-        na += m * sa[k] * sa[k];
-        nv += m * sv[k] * sv[k];
+#pragma unroll
+    for (int i = 0; i < W; ++i)
+#pragma unroll
+      for (int j = i; j < W; ++j, ++k) {
+        const float m = (i == j) ? 1.f : 2.f;
+        dot = fmaf(m * tot[k], tot[kG + k], dot);
+        na = fmaf(m * tot[k], tot[k], na);
+        nv = fmaf(m * tot[kG + k], tot[kG + k], nv);
       }
-    const double den = sqrt(na) * sqrt(nv);
-    c_out[f] = den > 0.0 ? static_cast<float>(dot / den) : 0.f;
-    d_out[f] = static_cast<float>(sqrt(sd));
+    const float den = sqrtf(na) * sqrtf(nv);
+    c_out[f] = den > 0.f ? dot / den : 0.f;
+    d_out[f] = sqrtf(tot[2 * kG]);
+    __threadfence();
+    last = atomicAdd(done, 1u) == static_cast<unsigned>(n_frames - 1);
   }
-}
-
-__global__ void __launch_bounds__(kGateThreads)
-    frame_gate_kernel(const float *__restrict__ c, const float *__restrict__ d, int n_frames, float tau, float beta,
-                      float *__restrict__ s_out, float *__restrict__ dn_out, float *__restrict__ cbar_out) {
-  __shared__ double rsum[kGateThreads / 32];
-  __shared__ float rmin[kGateThreads / 32], rmax[kGateThreads / 32];
+  __syncthreads();
+  if (!last) return;
+  // gate over the whole clip (every other CTA's c and d are visible after its fence)
+  __threadfence();
+  __shared__ double rsum[kWarps];
+  __shared__ float rmin[kWarps], rmax[kWarps];
   __shared__ double cbar_s;
   __shared__ float dmin_s, dmax_s;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const volatile float *cv = c_out;
+  const volatile float *dv = d_out;
   double cs = 0.0;
   float mn = INFINITY, mx = -INFINITY;
-  for (int f = threadIdx.x; f < n_frames; f += kGateThreads) {
-    cs += c[f];
-    mn = fminf(mn, d[f]);
-    mx = fmaxf(mx, d[f]);
+  for (int g = threadIdx.x; g < n_frames; g += kCkaThreads) {
+    cs += cv[g];
+    const float dg = dv[g];
+    mn = fminf(mn, dg);
+    mx = fmaxf(mx, dg);
   }
+#pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     cs += __shfl_xor_sync(0xffffffffu, cs, o);
     mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
@@ -178,24 +196,25 @@ __global__ void __launch_bounds__(kGateThreads)
   __syncthreads();
   if (threadIdx.x == 0) {
     double t = 0.0;
-    float a = INFINITY, b = -INFINITY;
-    for (int wp = 0; wp < kGateThreads / 32; ++wp) {
+    float lo_d = INFINITY, hi_d = -INFINITY;
+    for (int wp = 0; wp < kWarps; ++wp) {
       t += rsum[wp];
-      a = fminf(a, rmin[wp]);
-      b = fmaxf(b, rmax[wp]);
+      lo_d = fminf(lo_d, rmin[wp]);
+      hi_d = fmaxf(hi_d, rmax[wp]);
     }
     cbar_s = t / n_frames;
-    dmin_s = a;
-    dmax_s = b;
+    dmin_s = lo_d;
+    dmax_s = hi_d;
     if (cbar_out) *cbar_out = static_cast<float>(cbar_s);
   }
   __syncthreads();
   const bool blend = cbar_s < static_cast<double>(tau);
   const float span = dmax_s - dmin_s;
-  for (int f = threadIdx.x; f < n_frames; f += kGateThreads) {
-    const float dn = span > 0.f ? (d[f] - dmin_s) / span : 0.f;
-    if (dn_out) dn_out[f] = dn;
-    s_out[f] = blend ? (1.f - beta) * c[f] + beta * (1.f - dn) : c[f];
+  for (int g = threadIdx.x; g < n_frames; g += kCkaThreads) {
+    const float cg = cv[g];
+    const float dn = span > 0.f ? (dv[g] - dmin_s) / span : 0.f;
+    if (dn_out) dn_out[g] = dn;
+    s_out[g] = blend ? (1.f - beta) * cg + beta * (1.f - dn) : cg;
   }
 }
 
@@ -232,19 +251,37 @@ apack_status apack_frame_alignment(const void *visual, const void *audio, int32_
   apack_frame_alignment_workspace_size(n_frames, dim, &need);
   if (ws_bytes < need) return APACK_EWORKSPACE;
   uint8_t *w = static_cast<uint8_t *>(ws);
+  unsigned int *done = reinterpret_cast<unsigned int *>(w);
   float *vbuf = reinterpret_cast<float *>(w + 256);
   float *abuf = reinterpret_cast<float *>(w + 256 + up(static_cast<size_t>(n_frames) * dim * sizeof(float)));
   float *dbuf = reinterpret_cast<float *>(w + 256 + 2 * up(static_cast<size_t>(n_frames) * dim * sizeof(float)));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  dim3 pgrid(n_frames, static_cast<unsigned>((dim + kPoolThreads * 8 - 1) / (kPoolThreads * 8)));
-  frame_pool_kernel<<<pgrid, kPoolThreads, 0, s>>>(static_cast<const uint4 *>(visual), static_cast<const uint4 *>(audio),
-                                                  n_frames, tokens_per_frame, n_audio, dim, vbuf, abuf);
+  // one CTA per frame covers up to 4096 features; wider rows take more CTAs per frame
+  const int64_t vecs = dim / 8;
+  const int pthreads = static_cast<int>(std::min<int64_t>(kPoolMaxThreads, (vecs + 31) / 32 * 32));
+  dim3 pgrid(n_frames, static_cast<unsigned>((vecs + pthreads - 1) / pthreads));
+  frame_pool_kernel<<<pgrid, pthreads, 0, s>>>(static_cast<const uint4 *>(visual), static_cast<const uint4 *>(audio),
+                                              n_frames, tokens_per_frame, n_audio, dim, vbuf, abuf, done);
   count_launches(1);
   if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
-  frame_cka_kernel<<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, window, c_out, dbuf);
-  count_launches(1);
-  if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
-  frame_gate_kernel<<<1, kGateThreads, 0, s>>>(c_out, dbuf, n_frames, tau, beta, s_out, dnorm_out, cbar_out);
+  switch (window) {
+    case 1:
+      frame_cka_gate_kernel<1><<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, tau, beta, done, c_out,
+                                                                dbuf, s_out, dnorm_out, cbar_out);
+      break;
+    case 3:
+      frame_cka_gate_kernel<3><<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, tau, beta, done, c_out,
+                                                                dbuf, s_out, dnorm_out, cbar_out);
+      break;
+    case 5:
+      frame_cka_gate_kernel<5><<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, tau, beta, done, c_out,
+                                                                dbuf, s_out, dnorm_out, cbar_out);
+      break;
+    default:
+      frame_cka_gate_kernel<7><<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, tau, beta, done, c_out,
+                                                                dbuf, s_out, dnorm_out, cbar_out);
+      break;
+  }
   count_launches(1);
   if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
   return APACK_OK;

@@ -28,6 +28,8 @@ TID_HIDDEN = 4000   # hidden states
 TID_PLANT = 5000    # which tokens are planted
 TID_RAGGED = 6000   # per-sequence draws of the ragged batch
 TID_POS = 7000      # position ids
+TID_VIS_EMB = 8000  # visual encoder embeddings (pre-LLM alignment)
+TID_AUD_EMB = 8001  # audio encoder embeddings (pre-LLM alignment)
 
 _M64 = np.uint64(0xFFFFFFFFFFFFFFFF)
 _GOLDEN = np.uint64(0x9E3779B97F4A7C15)

@@ -28,7 +28,7 @@ def run(ap, vis, aud, F, tpf, dim, window, tau, beta):
     v_d = torch.from_numpy(vis.view(np.int16)).cuda()
     a_d = torch.from_numpy(aud.view(np.int16)).cuda()
     n = ap.apack_frame_alignment_workspace_size(F, dim)
-    ws = torch.zeros(n + 256, dtype=torch.uint8, device="cuda")
+    ws = torch.full((n + 256,), 0xA5, dtype=torch.uint8, device="cuda")   # no zeroed workspace needed
     off = (-ws.data_ptr()) % 256
     ws = ws[off:off + n]
     c = torch.empty(F, dtype=torch.float32, device="cuda")
@@ -42,9 +42,9 @@ def run(ap, vis, aud, F, tpf, dim, window, tau, beta):
 
 
 def inputs(seed, F, tpf, n_audio, dim):
-    from synth.gen import normal_bf16_bits
-    vis = normal_bf16_bits(seed, 8000, 0, F * tpf * dim).reshape(F * tpf, dim)
-    aud = normal_bf16_bits(seed, 8001, 0, n_audio * dim).reshape(n_audio, dim)
+    from synth.gen import normal_bf16_bits, TID_VIS_EMB, TID_AUD_EMB
+    vis = normal_bf16_bits(seed, TID_VIS_EMB, 0, F * tpf * dim).reshape(F * tpf, dim)
+    aud = normal_bf16_bits(seed, TID_AUD_EMB, 0, n_audio * dim).reshape(n_audio, dim)
     return vis, aud
 
 
