@@ -73,10 +73,10 @@ def measured_peaks():
     return FALLBACK_HBM_GBS, "fallback"
 
 
-def profiled_traffic(kernel_src):
-    """DRAM bytes per launch of the compaction kernel from the committed ncu
-    summary, if it was taken on the current kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", "gather_tma_traffic.json")
+def profiled_traffic(kernel_src, summary="gather_tma_traffic.json"):
+    """DRAM bytes of a profiled launch from a committed ncu summary, if it was
+    taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", summary)
     if not os.path.exists(path):
         return None
     with open(path) as f:
@@ -336,6 +336,8 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
     alg = token_bytes + frame_bytes
     achieved = alg / (ms / 1e3) / 1e9
     peak, peak_kind = measured_peaks()
+    prof = profiled_traffic("prellm.cu", "prellm_traffic.json")
+    traffic = int(prof["traffic_over_algorithmic"] * alg) if prof is not None else None
     del vis, aud, ws
     return {"metric": "frames aligned per second", "value": F / (ms / 1e3), "unit": "frames/s",
             "ms_per_clip": ms, "steps": k, "gpu_launches": int(launches),
@@ -343,9 +345,9 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
                        "window": 3, "tau": 0.78, "beta": 0.90,
                        "l2": "inputs larger than L2 (%.2f GB of bf16 encoder tokens)" % (token_bytes / 1e9)},
             "roofline": {"bound": "hbm", "kernel": "apack_frame_alignment call (frame_pool_kernel + "
-                                                   "frame_cka_kernel + frame_gate_kernel)",
+                                                   "frame_cka_gate_kernel)",
                          "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                         "traffic": None, "peak_source": peak_kind,
+                         "traffic": traffic, "peak_source": peak_kind,
                          "algorithmic_bytes_per_launch": alg,
                          "note": "bf16 tokens read once + fp32 frame embeddings written once, over the whole call"}}
 

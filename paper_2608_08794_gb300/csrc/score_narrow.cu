@@ -4,12 +4,16 @@
 //
 // With so few rows the step is bound by reading K from HBM, not by arithmetic, so
 // this path uses CUDA cores and reads K once:
-//   logits kernel:  one thread per key reads its whole token row (all KV heads,
-//                   16-byte loads) and dots it with the group's query rows held in
-//                   shared memory (fp32 FMA of exactly widened bf16); it stores the
-//                   log2-domain logits x * log2(e)/sqrt(D) (row-major per logit row,
-//                   key-contiguous) and per-CTA (max, sum of exp2) of every logit row
-//                   over the multimodal keys of its tile;
+//   logits kernel:  log2-domain logits x * log2(e)/sqrt(D) of every (logit row, key),
+//                   stored per logit row with a row stride padded to 64 keys, and per
+//                   CTA (max, sum of exp2) of every logit row over the multimodal keys of
+//                   its tile.  Two variants:
+//                   * rows8 (Hkv = 2 or 4, at most 8 rows per head group): a warp reads
+//                     token rows coalesced, 16 lanes per KV head with 8 features each,
+//                     holds its query slice in registers, and an 8-row reduce-scatter
+//                     over the 16 lanes leaves one finished logit per lane pair;
+//                   * general: one thread per key reads its whole token row and dots it
+//                     with the group's query rows held in shared memory;
 //   merge kernel:   per logit row, one block combines the CTA partials into lse2;
 //   final kernel:   one thread per key sums exp2(logit - lse2) over all logit rows
 //                   in a fixed order and scales by 1/(Hq n_q).
@@ -24,22 +28,28 @@ namespace apack {
 
 namespace {
 
-constexpr int kThreads = 256;          // keys per CTA
+constexpr int kThreads = 256;          // keys per CTA (general logits kernel, final kernel)
 constexpr int kWarps = kThreads / 32;
+constexpr int kRows8Tokens = 64;       // keys per CTA of the rows8 logits kernel
+constexpr int kLogitPad = 64;          // logit row stride: the key count rounded up to this
 
 struct NSeq {
   int32_t t0, len;
   int32_t q_off, n_q;
-  int32_t unit_begin;                  // first CTA of this sequence in the launch
+  int32_t unit_begin;                  // first 256-key CTA of this sequence (general logits, final)
+  int32_t unit8_begin;                 // first CTA of this sequence in the rows8 logits kernel
+  int32_t nparts;                      // CTA partials of the logits kernel in use
   int32_t rows;                        // logit rows R = Hq * n_q
-  int64_t logit_base;                  // float offset of this sequence's logits [R][len]
-  int64_t part_base;                   // float2 offset of its CTA partials [ctas][R]
+  int64_t lstride;                     // logit row stride: len rounded up to kLogitPad
+  int64_t logit_base;                  // float offset of this sequence's logits [R][lstride]
+  int64_t part_base;                   // float2 offset of its CTA partials [nparts][R]
   int64_t lse_base;                    // float offset of its lse2 [R]
 };
 
 struct NarrowPlan {
   int32_t nseq;
   int32_t total_units;
+  int32_t total_units8;
   int32_t hq, hkv, group;
   float scale2;
   NSeq seq[kSeqsPerLaunch];
@@ -48,6 +58,12 @@ struct NarrowPlan {
 __device__ __forceinline__ int find_unit_seq(const NarrowPlan &p, int u) {
   int s = 0;
   while (s + 1 < p.nseq && p.seq[s + 1].unit_begin <= u) ++s;
+  return s;
+}
+
+__device__ __forceinline__ int find_unit8_seq(const NarrowPlan &p, int u) {
+  int s = 0;
+  while (s + 1 < p.nseq && p.seq[s + 1].unit8_begin <= u) ++s;
   return s;
 }
 
@@ -132,7 +148,7 @@ __global__ void __launch_bounds__(kThreads)
       if (l < rg) {
         const int rho = qoff[l] / 128;
         const float y = acc[l] * plan.scale2;
-        if (in) logits[lbase + static_cast<int64_t>(rho) * sq.len] = y;
+        if (in) logits[lbase + static_cast<int64_t>(rho) * sq.lstride] = y;
         // this warp's (max, sum of exp2) of the row over its multimodal keys
         const float wm = warp_max(mm ? y : -INFINITY);
         const float ws = warp_sum(mm && wm != -INFINITY ? ex2_approx(y - wm) : 0.f);
@@ -154,6 +170,132 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
+// rows8 logits kernel: KV heads in pairs, a warp per (head pair, run of tokens).  Lane
+// l works on head 2 hp + (l >> 4) and features [8 (l & 15), 8 (l & 15) + 8) of it.
+// NPAIR = Hkv / 2 head pairs; a CTA covers kRows8Tokens keys.
+template <int NPAIR>
+__global__ void __launch_bounds__(kThreads, 2)
+    score_narrow_rows8_kernel(const __grid_constant__ NarrowPlan plan, const uint16_t *__restrict__ q,
+                              const uint8_t *__restrict__ k, int64_t k_stride, const uint8_t *__restrict__ modality,
+                              float *__restrict__ logits, float2 *__restrict__ part) {
+  constexpr int kTokensPerWarp = kRows8Tokens * NPAIR / kWarps;   // 8 or 16
+  __shared__ float2 wst[kWarps][16];
+  const int s = find_unit8_seq(plan, blockIdx.x);
+  const NSeq &sq = plan.seq[s];
+  const int G = plan.group;
+  const int rg = G * sq.n_q;
+  if (rg == 0) return;                                   // no query row: nothing to score
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int hp = warp % NPAIR, tb = warp / NPAIR;
+  const int h = 2 * hp + (lane >> 4), part16 = lane & 15;
+  // query slice: rows j < rg of head group h (logit row (j / G) Hq + h G + j % G)
+  float qf[8][8];
+  const uint4 *qrow = reinterpret_cast<const uint4 *>(q + static_cast<int64_t>(sq.q_off) * plan.hq * 128);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    uint4 w = make_uint4(0, 0, 0, 0);
+    if (j < rg) w = __ldg(qrow + ((j / G) * plan.hq + h * G + j % G) * 16 + part16);
+    bf16x8_to_f32(w, qf[j]);
+  }
+  const int r = (lane >> 1) & 7;                       // row this lane holds after the reduce-scatter
+  const bool row_ok = r < rg;
+  const int rho = row_ok ? (r / G) * plan.hq + h * G + r % G : 0;
+  const bool b1 = lane & 8, b2 = lane & 4, b3 = lane & 2;
+  const int unit = blockIdx.x - sq.unit8_begin;
+  const int tok0 = unit * kRows8Tokens + tb * kTokensPerWarp;
+  const uint8_t *kbase = k + static_cast<int64_t>(sq.t0) * k_stride + h * 256 + part16 * 16;
+  float m = -INFINITY, ssum = 0.f;
+#pragma unroll 1
+  for (int c0 = 0; c0 < kTokensPerWarp; c0 += 8) {
+    uint4 kv[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int t = tok0 + c0 + i;
+      kv[i] = t < sq.len ? __ldg(reinterpret_cast<const uint4 *>(kbase + static_cast<int64_t>(t) * k_stride))
+                         : make_uint4(0, 0, 0, 0);
+    }
+    const int tl = tok0 + c0 + (lane & 7);
+    const unsigned mmask = __ballot_sync(0xffffffffu, lane < 8 && tl < sq.len && is_mm(modality[sq.t0 + tl]));
+    float outv[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      float kf[8];
+      bf16x8_to_f32(kv[i], kf);
+      float acc[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        float2 a = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          a = ffma2(make_float2(kf[2 * e], kf[2 * e + 1]), make_float2(qf[j][2 * e], qf[j][2 * e + 1]), a);
+        acc[j] = a.x + a.y;
+      }
+      // reduce-scatter over the 16 lanes of the head: lane bits 3, 2, 1 pick the row
+      float v4[4], v2[2];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float send = b1 ? acc[e] : acc[e + 4];
+        const float keep = b1 ? acc[e + 4] : acc[e];
+        v4[e] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+      }
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const float send = b2 ? v4[e] : v4[e + 2];
+        const float keep = b2 ? v4[e + 2] : v4[e];
+        v2[e] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+      }
+      float v1;
+      {
+        const float send = b3 ? v2[0] : v2[1];
+        const float keep = b3 ? v2[1] : v2[0];
+        v1 = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+      }
+      v1 += __shfl_xor_sync(0xffffffffu, v1, 1);
+      outv[i] = v1 * plan.scale2;
+    }
+    // running (max, sum of exp2) of this lane's row over the chunk's multimodal keys
+    float cm = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      if ((mmask >> i) & 1u) cm = fmaxf(cm, outv[i]);
+    if (cm != -INFINITY) {
+      if (cm > m) {
+        ssum *= ex2_approx(m - cm);
+        m = cm;
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        if ((mmask >> i) & 1u) ssum += ex2_approx(outv[i] - m);
+    }
+    if (row_ok) {   // the lane pair writes the chunk's 8 logits of its row: 4 each
+      const bool odd = lane & 1;
+      const float4 w = odd ? make_float4(outv[4], outv[5], outv[6], outv[7])
+                           : make_float4(outv[0], outv[1], outv[2], outv[3]);
+      *reinterpret_cast<float4 *>(logits + sq.logit_base + static_cast<int64_t>(rho) * sq.lstride + tok0 + c0 +
+                                  (odd ? 4 : 0)) = w;
+    }
+  }
+  if ((lane & 1) == 0) wst[warp][lane >> 1] = make_float2(m, ssum);
+  __syncthreads();
+  // per (head, row): combine the warps of its head pair in token order
+  if (threadIdx.x < 16 * NPAIR) {
+    const int php = threadIdx.x >> 4, slot = threadIdx.x & 15;
+    const int rr = slot & 7, hh = 2 * php + (slot >> 3);
+    if (rr < rg) {
+      float mx = -INFINITY;
+      for (int b = 0; b < kWarps / NPAIR; ++b) mx = fmaxf(mx, wst[b * NPAIR + php][slot].x);
+      float sum = 0.f;
+      if (mx != -INFINITY)
+        for (int b = 0; b < kWarps / NPAIR; ++b) {
+          const float2 v = wst[b * NPAIR + php][slot];
+          if (v.x != -INFINITY) sum += v.y * ex2_approx(v.x - mx);
+        }
+      const int rh = (rr / G) * plan.hq + hh * G + rr % G;
+      part[sq.part_base + static_cast<int64_t>(unit) * sq.rows + rh] = make_float2(mx, sum);
+    }
+  }
+}
+
 // One block per (sequence, logit row): lse2 over the CTA partials.  Each thread
 // folds a fixed stride of partials, then a fixed-shape tree combines the
 // threads: the order never depends on timing, so lse2 is deterministic.
@@ -168,7 +310,7 @@ __global__ void __launch_bounds__(kThreads)
   while (s + 1 < plan.nseq && acc + plan.seq[s].rows <= e) acc += plan.seq[s++].rows;
   const NSeq &sq = plan.seq[s];
   const int rho = static_cast<int>(e - acc);
-  const int ctas = (sq.len + kThreads - 1) / kThreads;
+  const int ctas = sq.nparts;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   float m = -INFINITY;
   for (int c = tid; c < ctas; c += kThreads) m = fmaxf(m, part[sq.part_base + static_cast<int64_t>(c) * sq.rows + rho].x);
@@ -220,10 +362,10 @@ __global__ void __launch_bounds__(kThreads)
     float a0 = 0.f, a1 = 0.f;
     int rho = 0;
     for (; rho + 1 < R; rho += 2) {
-      a0 += ex2_approx(lp[static_cast<int64_t>(rho) * sq.len] - ls[rho]);
-      a1 += ex2_approx(lp[static_cast<int64_t>(rho + 1) * sq.len] - ls[rho + 1]);
+      a0 += ex2_approx(lp[static_cast<int64_t>(rho) * sq.lstride] - ls[rho]);
+      a1 += ex2_approx(lp[static_cast<int64_t>(rho + 1) * sq.lstride] - ls[rho + 1]);
     }
-    if (rho < R) a0 += ex2_approx(lp[static_cast<int64_t>(rho) * sq.len] - ls[rho]);
+    if (rho < R) a0 += ex2_approx(lp[static_cast<int64_t>(rho) * sq.lstride] - ls[rho]);
     out = (a0 + a1) / static_cast<float>(plan.hq * sq.n_q);
   }
   scores[key] = out;
@@ -259,8 +401,8 @@ void narrow_layout(const apack_seqs *s, size_t *logit_floats, size_t *part_float
   for (int b = 0; b < s->num_seqs; ++b) {
     const int64_t len = s->cu_seqlens_h[b + 1] - s->cu_seqlens_h[b];
     const int64_t R = static_cast<int64_t>(s->num_q_heads) * (s->cu_qlens_h[b + 1] - s->cu_qlens_h[b]);
-    lf += static_cast<size_t>(R * len);
-    pf += static_cast<size_t>(R * ((len + kThreads - 1) / kThreads));
+    lf += static_cast<size_t>(R * ((len + kLogitPad - 1) / kLogitPad * kLogitPad));
+    pf += static_cast<size_t>(R * ((len + kRows8Tokens - 1) / kRows8Tokens));   // enough for either kernel
     ef += static_cast<size_t>(R);
   }
   *logit_floats = lf;
@@ -286,7 +428,14 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
     P.hkv = hkv;
     P.group = G;
     P.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(APACK_HEAD_DIM)));
-    int units = 0, max_rows = 0, max_rg = 0;
+    // rows8 kernel: K read by whole warps, query slice in registers
+    int max_rg = 0;
+    for (int i = 0; i < ns; ++i) {
+      const int nq = seqs->cu_qlens_h[s0 + i + 1] - seqs->cu_qlens_h[s0 + i];
+      max_rg = G * nq > max_rg ? G * nq : max_rg;
+    }
+    const bool rows8 = (hkv == 2 || hkv == 4) && max_rg <= 8;
+    int units = 0, units8 = 0, max_rows = 0;
     int64_t rows_all = 0;
     for (int i = 0; i < ns; ++i) {
       const int b = s0 + i;
@@ -297,31 +446,46 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
       sq.n_q = seqs->cu_qlens_h[b + 1] - sq.q_off;
       sq.rows = hq * sq.n_q;
       sq.unit_begin = units;
+      sq.unit8_begin = units8;
+      sq.lstride = (sq.len + kLogitPad - 1) / kLogitPad * kLogitPad;
       sq.logit_base = logit_base;
       sq.part_base = part_base;
       sq.lse_base = lse_base;
       const int ctas = (sq.len + kThreads - 1) / kThreads;
+      const int ctas8 = (sq.len + kRows8Tokens - 1) / kRows8Tokens;
+      sq.nparts = rows8 ? ctas8 : ctas;
       units += ctas;
-      logit_base += static_cast<int64_t>(sq.rows) * sq.len;
-      part_base += static_cast<int64_t>(sq.rows) * ctas;
+      units8 += ctas8;
+      logit_base += static_cast<int64_t>(sq.rows) * sq.lstride;
+      part_base += static_cast<int64_t>(sq.rows) * ctas8;
       lse_base += sq.rows;
       rows_all += sq.rows;
       max_rows = sq.rows > max_rows ? sq.rows : max_rows;
-      max_rg = G * sq.n_q > max_rg ? G * sq.n_q : max_rg;
     }
     P.total_units = units;
+    P.total_units8 = units8;
     if (units == 0) continue;
-    const size_t smem = static_cast<size_t>(max_rows) * 128 * sizeof(float) +
-                        static_cast<size_t>(kWarps) * max_rows * sizeof(float2);
     cudaError_t e;
     const uint16_t *q16 = static_cast<const uint16_t *>(q);
     const uint8_t *k8 = static_cast<const uint8_t *>(k);
-    if (max_rg <= 8)
-      e = launch_logits<8>(units, smem, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part);
-    else if (max_rg <= 16)
-      e = launch_logits<16>(units, smem, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part);
-    else
-      e = launch_logits<32>(units, smem, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part);
+    if (rows8) {
+      if (hkv == 4)
+        score_narrow_rows8_kernel<2><<<units8, kThreads, 0, stream>>>(P, q16, k8, k_token_stride, seqs->modality,
+                                                                       logits, part);
+      else
+        score_narrow_rows8_kernel<1><<<units8, kThreads, 0, stream>>>(P, q16, k8, k_token_stride, seqs->modality,
+                                                                       logits, part);
+      e = cudaGetLastError();
+    } else {
+      const size_t smem = static_cast<size_t>(max_rows) * 128 * sizeof(float) +
+                          static_cast<size_t>(kWarps) * max_rows * sizeof(float2);
+      if (max_rg <= 8)
+        e = launch_logits<8>(units, smem, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part);
+      else if (max_rg <= 16)
+        e = launch_logits<16>(units, smem, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part);
+      else
+        e = launch_logits<32>(units, smem, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part);
+    }
     count_launches(1);
     if (check_cuda(e) != APACK_OK) return APACK_ECUDA;
     if (rows_all > 0) {

@@ -89,6 +89,12 @@ SHAPES = [
 # (the paper scores with the last query token only: G = 7 rows per group).
 NARROW_SHAPES = [
     ([1000], [1], 28, 4),
+    # at most 8 rows per KV head group with 2 or 4 KV heads: the warp-cooperative logits kernel
+    ([3000, 700, 1, 0, 90, 64, 65], [1, 1, 1, 1, 0, 1, 1], 28, 4),
+    ([5000, 333], [1, 1], 16, 2),           # 3B heads, 8 rows per group
+    ([4100], [2], 8, 4),                    # two query tokens, 4 rows per group
+    ([777, 1500], [2, 2], 8, 2),            # two query tokens, 8 rows per group
+    # more rows per group: the general logits kernel
     ([3000, 700, 1, 0, 90], [1, 4, 2, 1, 0], 28, 4),
     ([5000], [2], 16, 2),                   # 16 rows per group
     ([2049], [4], 8, 1),                    # 32 rows in one group
