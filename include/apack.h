@@ -207,6 +207,28 @@ apack_status apack_frame_alignment(const void *visual, const void *audio, int32_
                                    float tau, float beta, float *c_out, float *s_out, float *dnorm_out,
                                    float *cbar_out, void *ws, size_t ws_bytes, void *stream);
 
+/* ---- Decode-step attention over a (compacted) KV cache.
+   Sec. 3.2 (last sentence) and App. G: pruning shortens the cache that every
+   autoregressive decode step attends to.  One decode token per sequence:
+     out[b][h][:] = sum_j softmax_j(q[b][h] . k[j][g] / sqrt(128)) v[j][g][:],
+   g = h / (Hq / Hkv), j over all cu_seqlens_h[b] .. cu_seqlens_h[b+1]-1
+   (every cached token, not only the multimodal ones).
+   q: bf16 [num_seqs][Hq][128] (8-byte aligned); k, v: bf16 token rows
+   [T][Hkv][128] with kv_token_stride bytes between tokens (8-byte aligned,
+   >= Hkv*256); out: fp32 [num_seqs][Hq][128] (16-byte aligned, device).
+   cu_seqlens_h: host [num_seqs+1], starting at 0; an empty sequence gives
+   zeros.  Supported: Hq / Hkv <= 8 and Hkv in {1, 2, 4, 8}
+   (APACK_EUNSUPPORTED otherwise).  fp32 accumulation, fixed merge order
+   (deterministic).  ws: 256-byte aligned, apack_decode_workspace_size bytes
+   (the size depends on the device's SM count; query it on the device that
+   runs the call).  Two kernel launches per 64 sequences; no allocation, no
+   synchronisation. */
+apack_status apack_decode_workspace_size(int32_t num_seqs, const int32_t *cu_seqlens_h, int32_t num_q_heads,
+                                         int32_t num_kv_heads, size_t *bytes);
+apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_h, const void *q, const void *k,
+                                    const void *v, int64_t kv_token_stride, int32_t num_q_heads,
+                                    int32_t num_kv_heads, float *out, void *ws, size_t ws_bytes, void *stream);
+
 /* Synchronises `stream`, then reads the device error word of `ws` into
    *code_out (APACK_OK, APACK_ETIMEOUT or APACK_EDEVICE) and clears it when
    `clear` is non-zero. */

@@ -27,7 +27,8 @@ APACK_HEAD_DIM = 128
 
 EXPORTED = ("apack_workspace_size", "apack_keep_counts", "apack_score", "apack_select", "apack_compact",
             "apack_prune_step", "apack_device_error", "apack_launch_count", "apack_status_string",
-            "apack_score_static", "apack_frame_alignment_workspace_size", "apack_frame_alignment")
+            "apack_score_static", "apack_frame_alignment_workspace_size", "apack_frame_alignment",
+            "apack_decode_workspace_size", "apack_decode_attention")
 
 
 class ApackError(RuntimeError):
@@ -74,6 +75,8 @@ def _load():
     lib.apack_frame_alignment_workspace_size.argtypes = [I32, I64, P(SZ)]
     lib.apack_frame_alignment.argtypes = [VP, VP, I32, I32, I32, I64, I32, ctypes.c_float, ctypes.c_float, VP, VP,
                                           VP, VP, VP, SZ, VP]
+    lib.apack_decode_workspace_size.argtypes = [I32, PI32, I32, I32, P(SZ)]
+    lib.apack_decode_attention.argtypes = [I32, PI32, VP, VP, VP, I64, I32, I32, VP, VP, SZ, VP]
     lib.apack_launch_count.argtypes = []
     lib.apack_launch_count.restype = ctypes.c_uint64
     lib.apack_status_string.argtypes = [I32]
@@ -247,6 +250,23 @@ def apack_frame_alignment(visual, audio, n_frames, tokens_per_frame, n_audio, di
                                       int(dim), int(window), float(tau), float(beta), _ptr(c_out), _ptr(s_out),
                                       _ptr(dnorm_out), _ptr(cbar_out), _ptr(ws), ws.numel() * ws.element_size(),
                                       _stream(stream)), "apack_frame_alignment")
+
+
+def apack_decode_workspace_size(cu_seqlens, num_q_heads, num_kv_heads):
+    cu = _i32(cu_seqlens)
+    n = ctypes.c_size_t(0)
+    _check(_lib.apack_decode_workspace_size(len(cu) - 1, cu.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), int(num_q_heads),
+                                            int(num_kv_heads), ctypes.byref(n)), "apack_decode_workspace_size")
+    return n.value
+
+
+def apack_decode_attention(cu_seqlens, q, k, v, kv_token_stride, num_q_heads, num_kv_heads, out, ws, stream=None):
+    """Attention of one decode token per sequence over its KV cache (Sec. 3.2)."""
+    cu = _i32(cu_seqlens)
+    _check(_lib.apack_decode_attention(len(cu) - 1, cu.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), _ptr(q), _ptr(k), _ptr(v),
+                                       int(kv_token_stride), int(num_q_heads), int(num_kv_heads), _ptr(out),
+                                       _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)),
+           "apack_decode_attention")
 
 
 def apack_device_error(ws, stream=None, clear=True):

@@ -1,0 +1,108 @@
+"""Decode-step attention over a KV cache on the GPU against the fp64 oracle
+(one decode token per sequence, Sec. 3.2 last sentence).
+
+Tolerance: logits are fp32 dot products of 128 exactly widened bf16 products
+(error ~1e-6), probabilities use the hardware exp2 (relative error ~1e-7), and
+the weighted sums of up to 1.4e5 values run in fp32 in chunks of a few hundred
+keys before an fp32 merge; |gpu - oracle| <= 2e-4 + 2e-3 |oracle| covers that
+with margin, while leaving out one key of a few thousand (a change of order
+1e-3 of the output scale) fails it."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from synth.gen import f32_to_bf16_bits
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ap():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2608_08794_gb300 as ap
+    return ap
+
+
+def bits(rng, shape, scale=1.0):
+    return f32_to_bf16_bits((rng.standard_normal(shape) * scale).astype(np.float32))
+
+
+def run(ap, cu, q, k, v, hq, hkv, pad_heads=0):
+    """k, v: uint16 [T, Hkv, 128]; pad_heads > 0 places them in wider token rows."""
+    T = k.shape[0]
+    row = (hkv + pad_heads) * 128
+    kd = torch.zeros(max(T, 1), row, dtype=torch.int16, device="cuda")
+    vd = torch.zeros_like(kd)
+    if T:
+        kd[:, :hkv * 128] = torch.from_numpy(k.reshape(T, -1).view(np.int16)).cuda()
+        vd[:, :hkv * 128] = torch.from_numpy(v.reshape(T, -1).view(np.int16)).cuda()
+    qd = torch.from_numpy(q.view(np.int16)).cuda()
+    out = torch.full((len(cu) - 1, hq, 128), float("nan"), dtype=torch.float32, device="cuda")
+    ws = torch.empty(max(256, ap.apack_decode_workspace_size(cu, hq, hkv)), dtype=torch.uint8, device="cuda")
+    ap.apack_decode_attention(cu, qd, kd, vd, row * 2, hq, hkv, out, ws)
+    torch.cuda.synchronize()
+    return out.cpu().numpy()
+
+
+def check(got, ref):
+    np.testing.assert_allclose(got, ref, atol=2e-4, rtol=2e-3)
+
+
+CASES = [
+    ([1], 28, 4),
+    ([7, 64, 65, 1000, 0, 4099], 28, 4),      # ragged, one empty cache
+    ([5000, 333], 16, 2),                    # 3B heads
+    ([2000], 8, 8),                          # one query head per KV head
+    ([3000], 8, 1),                          # 8 query heads share one KV head
+    ([100, 200, 300], 12, 4),                # 3 rows per group
+]
+
+
+@pytest.mark.parametrize("lens,hq,hkv", CASES)
+def test_decode_attention_matches_oracle(ap, lens, hq, hkv):
+    rng = np.random.default_rng(sum(lens) + hq)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = int(cu[-1])
+    q = bits(rng, (len(lens), hq, 128))
+    k = bits(rng, (T, hkv, 128), 1.5)        # peaky softmax
+    v = bits(rng, (T, hkv, 128))
+    got = run(ap, cu, q, k, v, hq, hkv)
+    check(got, oracle.decode_attention(q, k, v, cu, hq, hkv))
+    again = run(ap, cu, q, k, v, hq, hkv)
+    assert got.tobytes() == again.tobytes()
+
+
+def test_decode_attention_strided_rows_and_uniform_keys(ap):
+    rng = np.random.default_rng(7)
+    cu = np.array([0, 777, 1500], np.int32)
+    q = bits(rng, (2, 28, 128))
+    k = np.repeat(bits(rng, (1, 4, 128)), 1500, axis=0)     # identical keys: plain mean of V
+    v = bits(rng, (1500, 4, 128))
+    got = run(ap, cu, q, k, v, 28, 4, pad_heads=3)
+    ref = oracle.decode_attention(q, k, v, cu, 28, 4)
+    check(got, ref)
+    vf = oracle.bf16_to_f64(v)
+    np.testing.assert_allclose(ref[1, 27], vf[777:1500, 3].mean(axis=0), rtol=1e-12, atol=1e-14)
+
+
+def test_decode_attention_full_ten_minute_cache(ap):
+    # the uncompressed 10-minute 7B cache (135272 tokens) and its final compacted length
+    rng = np.random.default_rng(8)
+    for T in (135272, 22772):
+        cu = np.array([0, T], np.int32)
+        q = bits(rng, (1, 28, 128))
+        k = bits(rng, (T, 4, 128))
+        v = bits(rng, (T, 4, 128))
+        check(run(ap, cu, q, k, v, 28, 4), oracle.decode_attention(q, k, v, cu, 28, 4))
+
+
+def test_decode_attention_rejects_unsupported_groups(ap):
+    rng = np.random.default_rng(9)
+    cu = np.array([0, 10], np.int32)
+    with pytest.raises(ap.ApackError):
+        ap.apack_decode_workspace_size(cu, 32, 2)            # 16 query rows per KV head
+    with pytest.raises(ap.ApackError):
+        ap.apack_decode_workspace_size(np.array([0, 5, 3], np.int32), 28, 4)   # decreasing offsets
