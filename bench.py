@@ -352,6 +352,64 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
                          "note": "bf16 tokens read once + fp32 frame embeddings written once, over the whole call"}}
 
 
+def decode_measure(ap, wl, pp, steps, warmup, stream, dist):
+    """Decode-step attention (one new token, Sec. 3.2 last sentence) over the
+    layers compacted by the last prune step, on their uncompressed cache and on
+    the compacted one: the decode-side effect of the schedule.  Each call is one
+    layer; the calls rotate over the layers (more bytes than L2 holds)."""
+    import torch
+    from synth.gen import TID_Q
+    from synth.device import fill_normal_bf16
+    if wl.num_seqs != 1:
+        return None
+    last = len(pp.t_out) - 1
+    l_last = wl.prune_layers[last]
+    nl = wl.num_layers - l_last
+    full_k = [pp.k_in[l_last - wl.prune_layers[0] + j] for j in range(nl)]
+    full_v = [pp.v_in[l_last - wl.prune_layers[0] + j] for j in range(nl)]
+    ck, cv = pp.output_kv(last)
+    hq, hkv = wl.num_q_heads, wl.num_kv_heads
+    q = torch.empty(1, hq, 128, dtype=torch.bfloat16, device="cuda")
+    fill_normal_bf16(q, wl.seed, TID_Q + 999, stream=stream)
+    out = torch.empty(1, hq, 128, dtype=torch.float32, device="cuda")
+    res = {}
+    for name, T, ks, vs in (("full", wl.total_tokens, full_k, full_v),
+                            ("compacted", int(pp.t_out[last]), [ck[j] for j in range(nl)], [cv[j] for j in range(nl)])):
+        cu = [0, T]
+        ws = torch.empty(max(256, ap.apack_decode_workspace_size(cu, hq, hkv)), dtype=torch.uint8, device="cuda")
+        stride = hkv * 128 * 2
+
+        def call(j):
+            ap.apack_decode_attention(cu, q, ks[j], vs[j], stride, hq, hkv, out, ws, stream=stream)
+
+        for j in range(max(3, warmup) * nl):
+            call(j % nl)
+        torch.cuda.synchronize()
+        n = max(3, min(steps, 50)) * nl
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        c0 = ap.apack_launch_count()
+        e0.record(stream)
+        for j in range(n):
+            call(j % nl)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        res[name] = (max_over_ranks(e0.elapsed_time(e1) / n, dist, "cuda"), T, ap.apack_launch_count() - c0, n)
+    peak, peak_kind = measured_peaks()
+    ms_full, T_full, launches, calls = res["full"]
+    alg = T_full * hkv * 128 * 2 * 2 + hq * 128 * (2 + 4)
+    achieved = alg / (ms_full / 1e3) / 1e9
+    return {"metric": "decode-step attention time per layer, uncompressed vs compacted cache",
+            "layers": f"{l_last}..{wl.num_layers - 1}", "tokens": [T_full, res["compacted"][1]],
+            "full_ms_per_layer": ms_full, "compacted_ms_per_layer": res["compacted"][0],
+            "speedup": ms_full / res["compacted"][0], "calls_timed": calls,
+            "gpu_launches_per_call": launches / calls,
+            "roofline": {"bound": "hbm", "kernel": "apack_decode_attention call on the uncompressed cache "
+                                                   "(decode_chunk_kernel + decode_combine_kernel)",
+                         "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": None, "peak_source": peak_kind, "algorithmic_bytes_per_launch": alg,
+                         "note": "K and V of one layer read once, q read and out written once"}}
+
+
 # ----------------------------------------------------------------------------- GPU leg
 
 def main():
@@ -486,6 +544,8 @@ def main():
 
     # the pre-LLM stage of the same clip, timed on its own after the prune steps
     prellm = prellm_measure(ap, wl, args.steps, args.warmup, stream, dist)
+    # decode-step attention over the last step's layers, before and after pruning
+    decode = decode_measure(ap, wl, pp, args.steps, args.warmup, stream, dist)
 
     if rank == 0:
         per_step_ms = ms / args.steps
@@ -523,6 +583,7 @@ def main():
             "context": schedule_context(wl, pp),
         }
         line["prellm_alignment"] = prellm
+        line["decode_attention"] = decode
         if world == 1 and not args.no_cpu_baseline:
             try:
                 line["cpu_baseline"] = cpu_baseline(args.workload)
