@@ -458,11 +458,15 @@ def main():
     comp_bytes = [2 * t * (2 * (wl.num_layers - l) * row + wl.hidden * 2) + 4 * t
                   for t, l in zip(pp.t_out, wl.prune_layers)]
 
+    def run_schedule(events=None):
+        pp.run(events=events, stream=stream)     # the whole schedule: one apack_prune_schedule call
+
     for _ in range(args.warmup):
-        pp.run(stream=stream)
+        run_schedule()
     torch.cuda.synchronize()
 
-    # timed region: K steps, stage events on the launching stream
+    # timed region: K iterations of the schedule; per step, events before scoring, after scoring,
+    # after selection and after compaction, on the launching stream
     ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(nsteps)]
           for _ in range(args.steps)]
     for per_iter in ev:       # torch creates events on first record; the C ABI records raw handles
@@ -481,7 +485,7 @@ def main():
         clocks.mark(True)
     t_start.record(stream)
     for k in range(args.steps):
-        pp.run(events=ev[k], stream=stream)
+        run_schedule(ev[k])
     t_end.record(stream)
     barrier()
     if clocks:
@@ -491,8 +495,9 @@ def main():
     stage_ms = np.zeros((nsteps, 3))
     for k in range(args.steps):
         for i in range(nsteps):
-            for s in range(3):
-                stage_ms[i, s] += ev[k][i][s].elapsed_time(ev[k][i][s + 1])
+            e = ev[k][i]
+            for st in range(3):
+                stage_ms[i, st] += e[st].elapsed_time(e[st + 1])
     stage_ms /= args.steps
 
     # end to end through the C ABI with host buffers: H2D of the step's inputs
@@ -521,7 +526,7 @@ def main():
         pp.hidden_in.copy_(h_h, non_blocking=True); pp.modality_in.copy_(h_m, non_blocking=True)
         for a, b in zip(pp.q, h_q):
             a.copy_(b, non_blocking=True)
-        pp.run(stream=stream)
+        run_schedule()
         o_k.copy_(ko, non_blocking=True); o_v.copy_(vo, non_blocking=True); o_h.copy_(ho, non_blocking=True)
         for i, t in enumerate(pp.t_out):
             o_i[i].copy_(pp.keep_idx[i][:t], non_blocking=True)

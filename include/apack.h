@@ -207,6 +207,42 @@ apack_status apack_frame_alignment(const void *visual, const void *audio, int32_
                                    float tau, float beta, float *c_out, float *s_out, float *dnorm_out,
                                    float *cbar_out, void *ws, size_t ws_bytes, void *stream);
 
+/* ---- A whole progressive schedule in one call.
+   Sec. 3.2: pruning is repeated at later layers, each step keeping a fraction of
+   the current tokens (Algorithm 1, the inner-LLM loop).  Step i does what
+   apack_prune_step does at layer steps_h[i].layer; its inputs are step i-1's
+   outputs (K/V from k_out/v_out at layer offset l_i - l_(i-1), hidden_out,
+   modality_out, new_cu_seqlens_h, and the counts kept as the new audio/visual
+   counts; (|S|, 0) in joint mode).  Layers are strictly ascending.  Each step
+   needs its own keep_idx; outputs of step i+1 may reuse step i-1's buffers
+   (ping-pong).  All steps are checked on the host before the first launch;
+   then everything runs in order on `stream` (bit-identical to one
+   apack_prune_step per step).  stage_events_h: NULL or 4*num_steps events
+   (entries may be NULL), recorded for step i before scoring [4i], after
+   scoring [4i+1], after selection [4i+2] and after compaction [4i+3].  ws must
+   hold apack_workspace_size of every step's sequences. */
+typedef struct apack_step {
+  int32_t layer;                   /* pruning layer l_i */
+  const void *q;                   /* bf16 [sum n_q][Hq][128]: query rows of layer l_i */
+  const int32_t *keep_count_h;     /* host [B][2] kept tokens after the step, or NULL */
+  const float *keep_ratio_h;       /* host [B][2] keep ratios, used when keep_count_h is NULL */
+  void *k_out, *v_out;             /* bf16 [L - l_i][T_i][Hkv][128] */
+  int64_t kv_out_layer_stride;     /* bytes between layers of k_out / v_out */
+  void *hidden_out;                /* bf16 [T_i][hidden_dim]; required when hidden is given */
+  const apack_plane *extra_planes_h; /* further per-token planes of this step, or NULL */
+  int32_t num_extra;
+  uint8_t *modality_out;           /* [T_i] */
+  int32_t *keep_idx;               /* [T_i] */
+  int32_t *new_cu_seqlens_h;       /* host [B+1], written by the call */
+  int32_t *new_cu_seqlens;         /* device [B+1] or NULL */
+} apack_step;
+
+apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, const void *k_cache,
+                                  const void *v_cache, int64_t kv_layer_stride, const void *hidden,
+                                  int64_t hidden_dim, int32_t select_mode, const apack_step *steps_h,
+                                  int32_t num_steps, float *scores, void *ws, size_t ws_bytes,
+                                  void *const *stage_events_h, void *stream);
+
 /* ---- Decode-step attention over a (compacted) KV cache.
    Sec. 3.2 (last sentence) and App. G: pruning shortens the cache that every
    autoregressive decode step attends to.  One decode token per sequence:

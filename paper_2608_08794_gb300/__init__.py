@@ -28,7 +28,7 @@ APACK_HEAD_DIM = 128
 EXPORTED = ("apack_workspace_size", "apack_keep_counts", "apack_score", "apack_select", "apack_compact",
             "apack_prune_step", "apack_device_error", "apack_launch_count", "apack_status_string",
             "apack_score_static", "apack_frame_alignment_workspace_size", "apack_frame_alignment",
-            "apack_decode_workspace_size", "apack_decode_attention")
+            "apack_decode_workspace_size", "apack_decode_attention", "apack_prune_schedule")
 
 
 class ApackError(RuntimeError):
@@ -56,6 +56,15 @@ class apack_plane(ctypes.Structure):
                 ("row_bytes", ctypes.c_int64), ("num_planes", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
+class apack_step(ctypes.Structure):
+    _fields_ = [("layer", ctypes.c_int32), ("q", ctypes.c_void_p),
+                ("keep_count_h", ctypes.POINTER(ctypes.c_int32)), ("keep_ratio_h", ctypes.POINTER(ctypes.c_float)),
+                ("k_out", ctypes.c_void_p), ("v_out", ctypes.c_void_p), ("kv_out_layer_stride", ctypes.c_int64),
+                ("hidden_out", ctypes.c_void_p), ("extra_planes_h", ctypes.POINTER(apack_plane)),
+                ("num_extra", ctypes.c_int32), ("modality_out", ctypes.c_void_p), ("keep_idx", ctypes.c_void_p),
+                ("new_cu_seqlens_h", ctypes.POINTER(ctypes.c_int32)), ("new_cu_seqlens", ctypes.c_void_p)]
+
+
 def _load():
     if not os.path.exists(LIB_PATH):
         raise ImportError(f"libapack.so is not built ({LIB_PATH}); run __graft_entry__.build()")
@@ -77,6 +86,8 @@ def _load():
                                           VP, VP, VP, SZ, VP]
     lib.apack_decode_workspace_size.argtypes = [I32, PI32, I32, I32, P(SZ)]
     lib.apack_decode_attention.argtypes = [I32, PI32, VP, VP, VP, I64, I32, I32, VP, VP, SZ, VP]
+    lib.apack_prune_schedule.argtypes = [P(apack_seqs), I32, VP, VP, I64, VP, I64, I32, P(apack_step), I32, VP, VP,
+                                         SZ, P(VP), VP]
     lib.apack_launch_count.argtypes = []
     lib.apack_launch_count.restype = ctypes.c_uint64
     lib.apack_status_string.argtypes = [I32]
@@ -227,6 +238,63 @@ def apack_prune_step(seqs, layer, num_layers, q, k_cache, v_cache, kv_layer_stri
         0 if ws is None else ws.numel() * ws.element_size(), ev, _stream(stream))
     _check(st, "apack_prune_step")
     return new_cu
+
+
+def _event_handles(events, n, what):
+    if events is None:
+        return None
+    handles = [0 if e is None else (e.cuda_event if hasattr(e, "cuda_event") else e) for e in events]
+    if len(handles) != n:
+        raise ValueError(f"{what}: {n} events expected")
+    return (ctypes.c_void_p * n)(*handles)
+
+
+def apack_prune_schedule(seqs, num_layers, k_cache, v_cache, kv_layer_stride, hidden, hidden_dim, steps,
+                         select_mode=APACK_SELECT_PER_MODALITY, scores=None, ws=None, stage_events=None, stream=None):
+    """A whole progressive schedule (one apack_prune_step per entry of `steps`, each
+    reading the previous step's outputs).  steps: dicts with layer, q, keep_count or
+    keep_ratio, k_out, v_out, kv_out_layer_stride, hidden_out, modality_out, keep_idx
+    and optionally new_cu_seqlens (device) and extra_planes.  stage_events: None or
+    4 * len(steps) created events.  Returns the new host offsets of every step."""
+    B = seqs.num_seqs
+    n = len(steps)
+    I32P = ctypes.POINTER(ctypes.c_int32)
+    keep = []                           # host arrays referenced by the call
+    arr = (apack_step * n)()
+    new_cus = []
+    for i, d in enumerate(steps):
+        st = arr[i]
+        st.layer = int(d["layer"])
+        st.q = _ptr(d["q"])
+        if d.get("keep_count") is not None:
+            kc = _i32(d["keep_count"]).reshape(-1)
+            keep.append(kc)
+            st.keep_count_h = kc.ctypes.data_as(I32P)
+        else:
+            r = np.ascontiguousarray(np.asarray(d["keep_ratio"], dtype=np.float32).reshape(B, 2))
+            keep.append(r)
+            st.keep_ratio_h = r.ctypes.data_as(ctypes.POINTER(ctypes.c_float))
+        st.k_out, st.v_out = _ptr(d["k_out"]), _ptr(d["v_out"])
+        st.kv_out_layer_stride = int(d["kv_out_layer_stride"])
+        st.hidden_out = _ptr(d.get("hidden_out"))
+        extra = d.get("extra_planes", ())
+        if extra:
+            ep = (apack_plane * len(extra))(*extra)
+            keep.append(ep)
+            st.extra_planes_h = ctypes.cast(ep, ctypes.POINTER(apack_plane))
+        st.num_extra = len(extra)
+        st.modality_out = _ptr(d["modality_out"])
+        st.keep_idx = _ptr(d["keep_idx"])
+        cu = np.zeros(B + 1, np.int32)
+        new_cus.append(cu)
+        st.new_cu_seqlens_h = cu.ctypes.data_as(I32P)
+        st.new_cu_seqlens = _ptr(d.get("new_cu_seqlens"))
+    stage = _event_handles(stage_events, 4 * n, "stage_events")
+    _check(_lib.apack_prune_schedule(
+        seqs.ref(), int(num_layers), _ptr(k_cache), _ptr(v_cache), int(kv_layer_stride), _ptr(hidden),
+        int(hidden_dim), int(select_mode), arr, n, _ptr(scores), _ptr(ws),
+        0 if ws is None else ws.numel() * ws.element_size(), stage, _stream(stream)), "apack_prune_schedule")
+    return new_cus
 
 
 def apack_score_static(seqs, q, k, k_token_stride, scores, device_error_out=None, stream=None):

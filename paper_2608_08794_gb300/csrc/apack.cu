@@ -105,6 +105,10 @@ bool ratios_ok(const apack_seqs *s, const float *r, int32_t mode) {
   return true;
 }
 
+}  // namespace
+
+namespace apack {
+
 apack_status counts_and_offsets(const apack_seqs *s, const float *ratio_h, const int32_t *count_h, int32_t mode,
                                  int32_t *k_out, int32_t *cu_out) {
   if (mode != APACK_SELECT_PER_MODALITY && mode != APACK_SELECT_JOINT) return APACK_EINVAL;
@@ -147,7 +151,7 @@ bool ws_ok(const apack_seqs *s, const void *ws, size_t bytes) {
   return bytes >= workspace_layout(s).total;
 }
 
-}  // namespace
+}  // namespace apack
 
 extern "C" {
 

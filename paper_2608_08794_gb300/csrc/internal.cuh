@@ -72,5 +72,8 @@ apack_status run_select(const apack_seqs *seqs, const float *scores, const int32
                         void *ws, cudaStream_t stream);
 apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes, int32_t num_groups,
                          DeviceError *err, cudaStream_t stream);
+apack_status counts_and_offsets(const apack_seqs *s, const float *ratio_h, const int32_t *count_h, int32_t mode,
+                                int32_t *k_out, int32_t *cu_out);
+bool ws_ok(const apack_seqs *s, const void *ws, size_t bytes);
 
 }  // namespace apack

@@ -2,11 +2,12 @@
 over pruning layers l >= L_mid; Sec. 3.2: pruning repeats at later layers on
 the already shortened sequence).
 
-Each step calls ``apack_prune_step`` once.  Step i prunes at layer l_i and
-compacts the K/V slabs of layers [l_i, L) plus the hidden states; step i+1
-reads its layer's keys from slab (l_{i+1} - l_i) of step i's output.  Two
-output buffers alternate (ping-pong), so the input cache of step 0 is never
-written and the schedule can be replayed on the same inputs.
+Step i prunes at layer l_i and compacts the K/V slabs of layers [l_i, L)
+plus the hidden states; step i+1 reads its layer's keys from slab
+(l_{i+1} - l_i) of step i's output.  Two output buffers alternate
+(ping-pong), so the input cache of step 0 is never written and the schedule
+can be replayed on the same inputs.  ``run_step`` calls ``apack_prune_step``
+for one step; ``run`` hands the whole schedule to ``apack_prune_schedule``.
 
 Only buffer management and argument marshalling happen here.
 """
@@ -14,8 +15,8 @@ Only buffer management and argument marshalling happen here.
 import numpy as np
 import torch
 
-from . import (Seqs, apack_prune_step, apack_workspace_size, apack_keep_counts, APACK_HEAD_DIM,
-               APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT)
+from . import (Seqs, apack_prune_step, apack_prune_schedule, apack_workspace_size, apack_keep_counts,
+               APACK_HEAD_DIM, APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT)
 
 
 def schedule_keep_counts(cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, num_kv_heads, modality,
@@ -116,7 +117,27 @@ class ProgressivePrune:
         return (self._step_seqs(i), k, v, t_prev * self.row, self.h_out[prev])
 
     def run(self, events=None, stream=None):
-        """Runs every step; events[i] = 4 CUDA events per step or None."""
+        """Runs every step through apack_prune_schedule.  events: None or 4 CUDA
+        events per step (before scoring, after scoring, after selection, after
+        compaction)."""
+        n = len(self.layers)
+        steps = []
+        for i in range(n):
+            o = i % 2
+            steps.append(dict(layer=self.layers[i], q=self.q[i], keep_count=self.counts[i], k_out=self.k_out[o],
+                              v_out=self.v_out[o], kv_out_layer_stride=self.t_out[i] * self.row,
+                              hidden_out=self.h_out[o], modality_out=self.mod_out[o], keep_idx=self.keep_idx[i]))
+        flat = None
+        if events is not None:
+            flat = [e for per_step in events for e in per_step]
+        self.new_cu = apack_prune_schedule(
+            self._step_seqs(0), self.L, self.k_in.view(-1), self.v_in.view(-1), self.T0 * self.row,
+            self.hidden_in, self.H, steps, select_mode=self.mode, scores=self.scores, ws=self.ws,
+            stage_events=flat, stream=stream)
+
+    def run_steps(self, events=None, stream=None):
+        """Runs every step with one apack_prune_step call each; events[i] = 4 CUDA
+        events per step or None."""
         self.new_cu = [None] * len(self.layers)
         for i in range(len(self.layers)):
             self.run_step(i, None if events is None else events[i], stream)

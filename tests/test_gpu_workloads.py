@@ -114,3 +114,57 @@ def test_workload_parity(ap, name):
     tok, _ = planted_tokens(wl)
     assert np.isin(tok, composite).all(), "a planted token was dropped"
     print(f"{name}: tie-exempt tokens {exempt_total}")
+
+
+def snapshot(pp):
+    """Every output the schedule leaves behind: per-step indices and offsets, the
+    last two steps' K/V (both ping-pong buffers), hidden states and modality."""
+    n = len(pp.layers)
+    out = {"keep": [pp.keep_idx[i][:pp.t_out[i]].clone() for i in range(n)],
+           "cu": [np.asarray(c).copy() for c in pp.new_cu]}
+    for i in range(max(0, n - 2), n):
+        k, v = pp.output_kv(i)
+        out[f"k{i}"], out[f"v{i}"] = k.clone(), v.clone()
+        out[f"h{i}"] = pp.output_hidden(i).clone()
+        out[f"m{i}"] = pp.mod_out[i % 2][:pp.t_out[i]].clone()
+    return out
+
+
+def same(a, b):
+    assert a.keys() == b.keys()
+    for key in a:
+        if key == "cu":
+            for x, y in zip(a[key], b[key]):
+                np.testing.assert_array_equal(x, y)
+        elif key == "keep":
+            for x, y in zip(a[key], b[key]):
+                assert torch.equal(x, y)
+        else:
+            assert torch.equal(a[key].view(torch.int8) if a[key].dtype != torch.uint8 else a[key],
+                               b[key].view(torch.int8) if b[key].dtype != torch.uint8 else b[key]), key
+
+
+@pytest.mark.parametrize("name", ["3b_60s", "7b_2min", "7b_10min", "7b_ragged16", "7b_10min_paper"])
+def test_schedule_runner_is_bit_identical_to_single_steps(ap, name):
+    """apack_prune_schedule leaves exactly the outputs of one apack_prune_step per step."""
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+
+    wl = workload(name)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod_d = torch.from_numpy(wl.modality()).cuda()
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_d,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
+    pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                          wl.prune_layers, counts, select_mode=mode)
+    fill_progressive_inputs(pp, wl)
+    pp.run_steps()
+    torch.cuda.synchronize()
+    ref = snapshot(pp)
+    pp.run()
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+    same(ref, snapshot(pp))
