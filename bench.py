@@ -376,7 +376,7 @@ def decode_measure(ap, wl, pp, steps, warmup, stream, dist):
     for name, T, ks, vs in (("full", wl.total_tokens, full_k, full_v),
                             ("compacted", int(pp.t_out[last]), [ck[j] for j in range(nl)], [cv[j] for j in range(nl)])):
         cu = [0, T]
-        ws = torch.empty(max(256, ap.apack_decode_workspace_size(cu, hq, hkv)), dtype=torch.uint8, device="cuda")
+        ws = torch.zeros(max(256, ap.apack_decode_workspace_size(cu, hq, hkv)), dtype=torch.uint8, device="cuda")
         stride = hkv * 128 * 2
 
         def call(j):

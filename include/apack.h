@@ -250,15 +250,17 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
    g = h / (Hq / Hkv), j over all cu_seqlens_h[b] .. cu_seqlens_h[b+1]-1
    (every cached token, not only the multimodal ones).
    q: bf16 [num_seqs][Hq][128] (8-byte aligned); k, v: bf16 token rows
-   [T][Hkv][128] with kv_token_stride bytes between tokens (8-byte aligned,
-   >= Hkv*256); out: fp32 [num_seqs][Hq][128] (16-byte aligned, device).
-   cu_seqlens_h: host [num_seqs+1], starting at 0; an empty sequence gives
-   zeros.  Supported: Hq / Hkv <= 8 and Hkv in {1, 2, 4, 8}
-   (APACK_EUNSUPPORTED otherwise).  fp32 accumulation, fixed merge order
-   (deterministic).  ws: 256-byte aligned, apack_decode_workspace_size bytes
-   (the size depends on the device's SM count; query it on the device that
-   runs the call).  Two kernel launches per 64 sequences; no allocation, no
-   synchronisation. */
+   [T][Hkv][128] with kv_token_stride bytes between tokens (16-byte aligned,
+   a multiple of 16, >= Hkv*256); out: fp32 [num_seqs][Hq][128] (16-byte
+   aligned, device).  cu_seqlens_h: host [num_seqs+1], starting at 0; an
+   empty sequence gives zeros.  Supported: Hq / Hkv <= 8 and Hkv in
+   {1, 2, 4, 8} (APACK_EUNSUPPORTED otherwise).  fp32 accumulation, fixed
+   merge order (deterministic).  ws: 256-byte aligned,
+   apack_decode_workspace_size bytes (the size depends on the device's SM
+   count: query it on the device that runs the call); its first 16 bytes are
+   a device error word read by apack_device_error, zeroed by the caller once.
+   A device-side wait that runs out records APACK_ETIMEOUT there.  Two kernel
+   launches per 64 sequences; no allocation, no synchronisation. */
 apack_status apack_decode_workspace_size(int32_t num_seqs, const int32_t *cu_seqlens_h, int32_t num_q_heads,
                                          int32_t num_kv_heads, size_t *bytes);
 apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_h, const void *q, const void *k,

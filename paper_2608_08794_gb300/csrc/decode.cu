@@ -6,15 +6,17 @@
 //   g(h) = h / (Hq / Hkv), j over every cached token of sequence b.
 //
 // Split-KV in two launches:
-//   chunk kernel:   one CTA per (sequence, chunk of keys), 8 warps; warp w works on KV
-//                   head w % Hkv and a contiguous run of the chunk's keys; lane l owns
-//                   features [4l, 4l + 4) of that head for all G <= 8 query rows of the
-//                   head group.  Per 8 keys: logits by a reduce-scatter of the 8 row
-//                   partials over the warp (the lane's query rows are stored in an
-//                   order that makes every step a plain shuffle and add), online max
-//                   and sum per row, probabilities handed to all lanes through shared
-//                   memory, P.V accumulated in registers.  Warps of the same head merge
-//                   in shared memory; the CTA writes (max, sum, o[128]) per query head.
+//   chunk kernel:   one CTA per (sequence, chunk of about T / #SMs keys).  K and V rows
+//                   stream into a 3-stage shared-memory ring by bulk async copies (issued
+//                   by one lane).  Each of 16 warps works on KV head
+//                   w % Hkv and one group of 8 keys of every stage; lane l owns features
+//                   [4l, 4l + 4) of that head for all G <= 8 query rows of the head group.
+//                   Per 8 keys: logits by a reduce-scatter of the 8 row partials over the
+//                   warp (the lane's query rows are stored in an order that makes every
+//                   step a plain shuffle and add), online max and sum per row,
+//                   probabilities handed to all lanes through shared memory, P.V
+//                   accumulated in registers.  The warps of a head merge in shared memory;
+//                   the CTA writes (max, sum, o[128]) per query head.
 //   combine kernel: one CTA per (sequence, query head) merges the chunks in order.
 // K and V are read once: the chunk kernel is HBM-bound.  All merges run in a fixed
 // order, so the output is deterministic.
@@ -28,9 +30,13 @@ namespace apack {
 
 namespace {
 
-constexpr int kDecThreads = 256;
-constexpr int kDecWarps = kDecThreads / 32;
-constexpr int kDecRows = 8;              // query rows per KV head group (G <= 8)
+constexpr int kDecConsumers = 16;                 // warps per CTA; lane 0 of the last also loads
+constexpr int kDecThreads = kDecConsumers * 32;
+constexpr int kDecStages = 3;                     // shared-memory ring of K/V stages
+constexpr int kStageBytes = 32768;                // K (and V) bytes per stage: 128 / Hkv tokens
+constexpr int kDecRows = 8;                       // query rows per KV head group (G <= 8)
+constexpr size_t kDecSmem = static_cast<size_t>(kDecStages) * 2 * kStageBytes + 2 * kDecStages * sizeof(uint64_t) +
+                            (kDecConsumers * 8 * kDecRows + kDecConsumers * kDecRows) * sizeof(float) + 16;
 constexpr int kDecCombineThreads = 512;
 constexpr int kDecCombineWarps = kDecCombineThreads / 32;
 
@@ -73,154 +79,218 @@ __device__ __forceinline__ void merge_state(float &m1, float &l1, float (&o1)[4]
 
 // q: bf16 [nseq][Hq][128] of this launch's sequences.  Partials per (chunk, query head):
 // opart [chunks][Hq][128], mlpart [chunks][Hq] = (max, sum) in log2 units.
-__global__ void __launch_bounds__(kDecThreads, 2)
+//
+// K and V rows stream into a ring of kDecStages shared-memory stages by bulk async copies;
+// a stage holds kStageBytes of K and of V (128 / Hkv tokens).  Warp w takes KV head w % Hkv
+// and the group of 8 keys (w / Hkv) of every stage, so all 16 warps consume a stage
+// together.  Lane 0 of the last warp is also the loader: it issues the first stages, and
+// after its own group of stage n, once every warp has released stage n, it refills that
+// stage's slot with stage n + kDecStages.
+__device__ __forceinline__ void decode_issue_stage(const DecSeq &sq, const uint8_t *k, const uint8_t *v,
+                                                   int64_t kv_stride, int64_t row, int stage_tok, int tb, int te,
+                                                   int n, uint8_t *stage_base, uint64_t *full) {
+  const int slot = n % kDecStages;
+  const int t = tb + n * stage_tok;
+  const int cnt = min(stage_tok, te - t);
+  uint8_t *ks = stage_base + static_cast<size_t>(slot) * 2 * kStageBytes;
+  uint8_t *vs = ks + kStageBytes;
+  mbar_arrive_expect_tx(&full[slot], static_cast<uint32_t>(2 * cnt * row));
+  const int64_t g0 = static_cast<int64_t>(sq.t0) + t;
+  if (kv_stride == row) {   // dense rows: one copy per tensor
+    bulk_load(ks, k + g0 * kv_stride, static_cast<uint32_t>(cnt * row), &full[slot]);
+    bulk_load(vs, v + g0 * kv_stride, static_cast<uint32_t>(cnt * row), &full[slot]);
+  } else {
+    for (int r = 0; r < cnt; ++r) {
+      bulk_load(ks + r * row, k + (g0 + r) * kv_stride, static_cast<uint32_t>(row), &full[slot]);
+      bulk_load(vs + r * row, v + (g0 + r) * kv_stride, static_cast<uint32_t>(row), &full[slot]);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kDecThreads, 1)
     decode_chunk_kernel(const __grid_constant__ DecPlan plan, const uint16_t *__restrict__ q,
                         const uint8_t *__restrict__ k, const uint8_t *__restrict__ v, int64_t kv_stride,
-                        float *__restrict__ opart, float2 *__restrict__ mlpart) {
-  __shared__ __align__(16) float ps[kDecWarps][8][kDecRows];   // [warp][key][row] probabilities
-  __shared__ __align__(16) float sc[kDecWarps][kDecRows];      // [warp][row] rescale factors
-  __shared__ __align__(16) float wo[kDecWarps][kDecRows][128]; // per warp o, for the head merge
-  __shared__ float2 wml[kDecWarps][kDecRows];                  // per warp (max, sum) per row
+                        float *__restrict__ opart, float2 *__restrict__ mlpart, DeviceError *err) {
+  extern __shared__ __align__(1024) uint8_t dsmem[];
+  uint8_t *stage_base = dsmem;                                               // [kDecStages][K | V]
+  uint64_t *full = reinterpret_cast<uint64_t *>(dsmem + kDecStages * 2 * kStageBytes);
+  uint64_t *empty = full + kDecStages;
+  float *ps = reinterpret_cast<float *>(empty + kDecStages);                 // [warp][key][row]
+  float *sc = ps + kDecConsumers * 8 * kDecRows;                             // [warp][row]
+  int *abort_flag = reinterpret_cast<int *>(sc + kDecConsumers * kDecRows);
   const int c = blockIdx.x;
   const int s = find_chunk_seq(plan, c);
   const DecSeq &sq = plan.seq[s];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int G = plan.group, hkv = plan.hkv;
-  const int h = warp % hkv, stream = warp / hkv, nstreams = kDecWarps / hkv;
-  // keys of this warp: a contiguous run of the chunk
-  const int cbeg = (c - sq.chunk_begin) * plan.chunk;
-  const int per = plan.chunk / nstreams;
-  const int tb = cbeg + stream * per;
-  const int te = min(sq.len, tb + per);
-  // query rows of the group, lane-permuted: slot j holds row j ^ cl
-  const int cl = (lane >> 2) & 7;
-  float qf[kDecRows][4];
+  const int64_t row = static_cast<int64_t>(hkv) * 256;
+  const int stage_tok = kStageBytes / static_cast<int>(row);
+  const int tb = (c - sq.chunk_begin) * plan.chunk;
+  const int te = min(sq.len, tb + plan.chunk);
+  const int nst = (te - tb + stage_tok - 1) / stage_tok;
+  const bool loader = warp == kDecConsumers - 1 && lane == 0;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kDecStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], kDecConsumers);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  volatile int *abort_v = abort_flag;
+  int issued = 0;
+  if (loader)
+    for (; issued < kDecStages && issued < nst; ++issued)
+      decode_issue_stage(sq, k, v, kv_stride, row, stage_tok, tb, te, issued, stage_base, full);
+
+  const int h = warp % hkv, grp = warp / hkv;
+  const int cl = (lane >> 2) & 7;       // after the reduce-scatter this lane holds row cl
+  float qf[kDecRows][4];                // query rows, lane-permuted: slot j holds row j ^ cl
   const uint16_t *qg = q + (static_cast<int64_t>(s) * plan.hq + h * G) * 128 + lane * 4;
 #pragma unroll
   for (int j = 0; j < kDecRows; ++j) {
-    const int row = j ^ cl;
+    const int r = j ^ cl;
     uint2 w = make_uint2(0, 0);
-    if (row < G) w = __ldg(reinterpret_cast<const uint2 *>(qg + row * 128));
+    if (r < G) w = __ldg(reinterpret_cast<const uint2 *>(qg + r * 128));
     bf16x4_to_f32(w, qf[j]);
   }
-  // after the reduce-scatter this lane holds the logit of row cl
   float o[kDecRows][4];
 #pragma unroll
   for (int j = 0; j < kDecRows; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
   float m_own = -INFINITY, l_own = 0.f;
-  const uint8_t *kb = k + static_cast<int64_t>(sq.t0) * kv_stride + h * 256 + lane * 8;
-  const uint8_t *vb = v + static_cast<int64_t>(sq.t0) * kv_stride + h * 256 + lane * 8;
-#pragma unroll 1
-  for (int t0 = tb; t0 < te; t0 += 8) {
-    uint2 kr[8], vr[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const bool ok = t0 + i < te;
-      kr[i] = ok ? __ldg(reinterpret_cast<const uint2 *>(kb + static_cast<int64_t>(t0 + i) * kv_stride))
-                 : make_uint2(0, 0);
-      vr[i] = ok ? __ldg(reinterpret_cast<const uint2 *>(vb + static_cast<int64_t>(t0 + i) * kv_stride))
-                 : make_uint2(0, 0);
-    }
-    float x[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      float kf[4];
-      bf16x4_to_f32(kr[i], kf);
-      float acc[kDecRows];
-#pragma unroll
-      for (int j = 0; j < kDecRows; j += 2) {
-        float2 a = make_float2(0.f, 0.f);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) a = ffma2(make_float2(kf[e], kf[e]), make_float2(qf[j][e], qf[j + 1][e]), a);
-        acc[j] = a.x;
-        acc[j + 1] = a.y;
+  float *wps = ps + warp * 8 * kDecRows;
+  float *wsc = sc + warp * kDecRows;
+  for (int n = 0; n < nst; ++n) {
+    const int slot = n % kDecStages;
+    // the decision to go on is warp-uniform: every lane waited, and all must have succeeded
+    if (!__all_sync(0xffffffffu, mbar_wait(&full[slot], (n / kDecStages) & 1u, kWaitLimitNs))) {
+      if (lane == 0) {
+        raise_device_error(err, APACK_ETIMEOUT, 62, c, n);
+        *abort_v = 1;
       }
-      // slot e and the partner's slot e + half hold the same row at every level
-#pragma unroll
-      for (int e = 0; e < 4; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e + 4], 16);
-#pragma unroll
-      for (int e = 0; e < 2; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e + 2], 8);
-      acc[0] += __shfl_xor_sync(0xffffffffu, acc[1], 4);
-      acc[0] += __shfl_xor_sync(0xffffffffu, acc[0], 2);
-      acc[0] += __shfl_xor_sync(0xffffffffu, acc[0], 1);
-      x[i] = t0 + i < te ? acc[0] * plan.scale2 : -INFINITY;
+      break;
     }
-    // online softmax of row cl over these keys (key t0 is always valid)
-    float cm = x[0];
+    const int t = tb + n * stage_tok + grp * 8;
+    const int valid = min(8, te - t);
+    if (valid > 0) {
+      const uint8_t *ks = stage_base + static_cast<size_t>(slot) * 2 * kStageBytes +
+                          static_cast<size_t>(grp) * 8 * row + h * 256 + lane * 8;
+      const uint8_t *vs = ks + kStageBytes;
+      float x[8];
 #pragma unroll
-    for (int i = 1; i < 8; ++i) cm = fmaxf(cm, x[i]);
-    const float mn = fmaxf(m_own, cm);
-    const float scale = ex2_approx(m_own - mn);
-    float psum = 0.f;
-    __syncwarp();
+      for (int i = 0; i < 8; ++i) {
+        float kf[4];
+        bf16x4_to_f32(i < valid ? *reinterpret_cast<const uint2 *>(ks + i * row) : make_uint2(0, 0), kf);
+        float acc[kDecRows];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float p = ex2_approx(x[i] - mn);
-      psum += p;
-      ps[warp][i][cl] = p;               // the four lanes of a row write the same value
-    }
-    sc[warp][cl] = scale;
-    l_own = l_own * scale + psum;
-    m_own = mn;
-    __syncwarp();
-    {
-      const float4 sa = *reinterpret_cast<const float4 *>(&sc[warp][0]);
-      const float4 sb = *reinterpret_cast<const float4 *>(&sc[warp][4]);
-      const float sr[8] = {sa.x, sa.y, sa.z, sa.w, sb.x, sb.y, sb.z, sb.w};
+        for (int j = 0; j < kDecRows; j += 2) {
+          float2 a = make_float2(0.f, 0.f);
 #pragma unroll
-      for (int j = 0; j < kDecRows; ++j)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) o[j][e] *= sr[j];
-    }
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      float vf[4];
-      bf16x4_to_f32(vr[i], vf);
-      const float4 pa = *reinterpret_cast<const float4 *>(&ps[warp][i][0]);
-      const float4 pb = *reinterpret_cast<const float4 *>(&ps[warp][i][4]);
-      const float pr[8] = {pa.x, pa.y, pa.z, pa.w, pb.x, pb.y, pb.z, pb.w};
-#pragma unroll
-      for (int j = 0; j < kDecRows; j += 2)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 r = ffma2(make_float2(pr[j], pr[j + 1]), make_float2(vf[e], vf[e]),
-                                 make_float2(o[j][e], o[j + 1][e]));
-          o[j][e] = r.x;
-          o[j + 1][e] = r.y;
+          for (int e = 0; e < 4; ++e) a = ffma2(make_float2(kf[e], kf[e]), make_float2(qf[j][e], qf[j + 1][e]), a);
+          acc[j] = a.x;
+          acc[j + 1] = a.y;
         }
+        // slot e and the partner's slot e + half hold the same row at every level
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e + 4], 16);
+#pragma unroll
+        for (int e = 0; e < 2; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e + 2], 8);
+        acc[0] += __shfl_xor_sync(0xffffffffu, acc[1], 4);
+        acc[0] += __shfl_xor_sync(0xffffffffu, acc[0], 2);
+        acc[0] += __shfl_xor_sync(0xffffffffu, acc[0], 1);
+        x[i] = i < valid ? acc[0] * plan.scale2 : -INFINITY;
+      }
+      // online softmax of row cl over these keys (key 0 of the group is valid)
+      float cm = x[0];
+#pragma unroll
+      for (int i = 1; i < 8; ++i) cm = fmaxf(cm, x[i]);
+      const float mn = fmaxf(m_own, cm);
+      const float scale = ex2_approx(m_own - mn);
+      float psum = 0.f;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float p = ex2_approx(x[i] - mn);
+        psum += p;
+        wps[i * kDecRows + cl] = p;        // the four lanes of a row write the same value
+      }
+      wsc[cl] = scale;
+      l_own = l_own * scale + psum;
+      m_own = mn;
+      __syncwarp();
+      {
+        const float4 sa = *reinterpret_cast<const float4 *>(wsc);
+        const float4 sb = *reinterpret_cast<const float4 *>(wsc + 4);
+        const float sr[8] = {sa.x, sa.y, sa.z, sa.w, sb.x, sb.y, sb.z, sb.w};
+#pragma unroll
+        for (int j = 0; j < kDecRows; ++j)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) o[j][e] *= sr[j];
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        float vf[4];
+        bf16x4_to_f32(i < valid ? *reinterpret_cast<const uint2 *>(vs + i * row) : make_uint2(0, 0), vf);
+        const float4 pa = *reinterpret_cast<const float4 *>(wps + i * kDecRows);
+        const float4 pb = *reinterpret_cast<const float4 *>(wps + i * kDecRows + 4);
+        const float pr[8] = {pa.x, pa.y, pa.z, pa.w, pb.x, pb.y, pb.z, pb.w};
+#pragma unroll
+        for (int j = 0; j < kDecRows; j += 2)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 r2 = ffma2(make_float2(pr[j], pr[j + 1]), make_float2(vf[e], vf[e]),
+                                    make_float2(o[j][e], o[j + 1][e]));
+            o[j][e] = r2.x;
+            o[j + 1][e] = r2.y;
+          }
+      }
     }
+    __syncwarp();                        // this warp is done with the stage and its scratch
+    if (lane == 0) mbar_arrive(&empty[slot]);
+    if (loader && issued < nst) {
+      // every warp has released stage n: refill its slot
+      if (!mbar_wait(&empty[slot], (n / kDecStages) & 1u, kWaitLimitNs)) {
+        raise_device_error(err, APACK_ETIMEOUT, 61, c, n);
+        *abort_v = 1;
+      } else {
+        decode_issue_stage(sq, k, v, kv_stride, row, stage_tok, tb, te, issued, stage_base, full);
+        ++issued;
+      }
+    }
+    __syncwarp();
+    if (*abort_v) break;
   }
-  // merge the warps of each head in stream order, then write the chunk's partials
+  // after an abort, stages may still be in flight: wait for them (bounded) before the
+  // shared memory is reused or the CTA exits
+  if (loader && *abort_v)
+    for (int n = max(0, issued - kDecStages); n < issued; ++n)
+      mbar_wait(&full[n % kDecStages], (n / kDecStages) & 1u, kWaitLimitNs / 4);
+  __syncthreads();
+  if (*abort_v) return;
+  // merge the warps of each head in group order; the stages are free now
+  float *wo = reinterpret_cast<float *>(stage_base);                   // [warp][row][128]
+  float2 *wml = reinterpret_cast<float2 *>(wo + kDecConsumers * kDecRows * 128);
 #pragma unroll
   for (int j = 0; j < kDecRows; ++j)
-    *reinterpret_cast<float4 *>(&wo[warp][j][lane * 4]) = make_float4(o[j][0], o[j][1], o[j][2], o[j][3]);
-  if ((lane & 3) == 0) wml[warp][cl] = make_float2(m_own, l_own);
+    *reinterpret_cast<float4 *>(wo + (warp * kDecRows + j) * 128 + lane * 4) =
+        make_float4(o[j][0], o[j][1], o[j][2], o[j][3]);
+  if ((lane & 3) == 0) wml[warp * kDecRows + cl] = make_float2(m_own, l_own);
   __syncthreads();
-  if (stream == 0) {
-    // this warp (stream 0 of head h) folds in streams 1.. of the same head
-    for (int st = 1; st < nstreams; ++st) {
-      const int w2 = st * hkv + h;
-#pragma unroll
-      for (int j = 0; j < kDecRows; ++j) {
-        float m1 = wml[warp][j].x, l1 = wml[warp][j].y;
-        const float2 ml2 = wml[w2][j];
-        float o1[4], o2[4];
-        const float4 a = *reinterpret_cast<const float4 *>(&wo[warp][j][lane * 4]);
-        const float4 b = *reinterpret_cast<const float4 *>(&wo[w2][j][lane * 4]);
-        o1[0] = a.x; o1[1] = a.y; o1[2] = a.z; o1[3] = a.w;
-        o2[0] = b.x; o2[1] = b.y; o2[2] = b.z; o2[3] = b.w;
-        merge_state(m1, l1, o1, ml2.x, ml2.y, o2);
-        *reinterpret_cast<float4 *>(&wo[warp][j][lane * 4]) = make_float4(o1[0], o1[1], o1[2], o1[3]);
-        __syncwarp();
-        if (lane == 0) wml[warp][j] = make_float2(m1, l1);
-        __syncwarp();
-      }
-    }
+  if (grp == 0) {
     for (int j = 0; j < G; ++j) {
+      float m1 = wml[warp * kDecRows + j].x, l1 = wml[warp * kDecRows + j].y;
+      const float4 a = *reinterpret_cast<const float4 *>(wo + (warp * kDecRows + j) * 128 + lane * 4);
+      float o1[4] = {a.x, a.y, a.z, a.w};
+      for (int g2 = 1; g2 < kDecConsumers / hkv; ++g2) {
+        const int w2 = g2 * hkv + h;
+        const float2 ml2 = wml[w2 * kDecRows + j];
+        const float4 b = *reinterpret_cast<const float4 *>(wo + (w2 * kDecRows + j) * 128 + lane * 4);
+        const float o2[4] = {b.x, b.y, b.z, b.w};
+        merge_state(m1, l1, o1, ml2.x, ml2.y, o2);
+      }
       const int64_t hq_idx = static_cast<int64_t>(c) * plan.hq + h * G + j;
-      *reinterpret_cast<float4 *>(opart + hq_idx * 128 + lane * 4) =
-          *reinterpret_cast<const float4 *>(&wo[warp][j][lane * 4]);
-      if (lane == 0) mlpart[hq_idx] = wml[warp][j];
+      *reinterpret_cast<float4 *>(opart + hq_idx * 128 + lane * 4) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+      if (lane == 0) mlpart[hq_idx] = make_float2(m1, l1);
     }
   }
 }
@@ -271,19 +341,20 @@ __global__ void __launch_bounds__(kDecCombineThreads)
   }
 }
 
-// Keys per chunk: about two CTAs per SM over the whole batch, a multiple of 64.
-int decode_chunk_keys(int64_t total_tokens) {
-  const int64_t ctas = 2 * static_cast<int64_t>(device_sm_count());
+// Keys per chunk: about one CTA per SM over the whole batch, a multiple of a stage.
+int decode_chunk_keys(int64_t total_tokens, int32_t hkv) {
+  const int64_t stage_tok = kStageBytes / (static_cast<int64_t>(hkv) * 256);
+  const int64_t ctas = device_sm_count();
   int64_t c = (total_tokens + ctas - 1) / std::max<int64_t>(1, ctas);
-  c = (c + 63) / 64 * 64;
-  return static_cast<int>(std::min<int64_t>(std::max<int64_t>(c, 64), 1 << 16));
+  c = (c + stage_tok - 1) / stage_tok * stage_tok;
+  return static_cast<int>(std::min<int64_t>(std::max<int64_t>(c, stage_tok), 1 << 20));
 }
 
 apack_status decode_validate(int32_t num_seqs, const int32_t *cu_seqlens_h, int32_t hq, int32_t hkv,
                              int64_t *total) {
   if (num_seqs < 0 || (num_seqs > 0 && !cu_seqlens_h)) return APACK_EINVAL;
   if (hq < 1 || hkv < 1 || hq % hkv != 0) return APACK_EINVAL;
-  if (hq / hkv > kDecRows || kDecWarps % hkv != 0) return APACK_EUNSUPPORTED;
+  if (hq / hkv > kDecRows || hkv > 8 || kDecConsumers % hkv != 0) return APACK_EUNSUPPORTED;
   if (num_seqs > 0 && cu_seqlens_h[0] != 0) return APACK_EINVAL;
   for (int b = 0; b < num_seqs; ++b)
     if (cu_seqlens_h[b + 1] < cu_seqlens_h[b]) return APACK_EINVAL;
@@ -307,10 +378,11 @@ apack_status apack_decode_workspace_size(int32_t num_seqs, const int32_t *cu_seq
   int64_t total = 0;
   const apack_status st = decode_validate(num_seqs, cu_seqlens_h, num_q_heads, num_kv_heads, &total);
   if (st != APACK_OK) return st;
-  const int chunk = decode_chunk_keys(total);
+  const int chunk = decode_chunk_keys(total, num_kv_heads);
   int64_t chunks = 0;
   for (int b = 0; b < num_seqs; ++b) chunks += (cu_seqlens_h[b + 1] - cu_seqlens_h[b] + chunk - 1) / chunk;
-  *bytes = up256(static_cast<size_t>(chunks) * num_q_heads * 128 * sizeof(float)) +
+  // device error word, chunk partials o [chunks][Hq][128] and (max, sum) [chunks][Hq]
+  *bytes = 256 + up256(static_cast<size_t>(chunks) * num_q_heads * 128 * sizeof(float)) +
            up256(static_cast<size_t>(chunks) * num_q_heads * sizeof(float2));
   return APACK_OK;
 }
@@ -323,20 +395,28 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
   if (st != APACK_OK) return st;
   if (num_seqs == 0) return APACK_OK;
   if (!q || !k || !v || !out || !ws) return APACK_EINVAL;
-  if ((reinterpret_cast<uintptr_t>(q) & 7) || (reinterpret_cast<uintptr_t>(k) & 7) ||
-      (reinterpret_cast<uintptr_t>(v) & 7) || (reinterpret_cast<uintptr_t>(out) & 15) ||
-      (reinterpret_cast<uintptr_t>(ws) & 255) || (kv_token_stride & 7) ||
+  if ((reinterpret_cast<uintptr_t>(q) & 7) || (reinterpret_cast<uintptr_t>(k) & 15) ||
+      (reinterpret_cast<uintptr_t>(v) & 15) || (reinterpret_cast<uintptr_t>(out) & 15) ||
+      (reinterpret_cast<uintptr_t>(ws) & 255) || (kv_token_stride & 15) ||
       kv_token_stride < static_cast<int64_t>(num_kv_heads) * 256)
     return APACK_EINVAL;
   size_t need = 0;
   apack_decode_workspace_size(num_seqs, cu_seqlens_h, num_q_heads, num_kv_heads, &need);
   if (ws_bytes < need) return APACK_EWORKSPACE;
-  const int chunk = decode_chunk_keys(total);
+  const int chunk = decode_chunk_keys(total, num_kv_heads);
   int64_t chunks_all = 0;
   for (int b = 0; b < num_seqs; ++b) chunks_all += (cu_seqlens_h[b + 1] - cu_seqlens_h[b] + chunk - 1) / chunk;
-  float *opart = static_cast<float *>(ws);
-  float2 *mlpart = reinterpret_cast<float2 *>(static_cast<uint8_t *>(ws) +
+  DeviceError *err = static_cast<DeviceError *>(ws);
+  float *opart = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + 256);
+  float2 *mlpart = reinterpret_cast<float2 *>(static_cast<uint8_t *>(ws) + 256 +
                                               up256(static_cast<size_t>(chunks_all) * num_q_heads * 128 * sizeof(float)));
+  static bool attr_done = false;
+  if (!attr_done) {
+    if (check_cuda(cudaFuncSetAttribute(decode_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        static_cast<int>(kDecSmem))) != APACK_OK)
+      return APACK_ECUDA;
+    attr_done = true;
+  }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const uint16_t *q16 = static_cast<const uint16_t *>(q);
   int64_t chunk_base = 0;
@@ -347,7 +427,7 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
     P.hq = num_q_heads;
     P.hkv = num_kv_heads;
     P.group = num_q_heads / num_kv_heads;
-    P.chunk = chunk;
+    P.chunk = chunk;                    // a multiple of the stage size
     P.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(APACK_HEAD_DIM)));
     int chunks = 0;
     for (int i = 0; i < ns; ++i) {
@@ -363,8 +443,9 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
     float2 *mp = mlpart + chunk_base * num_q_heads;
     const uint16_t *qs = q16 + static_cast<int64_t>(s0) * num_q_heads * 128;
     if (chunks > 0) {
-      decode_chunk_kernel<<<chunks, kDecThreads, 0, s>>>(P, qs, static_cast<const uint8_t *>(k),
-                                                         static_cast<const uint8_t *>(v), kv_token_stride, op, mp);
+      decode_chunk_kernel<<<chunks, kDecThreads, kDecSmem, s>>>(P, qs, static_cast<const uint8_t *>(k),
+                                                                static_cast<const uint8_t *>(v), kv_token_stride,
+                                                                op, mp, err);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }

@@ -41,9 +41,10 @@ def run(ap, cu, q, k, v, hq, hkv, pad_heads=0):
         vd[:, :hkv * 128] = torch.from_numpy(v.reshape(T, -1).view(np.int16)).cuda()
     qd = torch.from_numpy(q.view(np.int16)).cuda()
     out = torch.full((len(cu) - 1, hq, 128), float("nan"), dtype=torch.float32, device="cuda")
-    ws = torch.empty(max(256, ap.apack_decode_workspace_size(cu, hq, hkv)), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(max(256, ap.apack_decode_workspace_size(cu, hq, hkv)), dtype=torch.uint8, device="cuda")
     ap.apack_decode_attention(cu, qd, kd, vd, row * 2, hq, hkv, out, ws)
     torch.cuda.synchronize()
+    assert ap.apack_device_error(ws) == ap.APACK_OK
     return out.cpu().numpy()
 
 
