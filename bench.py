@@ -21,6 +21,7 @@ import argparse
 import hashlib
 import json
 import os
+import platform
 import subprocess
 import sys
 import threading
@@ -33,6 +34,7 @@ METRIC = "prune-step multimodal tokens/s; KV-compaction HBM GB/s vs peak (7B-sha
 UNIT = "multimodal tokens/s"
 WORKLOAD = "7b_10min"
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
 
 
 def parse():
@@ -71,6 +73,37 @@ def measured_peaks():
             d = json.load(f)
         return float(d.get("hbm_gbs", FALLBACK_HBM_GBS)), "measured"
     return FALLBACK_HBM_GBS, "fallback"
+
+
+def measured_tensor_peak():
+    """Sustained dense bf16 TFLOP/s (for kernels timed inside a long step)."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        if "bf16_tflops_sustained" in d:
+            return float(d["bf16_tflops_sustained"]), "measured (sustained)"
+    return FALLBACK_BF16_TFLOPS_SUSTAINED, "fallback (sustained)"
+
+
+def host_cpu():
+    """CPU model and logical cores of this host."""
+    model, arm = None, {}
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if ":" not in line:
+                    continue
+                key, val = (x.strip() for x in line.split(":", 1))
+                if key.lower() in ("model name", "cpu model", "processor name") and model is None:
+                    model = val
+                elif key in ("CPU implementer", "CPU part") and key not in arm:
+                    arm[key] = val
+    except OSError:
+        pass
+    if model is None and arm:
+        model = f"{platform.machine()} (implementer {arm.get('CPU implementer')}, part {arm.get('CPU part')})"
+    return {"cpu_model": model or platform.processor() or platform.machine(), "nproc": os.cpu_count()}
 
 
 def profiled_traffic(kernel_src, summary="gather_tma_traffic.json"):
@@ -225,7 +258,7 @@ def run_oracle(name, dur, reps):
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
-def cpu_sample_duration(name, budget_s, max_dur=120):
+def cpu_sample_duration(name, budget_s, max_dur=360):
     """Clip length (even seconds) whose oracle schedule takes about budget_s."""
     probe = run_oracle(name, 10, 1)
     per_s = probe["times"][0] / 10.0
@@ -237,7 +270,7 @@ def cpu_baseline(name, budget_s=15.0):
     dur = cpu_sample_duration(name, budget_s)
     d = run_oracle(name, dur, 1)
     v = d["mm"] / d["times"][0]
-    return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+    return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", **host_cpu(),
             "sample": f"first {dur} s of the {name} sequence ({d['tokens']} tokens), same heads, query rows and "
                       f"3-step schedule, single-threaded numpy fp64 oracle, {d['times'][0]:.1f} s"}
 
@@ -257,7 +290,7 @@ def reference_arm(args, rank, world):
             "warmup": args.warmup, "ms_per_step": 1e3 * t / len(times), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": args.workload, "sample_seconds": dur},
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample, **host_cpu()},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -293,7 +326,7 @@ def prellm_cpu_baseline(wl, frames=24):
     if r.returncode != 0:
         raise RuntimeError(r.stderr[-2000:])
     sec = json.loads(r.stdout.strip().splitlines()[-1])["seconds"]
-    return {"value": fs / sec, "unit": "frames/s", "cores": 1, "kind": "oracle",
+    return {"value": fs / sec, "unit": "frames/s", "cores": 1, "kind": "oracle", **host_cpu(),
             "sample": f"{fs} frames x {tpf} visual tokens, {nas} audio tokens, d={dim}; single-threaded numpy "
                       f"fp64 oracle (literal d x d products), {sec:.1f} s"}
 
@@ -350,6 +383,24 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
                          "traffic": traffic, "peak_source": peak_kind,
                          "algorithmic_bytes_per_launch": alg,
                          "note": "bf16 tokens read once + fp32 frame embeddings written once, over the whole call"}}
+
+
+def scoring_roofline(wl, pp, cuq, score_ms_per_step):
+    """Useful tensor work of the scoring stage: one Q K^T over the multimodal keys per
+    step (2 n_q Hq |S| D flop).  The two-pass softmax computes Q K^T twice and every
+    logit also needs one exp2 per pass (the SFU is the second ceiling), so this
+    fraction understates how busy the tensor pipe is."""
+    import numpy as np
+    nq = int(cuq[-1])
+    flops = [2.0 * nq * wl.num_q_heads * s * wl.head_dim for s in pp.mm_tokens_per_step()]
+    ms = float(np.sum(score_ms_per_step))
+    achieved = sum(flops) / (ms / 1e3) / 1e12
+    peak, kind = measured_tensor_peak()
+    return {"bound": "tensor", "kernel": "score_rowstats_kernel + score_colsum_kernel (+ q_pack, merge, finalize)",
+            "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+            "peak_source": kind, "useful_flops_per_iter": sum(flops),
+            "logits_per_iter": sum(flops) / (2.0 * wl.head_dim), "exp2_per_iter": 2 * sum(flops) / (2.0 * wl.head_dim),
+            "note": "useful flops = one Q K^T per step over the multimodal keys; the stage runs two passes"}
 
 
 def decode_measure(ap, wl, pp, steps, warmup, stream, dist):
@@ -580,6 +631,7 @@ def main():
                          "traffic": traffic, "peak_source": peak_kind,
                          "algorithmic_bytes_per_launch": comp_bytes,
                          "avg_launch_ms": [float(x) for x in comp_ms]},
+            "roofline_scoring": scoring_roofline(wl, pp, cuq, stage_ms[:, 0]),
             "stages_ms_per_iter": {"score": float(score_ms), "select": float(select_ms),
                                    "compact": float(comp_ms.sum())},
             "e2e": {"value": whole_job_value(mm_per_iter, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": int(h2d),

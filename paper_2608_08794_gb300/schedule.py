@@ -15,8 +15,14 @@ Only buffer management and argument marshalling happen here.
 import numpy as np
 import torch
 
-from . import (Seqs, apack_prune_step, apack_prune_schedule, apack_workspace_size, apack_keep_counts,
+from . import (Seqs, apack_plane, apack_prune_step, apack_prune_schedule, apack_workspace_size, apack_keep_counts,
                APACK_HEAD_DIM, APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT)
+
+
+def _plane(src, dst, src_plane_stride, dst_plane_stride, row_bytes, num_planes):
+    return apack_plane(src=src, dst=dst, src_plane_stride=src_plane_stride, dst_plane_stride=dst_plane_stride,
+                       src_row_stride=row_bytes, dst_row_stride=row_bytes, row_bytes=row_bytes,
+                       num_planes=num_planes)
 
 
 def schedule_keep_counts(cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, num_kv_heads, modality,
@@ -45,8 +51,13 @@ def schedule_keep_counts(cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, n
 class ProgressivePrune:
     def __init__(self, cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, num_kv_heads, num_layers, hidden_dim,
                  prune_layers, keep_counts, device="cuda", select_mode=APACK_SELECT_PER_MODALITY,
-                 with_hidden=True):
-        """keep_counts[i]: int array [B, 2] of the tokens each segment keeps after step i."""
+                 with_hidden=True, slice_below=False):
+        """keep_counts[i]: int array [B, 2] of the tokens each segment keeps after step i.
+
+        slice_below: also compact, at every step, the K/V of the layers below its
+        pruning layer, so that after the schedule every layer's cache holds only the
+        kept tokens (for decoding).  The caches of layers [0, l_0) are then inputs
+        too (``k_low_in`` / ``v_low_in``); ``output_low_kv`` gives layers [0, l_i)."""
         self.dev = torch.device(device)
         self.cu0 = np.asarray(cu_seqlens, np.int32)
         self.cuq = np.asarray(cu_qlens, np.int32)
@@ -77,6 +88,14 @@ class ProgressivePrune:
         self.h_out = [torch.empty((t1, hidden_dim), dtype=torch.bfloat16, device=dev) if with_hidden else None
                       for _ in range(2)]
         self.mod_out = [torch.empty(t1, dtype=torch.uint8, device=dev) for _ in range(2)]
+        self.slice_below = slice_below
+        if slice_below:
+            l0, l_last = self.layers[0], self.layers[-1]
+            self.k_low_in = torch.empty((l0, T0, num_kv_heads, APACK_HEAD_DIM), dtype=torch.bfloat16, device=dev)
+            self.v_low_in = torch.empty_like(self.k_low_in)
+            self.k_low = [torch.empty(max(1, l_last * t1 * self.row // 2), dtype=torch.bfloat16, device=dev)
+                          for _ in range(2)]
+            self.v_low = [torch.empty_like(self.k_low[0]) for _ in range(2)]
         self.keep_idx = [torch.empty(max(1, t), dtype=torch.int32, device=dev) for t in self.t_out]
         self.scores = torch.empty(max(1, T0), dtype=torch.float32, device=dev)
         self._seqs = []
@@ -126,7 +145,8 @@ class ProgressivePrune:
             o = i % 2
             steps.append(dict(layer=self.layers[i], q=self.q[i], keep_count=self.counts[i], k_out=self.k_out[o],
                               v_out=self.v_out[o], kv_out_layer_stride=self.t_out[i] * self.row,
-                              hidden_out=self.h_out[o], modality_out=self.mod_out[o], keep_idx=self.keep_idx[i]))
+                              hidden_out=self.h_out[o], modality_out=self.mod_out[o], keep_idx=self.keep_idx[i],
+                              extra_planes=self._below_planes(i)))
         flat = None
         if events is not None:
             flat = [e for per_step in events for e in per_step]
@@ -154,6 +174,35 @@ class ProgressivePrune:
             hidden_out=self.h_out[o], modality_out=self.mod_out[o], keep_idx=self.keep_idx[i],
             scores=self.scores, ws=self.ws, stage_events=events, stream=stream)
         return self.new_cu[i]
+
+    def _below_planes(self, i):
+        """Extra planes of step i when slicing below: layers [0, l_(i-1)) from the
+        previous below-cache and layers [l_(i-1), l_i) from the previous step's main
+        output (for step 0: layers [0, l_0) from the inputs), into layers [0, l_i)."""
+        if not self.slice_below:
+            return ()
+        row, t = self.row, self.t_out[i]
+        o = i % 2
+        groups = []
+        for src_in, out, low in ((self.k_low_in, self.k_out, self.k_low), (self.v_low_in, self.v_out, self.v_low)):
+            dst = low[o].data_ptr()
+            if i == 0:
+                if self.layers[0] > 0:
+                    groups.append(_plane(src_in.data_ptr(), dst, self.T0 * row, t * row, row, self.layers[0]))
+                continue
+            p, tp = (i - 1) % 2, self.t_out[i - 1]
+            lp, li = self.layers[i - 1], self.layers[i]
+            if lp > 0:
+                groups.append(_plane(low[p].data_ptr(), dst, tp * row, t * row, row, lp))
+            groups.append(_plane(out[p].data_ptr(), dst + lp * t * row, tp * row, t * row, row, li - lp))
+        return groups
+
+    def output_low_kv(self, i):
+        """Views of step i's below-layer caches (slice_below): [l_i, t_out_i, Hkv, D]."""
+        o = i % 2
+        n = self.layers[i] * self.t_out[i] * self.row // 2
+        shape = (self.layers[i], self.t_out[i], self.hkv, APACK_HEAD_DIM)
+        return self.k_low[o][:n].view(shape), self.v_low[o][:n].view(shape)
 
     def output_kv(self, i):
         """Views of step i's compacted K and V: [L - l_i, t_out_i, Hkv, D]."""

@@ -47,6 +47,10 @@ def fill_progressive_inputs(pp, wl):
     for j in range(pp.k_in.shape[0]):
         fill_normal_bf16(pp.k_in[j], wl.seed, TID_K + l0 + j)
         fill_normal_bf16(pp.v_in[j], wl.seed, TID_V + l0 + j)
+    if getattr(pp, "slice_below", False):
+        for j in range(pp.k_low_in.shape[0]):
+            fill_normal_bf16(pp.k_low_in[j], wl.seed, TID_K + j)
+            fill_normal_bf16(pp.v_low_in[j], wl.seed, TID_V + j)
     if pp.hidden_in is not None:
         fill_normal_bf16(pp.hidden_in, wl.seed, TID_HIDDEN)
     pp.modality_in.copy_(torch.from_numpy(wl.modality()))

@@ -168,3 +168,41 @@ def test_schedule_runner_is_bit_identical_to_single_steps(ap, name):
     torch.cuda.synchronize()
     assert ap.apack_device_error(pp.ws) == ap.APACK_OK
     same(ref, snapshot(pp))
+
+
+@pytest.mark.parametrize("name", ["7b_2min", "7b_10min_paper"])
+def test_slicing_below_the_pruning_layers_keeps_every_layer_consistent(ap, name):
+    """With slice_below, every step also compacts the caches of the layers below its
+    pruning layer; afterwards layer j's cache holds the original rows of layer j at
+    the tokens kept by all steps, for every layer (checked bit for bit)."""
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+
+    wl = workload(name)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod_d = torch.from_numpy(wl.modality()).cuda()
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_d,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
+    pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                          wl.prune_layers, counts, select_mode=mode, slice_below=True)
+    fill_progressive_inputs(pp, wl)
+    pp.run()
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+    composite = torch.arange(wl.total_tokens, device="cuda")
+    for i in range(len(wl.prune_layers)):
+        composite = composite.index_select(0, pp.keep_idx[i][:pp.t_out[i]].long())
+    last = len(wl.prune_layers) - 1
+    l0, l_last = wl.prune_layers[0], wl.prune_layers[last]
+    low_k, low_v = pp.output_low_kv(last)
+    top_k, top_v = pp.output_kv(last)
+    for j in range(wl.num_layers):
+        src_k = pp.k_low_in[j] if j < l0 else pp.k_in[j - l0]
+        src_v = pp.v_low_in[j] if j < l0 else pp.v_in[j - l0]
+        got_k = low_k[j] if j < l_last else top_k[j - l_last]
+        got_v = low_v[j] if j < l_last else top_v[j - l_last]
+        assert torch.equal(got_k.view(torch.int16), src_k.index_select(0, composite).view(torch.int16)), j
+        assert torch.equal(got_v.view(torch.int16), src_v.index_select(0, composite).view(torch.int16)), j
