@@ -216,14 +216,15 @@ __device__ __forceinline__ Unit1 decode_unit1(const ScorePlan &p, int u) {
 // is only raised when a value exceeds it by 2^64 (sum overflow check), which
 // keeps the max computation off the common path.  Four independent partial
 // sums keep the add chain short.
-__device__ __forceinline__ void online_chunk(const uint32_t (&r)[32], uint32_t mask, float c2, float &m,
+template <int OFF>
+__device__ __forceinline__ void online_chunk(const uint32_t (&r)[64], uint32_t mask, float c2, float &m,
                                              float &sum) {
   if (mask == 0u) return;
   if (m == -INFINITY) {
     float mx = -INFINITY;
 #pragma unroll
     for (int i = 0; i < 32; ++i)
-      if ((mask >> i) & 1u) mx = fmaxf(mx, __uint_as_float(r[i]));
+      if ((mask >> i) & 1u) mx = fmaxf(mx, __uint_as_float(r[OFF + i]));
     m = mx * c2;
   }
   float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
@@ -231,13 +232,13 @@ __device__ __forceinline__ void online_chunk(const uint32_t (&r)[32], uint32_t m
   if (mask == 0xffffffffu) {
 #pragma unroll
     for (int i = 0; i < 32; i += 2) {
-      const float2 y = ffma2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), cc, nm);
+      const float2 y = ffma2(make_float2(__uint_as_float(r[OFF + i]), __uint_as_float(r[OFF + i + 1])), cc, nm);
       a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(y.x), ex2_approx(y.y)));
     }
   } else {
 #pragma unroll
     for (int i = 0; i < 32; i += 2) {
-      const float2 y = ffma2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), cc, nm);
+      const float2 y = ffma2(make_float2(__uint_as_float(r[OFF + i]), __uint_as_float(r[OFF + i + 1])), cc, nm);
       a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(((mask >> i) & 1u) ? ex2_approx(y.x) : 0.f,
                                                            ((mask >> (i + 1)) & 1u) ? ex2_approx(y.y) : 0.f));
     }
@@ -249,14 +250,14 @@ __device__ __forceinline__ void online_chunk(const uint32_t (&r)[32], uint32_t m
     float mx = -INFINITY;
 #pragma unroll
     for (int i = 0; i < 32; ++i)
-      if ((mask >> i) & 1u) mx = fmaxf(mx, __uint_as_float(r[i]));
+      if ((mask >> i) & 1u) mx = fmaxf(mx, __uint_as_float(r[OFF + i]));
     mx *= c2;
     sum *= ex2_approx(m - mx);
     m = mx;
     t = 0.f;
 #pragma unroll
     for (int i = 0; i < 32; ++i)
-      if ((mask >> i) & 1u) t += ex2_approx(fmaf(__uint_as_float(r[i]), c2, -m));
+      if ((mask >> i) & 1u) t += ex2_approx(fmaf(__uint_as_float(r[OFF + i]), c2, -m));
   }
   sum += t;
 }
@@ -382,16 +383,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         if (active && (mask[0] | mask[1])) {
           const uint32_t tcol = bars->tmem_base + lane_off + ci * 256 + t * 128 + h * 64;
-          uint32_t ra[32], rb[32];
-          tmem_ld32(tcol, ra);
-          tmem_ld32(tcol + 32, rb);
-          tmem_wait32(ra);
-          tmem_wait32(rb);
+          uint32_t rr[64];
+          tmem_ld64_wait(tcol, rr);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->acc_empty[ci]);   // registers hold the data: release early
-          online_chunk(ra, mask[0], c2, m, sum);
-          online_chunk(rb, mask[1], c2, m, sum);
+          online_chunk<0>(rr, mask[0], c2, m, sum);
+          online_chunk<32>(rr, mask[1], c2, m, sum);
         } else {
           tc_fence_before();
           __syncwarp();
@@ -492,14 +490,16 @@ __device__ __forceinline__ Unit2 decode_unit2(const ScorePlan &p, int u) {
 }
 
 // a[0..3] += 2^(x c2 + nl[col]) over 32 columns (four independent partial sums).
-__device__ __forceinline__ void colsum_chunk(const uint32_t (&r)[32], const float *nl, float c2, float2 (&a)[4]) {
+template <int OFF>
+__device__ __forceinline__ void colsum_chunk(const uint32_t (&r)[64], const float *nl, float c2, float2 (&a)[4]) {
   const float2 cc = make_float2(c2, c2);
 #pragma unroll
   for (int i = 0; i < 32; i += 4) {
     const float4 L = *reinterpret_cast<const float4 *>(nl + i);
-    const float2 y0 = ffma2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), cc, make_float2(L.x, L.y));
-    const float2 y1 =
-        ffma2(make_float2(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])), cc, make_float2(L.z, L.w));
+    const float2 y0 = ffma2(make_float2(__uint_as_float(r[OFF + i]), __uint_as_float(r[OFF + i + 1])), cc,
+                            make_float2(L.x, L.y));
+    const float2 y1 = ffma2(make_float2(__uint_as_float(r[OFF + i + 2]), __uint_as_float(r[OFF + i + 3])), cc,
+                            make_float2(L.z, L.w));
     a[(i >> 2) & 3] = fadd2(a[(i >> 2) & 3], make_float2(ex2_approx(y0.x), ex2_approx(y0.y)));
     a[(i >> 2) & 3] = fadd2(a[(i >> 2) & 3], make_float2(ex2_approx(y1.x), ex2_approx(y1.y)));
   }
@@ -620,16 +620,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (active) {
           const float *nl = lse_s + li * kBRows + h * 64;
           const uint32_t tcol = bars->tmem_base + lane_off + ci * 256 + t * 128 + h * 64;
-          uint32_t ra[32], rb[32];
-          tmem_ld32(tcol, ra);
-          tmem_ld32(tcol + 32, rb);
-          tmem_wait32(ra);
-          tmem_wait32(rb);
+          uint32_t rr[64];
+          tmem_ld64_wait(tcol, rr);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->acc_empty[ci]);   // registers hold the data: release early
-          colsum_chunk(ra, nl, c2, a);
-          colsum_chunk(rb, nl + 32, c2, a);
+          colsum_chunk<0>(rr, nl, c2, a);
+          colsum_chunk<32>(rr, nl + 32, c2, a);
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->l_empty[li]);
         } else {
