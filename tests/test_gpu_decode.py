@@ -107,3 +107,15 @@ def test_decode_attention_rejects_unsupported_groups(ap):
         ap.apack_decode_workspace_size(cu, 32, 2)            # 16 query rows per KV head
     with pytest.raises(ap.ApackError):
         ap.apack_decode_workspace_size(np.array([0, 5, 3], np.int32), 28, 4)   # decreasing offsets
+
+
+def test_decode_attention_batch_beyond_one_launch(ap):
+    # 70 sequences: the chunk and combine kernels run in two launches
+    rng = np.random.default_rng(70)
+    lens = [int(x) for x in rng.integers(0, 700, 70)]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = int(cu[-1])
+    q = bits(rng, (70, 28, 128))
+    k = bits(rng, (T, 4, 128), 1.5)
+    v = bits(rng, (T, 4, 128))
+    check(run(ap, cu, q, k, v, 28, 4), oracle.decode_attention(q, k, v, cu, 28, 4))

@@ -293,3 +293,34 @@ def test_compact_strided_destination_rows(ap):
     out = d.cpu().numpy()
     np.testing.assert_array_equal(out[:, :, :rb], src[:, keep, :])
     assert not out[:, :, rb:].any()
+
+
+# ------------------------------------------------------------------------------ batch limits
+
+@pytest.mark.parametrize("path", ["narrow", "wide"])
+def test_scores_batch_beyond_one_launch(ap, path):
+    # 70 sequences: more than one launch's 64, on both scoring paths
+    rng = np.random.default_rng(70 if path == "narrow" else 71)
+    lens = [int(x) for x in rng.integers(0, 400, 70)]
+    nqs = [int(x) for x in (rng.integers(0, 4, 70) if path == "narrow" else rng.integers(5, 41, 70))]
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, lens, nqs, 28, 4)
+    got = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, 28, 4)
+    check_scores(got, oracle.relevance_scores(q, k, cu, cuq, mod, 28, 4))
+
+
+def test_maximum_number_of_sequences(ap):
+    # APACK_MAX_SEQS short sequences through scoring (narrow path) and selection
+    rng = np.random.default_rng(4096)
+    B = 4096
+    lens = [int(x) for x in rng.integers(0, 40, B)]
+    nqs = [int(x) for x in rng.integers(0, 2, B)]
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, lens, nqs, 4, 2)
+    got = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, 4, 2)
+    ref = oracle.relevance_scores(q, k, cu, cuq, mod, 4, 2)
+    check_scores(got, ref)
+    counts = [(a // 2, (v * 3) // 4) for a, v in zip(na, nv)]
+    keep, mod_o, _, ncu, err = gpu_select(ap, got, mod, cu, counts, na, nv, 0)
+    assert err == ap.APACK_OK
+    ref_keep = oracle.select_keep(got, mod, cu, counts)
+    np.testing.assert_array_equal(keep, ref_keep)
+    np.testing.assert_array_equal(ncu, oracle.new_cu_seqlens(ref_keep, cu))
