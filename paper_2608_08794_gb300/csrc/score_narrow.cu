@@ -19,6 +19,7 @@
 //                   in a fixed order and scales by 1/(Hq n_q).
 // The logits of the 10-minute 7B sequence with one query row take 15 MB and stay
 // in L2 between the first and the last kernel.
+#include <algorithm>
 #include <cmath>
 
 #include "internal.cuh"
@@ -30,14 +31,20 @@ namespace {
 
 constexpr int kThreads = 256;          // keys per CTA (general logits kernel, final kernel)
 constexpr int kWarps = kThreads / 32;
-constexpr int kRows8Tokens = 64;       // keys per CTA of the rows8 logits kernel
+constexpr int kRows8Tokens = 64;       // smallest key chunk of the rows8 logits kernel (sizes partials)
+constexpr int kStrmWarps = 16;         // rows8 kernel: warps per CTA (lane 0 of the last also loads)
+constexpr int kStrmThreads = kStrmWarps * 32;
+constexpr int kStrmStages = 3;
+constexpr int kStrmStageBytes = 65536; // K rows per stage: 64 tokens of 4 KV heads, 128 of 2
+constexpr size_t kStrmSmem = static_cast<size_t>(kStrmStages) * kStrmStageBytes + 2 * kStrmStages * sizeof(uint64_t) +
+                             kStrmWarps * 16 * sizeof(float2) + 16;
 constexpr int kLogitPad = 64;          // logit row stride: the key count rounded up to this
 
 struct NSeq {
   int32_t t0, len;
   int32_t q_off, n_q;
   int32_t unit_begin;                  // first 256-key CTA of this sequence (general logits, final)
-  int32_t unit8_begin;                 // first CTA of this sequence in the rows8 logits kernel
+  int32_t unit8_begin;                 // first chunk (CTA) of this sequence in the rows8 logits kernel
   int32_t nparts;                      // CTA partials of the logits kernel in use
   int32_t rows;                        // logit rows R = Hq * n_q
   int64_t lstride;                     // logit row stride: len rounded up to kLogitPad
@@ -50,6 +57,7 @@ struct NarrowPlan {
   int32_t nseq;
   int32_t total_units;
   int32_t total_units8;
+  int32_t chunk;                       // keys per CTA of the rows8 kernel (a multiple of a stage)
   int32_t hq, hkv, group;
   float scale2;
   NSeq seq[kSeqsPerLaunch];
@@ -170,23 +178,68 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
-// rows8 logits kernel: KV heads in pairs, a warp per (head pair, run of tokens).  Lane
-// l works on head 2 hp + (l >> 4) and features [8 (l & 15), 8 (l & 15) + 8) of it.
-// NPAIR = Hkv / 2 head pairs; a CTA covers kRows8Tokens keys.
+// rows8 logits kernel (Hkv = 2 or 4, at most 8 rows per head group): one CTA per chunk
+// of a sequence's keys (about T / #SMs keys).  The chunk's K rows stream into a ring of
+// kStrmStages shared-memory stages by bulk async copies (64 KB per stage: 64 tokens of
+// 4 KV heads or 128 of 2); lane 0 of the last warp issues them and refills a slot once all
+// warps have released it.  Warp w takes head pair w % NPAIR and the group of 8 keys
+// (w / NPAIR) of every stage; lane l works on head 2 hp + (l >> 4) and features
+// [8 (l & 15), 8 (l & 15) + 8), with its query slice in registers.  Per CTA it writes the
+// (max, sum of exp2) of every logit row over its multimodal keys.
 template <int NPAIR>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kStrmThreads, 1)
     score_narrow_rows8_kernel(const __grid_constant__ NarrowPlan plan, const uint16_t *__restrict__ q,
                               const uint8_t *__restrict__ k, int64_t k_stride, const uint8_t *__restrict__ modality,
-                              float *__restrict__ logits, float2 *__restrict__ part) {
-  constexpr int kTokensPerWarp = kRows8Tokens * NPAIR / kWarps;   // 8 or 16
-  __shared__ float2 wst[kWarps][16];
-  const int s = find_unit8_seq(plan, blockIdx.x);
+                              float *__restrict__ logits, float2 *__restrict__ part, DeviceError *err) {
+  extern __shared__ __align__(1024) uint8_t dsm[];
+  uint8_t *stage_base = dsm;
+  uint64_t *full = reinterpret_cast<uint64_t *>(dsm + kStrmStages * kStrmStageBytes);
+  uint64_t *empty = full + kStrmStages;
+  float2 *wst = reinterpret_cast<float2 *>(empty + kStrmStages);          // [warp][16]
+  int *abort_flag = reinterpret_cast<int *>(wst + kStrmWarps * 16);
+  const int c = blockIdx.x;
+  const int s = find_unit8_seq(plan, c);
   const NSeq &sq = plan.seq[s];
   const int G = plan.group;
   const int rg = G * sq.n_q;
-  if (rg == 0) return;                                   // no query row: nothing to score
+  if (rg == 0) return;                                   // no query row: nothing to score (CTA-uniform)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int hp = warp % NPAIR, tb = warp / NPAIR;
+  const int64_t row = static_cast<int64_t>(plan.hkv) * 256;
+  const int stage_tok = kStrmStageBytes / static_cast<int>(row);
+  const int tb = (c - sq.unit8_begin) * plan.chunk;
+  const int te = min(sq.len, tb + plan.chunk);
+  const int nst = (te - tb + stage_tok - 1) / stage_tok;
+  const bool loader = warp == kStrmWarps - 1 && lane == 0;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStrmStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], kStrmWarps);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  volatile int *abort_v = abort_flag;
+  const uint8_t *kseq = k + static_cast<int64_t>(sq.t0) * k_stride;
+  auto issue = [&](int n) {
+    const int slot = n % kStrmStages;
+    const int t = tb + n * stage_tok;
+    const int cnt = min(stage_tok, te - t);
+    uint8_t *dst = stage_base + static_cast<size_t>(slot) * kStrmStageBytes;
+    mbar_arrive_expect_tx(&full[slot], static_cast<uint32_t>(cnt * row));
+    if (k_stride == row) {
+      bulk_load(dst, kseq + static_cast<int64_t>(t) * k_stride, static_cast<uint32_t>(cnt * row), &full[slot]);
+    } else {
+      for (int r = 0; r < cnt; ++r)
+        bulk_load(dst + r * row, kseq + static_cast<int64_t>(t + r) * k_stride, static_cast<uint32_t>(row),
+                  &full[slot]);
+    }
+  };
+  int issued = 0;
+  if (loader)
+    for (; issued < kStrmStages && issued < nst; ++issued) issue(issued);
+
+  const int hp = warp % NPAIR, grp = warp / NPAIR;
   const int h = 2 * hp + (lane >> 4), part16 = lane & 15;
   // query slice: rows j < rg of head group h (logit row (j / G) Hq + h G + j % G)
   float qf[8][8];
@@ -201,97 +254,119 @@ __global__ void __launch_bounds__(kThreads, 2)
   const bool row_ok = r < rg;
   const int rho = row_ok ? (r / G) * plan.hq + h * G + r % G : 0;
   const bool b1 = lane & 8, b2 = lane & 4, b3 = lane & 2;
-  const int unit = blockIdx.x - sq.unit8_begin;
-  const int tok0 = unit * kRows8Tokens + tb * kTokensPerWarp;
-  const uint8_t *kbase = k + static_cast<int64_t>(sq.t0) * k_stride + h * 256 + part16 * 16;
   float m = -INFINITY, ssum = 0.f;
-#pragma unroll 1
-  for (int c0 = 0; c0 < kTokensPerWarp; c0 += 8) {
-    uint4 kv[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int t = tok0 + c0 + i;
-      kv[i] = t < sq.len ? __ldg(reinterpret_cast<const uint4 *>(kbase + static_cast<int64_t>(t) * k_stride))
-                         : make_uint4(0, 0, 0, 0);
+  for (int n = 0; n < nst; ++n) {
+    const int slot = n % kStrmStages;
+    if (!__all_sync(0xffffffffu, mbar_wait(&full[slot], (n / kStrmStages) & 1u, kWaitLimitNs))) {
+      if (lane == 0) {
+        raise_device_error(err, APACK_ETIMEOUT, 71, c, n);
+        *abort_v = 1;
+      }
+      break;
     }
-    const int tl = tok0 + c0 + (lane & 7);
-    const unsigned mmask = __ballot_sync(0xffffffffu, lane < 8 && tl < sq.len && is_mm(modality[sq.t0 + tl]));
-    float outv[8];
+    const int t0 = tb + n * stage_tok + grp * 8;
+    const int valid = min(8, te - t0);
+    if (valid > 0) {
+      const uint8_t *ks = stage_base + static_cast<size_t>(slot) * kStrmStageBytes +
+                          static_cast<size_t>(grp) * 8 * row + h * 256 + part16 * 16;
+      const int tl = t0 + (lane & 7);
+      const unsigned mmask = __ballot_sync(0xffffffffu, lane < 8 && tl < te && is_mm(modality[sq.t0 + tl]));
+      float outv[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      float kf[8];
-      bf16x8_to_f32(kv[i], kf);
-      float acc[8];
+      for (int i = 0; i < 8; ++i) {
+        float kf[8];
+        bf16x8_to_f32(i < valid ? *reinterpret_cast<const uint4 *>(ks + i * row) : make_uint4(0, 0, 0, 0), kf);
+        float acc[8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        float2 a = make_float2(0.f, 0.f);
+        for (int j = 0; j < 8; ++j) {
+          float2 a2 = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int e = 0; e < 4; ++e)
-          a = ffma2(make_float2(kf[2 * e], kf[2 * e + 1]), make_float2(qf[j][2 * e], qf[j][2 * e + 1]), a);
-        acc[j] = a.x + a.y;
+          for (int e = 0; e < 4; ++e)
+            a2 = ffma2(make_float2(kf[2 * e], kf[2 * e + 1]), make_float2(qf[j][2 * e], qf[j][2 * e + 1]), a2);
+          acc[j] = a2.x + a2.y;
+        }
+        // reduce-scatter over the 16 lanes of the head: lane bits 3, 2, 1 pick the row
+        float v4[4], v2[2];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float send = b1 ? acc[e] : acc[e + 4];
+          const float keep = b1 ? acc[e + 4] : acc[e];
+          v4[e] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+        }
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const float send = b2 ? v4[e] : v4[e + 2];
+          const float keep = b2 ? v4[e + 2] : v4[e];
+          v2[e] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+        }
+        float v1;
+        {
+          const float send = b3 ? v2[0] : v2[1];
+          const float keep = b3 ? v2[1] : v2[0];
+          v1 = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+        }
+        v1 += __shfl_xor_sync(0xffffffffu, v1, 1);
+        outv[i] = v1 * plan.scale2;
       }
-      // reduce-scatter over the 16 lanes of the head: lane bits 3, 2, 1 pick the row
-      float v4[4], v2[2];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float send = b1 ? acc[e] : acc[e + 4];
-        const float keep = b1 ? acc[e + 4] : acc[e];
-        v4[e] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
-      }
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const float send = b2 ? v4[e] : v4[e + 2];
-        const float keep = b2 ? v4[e + 2] : v4[e];
-        v2[e] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
-      }
-      float v1;
-      {
-        const float send = b3 ? v2[0] : v2[1];
-        const float keep = b3 ? v2[1] : v2[0];
-        v1 = keep + __shfl_xor_sync(0xffffffffu, send, 2);
-      }
-      v1 += __shfl_xor_sync(0xffffffffu, v1, 1);
-      outv[i] = v1 * plan.scale2;
-    }
-    // running (max, sum of exp2) of this lane's row over the chunk's multimodal keys
-    float cm = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      if ((mmask >> i) & 1u) cm = fmaxf(cm, outv[i]);
-    if (cm != -INFINITY) {
-      if (cm > m) {
-        ssum *= ex2_approx(m - cm);
-        m = cm;
-      }
+      // running (max, sum of exp2) of this lane's row over the group's multimodal keys
+      float cm = -INFINITY;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
-        if ((mmask >> i) & 1u) ssum += ex2_approx(outv[i] - m);
+        if ((mmask >> i) & 1u) cm = fmaxf(cm, outv[i]);
+      if (cm != -INFINITY) {
+        if (cm > m) {
+          ssum *= ex2_approx(m - cm);
+          m = cm;
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if ((mmask >> i) & 1u) ssum += ex2_approx(outv[i] - m);
+      }
+      if (row_ok) {   // the lane pair writes the group's 8 logits of its row: 4 each
+        const bool odd = lane & 1;
+        const float4 w = odd ? make_float4(outv[4], outv[5], outv[6], outv[7])
+                             : make_float4(outv[0], outv[1], outv[2], outv[3]);
+        *reinterpret_cast<float4 *>(logits + sq.logit_base + static_cast<int64_t>(rho) * sq.lstride + t0 +
+                                    (odd ? 4 : 0)) = w;
+      }
     }
-    if (row_ok) {   // the lane pair writes the chunk's 8 logits of its row: 4 each
-      const bool odd = lane & 1;
-      const float4 w = odd ? make_float4(outv[4], outv[5], outv[6], outv[7])
-                           : make_float4(outv[0], outv[1], outv[2], outv[3]);
-      *reinterpret_cast<float4 *>(logits + sq.logit_base + static_cast<int64_t>(rho) * sq.lstride + tok0 + c0 +
-                                  (odd ? 4 : 0)) = w;
+    __syncwarp();                        // this warp is done with the stage
+    if (lane == 0) mbar_arrive(&empty[slot]);
+    if (loader && issued < nst) {
+      // every warp has released stage n: refill its slot
+      if (!mbar_wait(&empty[slot], (n / kStrmStages) & 1u, kWaitLimitNs)) {
+        raise_device_error(err, APACK_ETIMEOUT, 72, c, n);
+        *abort_v = 1;
+      } else {
+        issue(issued);
+        ++issued;
+      }
     }
+    __syncwarp();
+    if (*abort_v) break;
   }
-  if ((lane & 1) == 0) wst[warp][lane >> 1] = make_float2(m, ssum);
+  // after an abort, stages may still be in flight: wait for them (bounded) before exit
+  if (loader && *abort_v)
+    for (int n = max(0, issued - kStrmStages); n < issued; ++n)
+      mbar_wait(&full[n % kStrmStages], (n / kStrmStages) & 1u, kWaitLimitNs / 4);
+  if ((lane & 1) == 0) wst[warp * 16 + (lane >> 1)] = make_float2(m, ssum);
   __syncthreads();
-  // per (head, row): combine the warps of its head pair in token order
+  if (*abort_v) return;
+  // per (head, row): combine the warps of its head pair in key order
   if (threadIdx.x < 16 * NPAIR) {
     const int php = threadIdx.x >> 4, slot = threadIdx.x & 15;
     const int rr = slot & 7, hh = 2 * php + (slot >> 3);
     if (rr < rg) {
       float mx = -INFINITY;
-      for (int b = 0; b < kWarps / NPAIR; ++b) mx = fmaxf(mx, wst[b * NPAIR + php][slot].x);
+      for (int g2 = 0; g2 < kStrmWarps / NPAIR; ++g2) mx = fmaxf(mx, wst[(g2 * NPAIR + php) * 16 + slot].x);
       float sum = 0.f;
       if (mx != -INFINITY)
-        for (int b = 0; b < kWarps / NPAIR; ++b) {
-          const float2 v = wst[b * NPAIR + php][slot];
+        for (int g2 = 0; g2 < kStrmWarps / NPAIR; ++g2) {
+          const float2 v = wst[(g2 * NPAIR + php) * 16 + slot];
           if (v.x != -INFINITY) sum += v.y * ex2_approx(v.x - mx);
         }
       const int rh = (rr / G) * plan.hq + hh * G + rr % G;
-      part[sq.part_base + static_cast<int64_t>(unit) * sq.rows + rh] = make_float2(mx, sum);
+      part[sq.part_base + static_cast<int64_t>(c - sq.unit8_begin) * sq.rows + rh] = make_float2(mx, sum);
     }
   }
 }
@@ -358,15 +433,18 @@ __global__ void __launch_bounds__(kThreads)
   if (key >= sq.t0 + sq.len) return;
   float out = 0.f;
   if (sq.n_q > 0 && is_mm(modality[key])) {
+    // eight independent sums, the loads of a block of 8 rows issued together
     const float *lp = logits + sq.logit_base + (key - sq.t0);
-    float a0 = 0.f, a1 = 0.f;
-    int rho = 0;
-    for (; rho + 1 < R; rho += 2) {
-      a0 += ex2_approx(lp[static_cast<int64_t>(rho) * sq.lstride] - ls[rho]);
-      a1 += ex2_approx(lp[static_cast<int64_t>(rho + 1) * sq.lstride] - ls[rho + 1]);
+    float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int r0 = 0; r0 < R; r0 += 8) {
+      float x[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        x[u] = r0 + u < R ? lp[static_cast<int64_t>(r0 + u) * sq.lstride] - ls[r0 + u] : -INFINITY;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) a[u] += ex2_approx(x[u]);
     }
-    if (rho < R) a0 += ex2_approx(lp[static_cast<int64_t>(rho) * sq.lstride] - ls[rho]);
-    out = (a0 + a1) / static_cast<float>(plan.hq * sq.n_q);
+    out = (((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]))) / static_cast<float>(plan.hq * sq.n_q);
   }
   scores[key] = out;
 }
@@ -382,6 +460,22 @@ cudaError_t launch_logits(int grid, size_t smem, cudaStream_t stream, const Narr
     attr = true;
   }
   score_narrow_logits_kernel<RG><<<grid, kThreads, smem, stream>>>(P, q, k, k_stride, modality, logits, part);
+  return cudaGetLastError();
+}
+
+template <int NPAIR>
+cudaError_t launch_rows8(int grid, cudaStream_t stream, const NarrowPlan &P, const uint16_t *q, const uint8_t *k,
+                         int64_t k_stride, const uint8_t *modality, float *logits, float2 *part, DeviceError *err) {
+  static bool attr = false;
+  if (!attr) {
+    const cudaError_t e = cudaFuncSetAttribute(score_narrow_rows8_kernel<NPAIR>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               static_cast<int>(kStrmSmem));
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  score_narrow_rows8_kernel<NPAIR><<<grid, kStrmThreads, kStrmSmem, stream>>>(P, q, k, k_stride, modality, logits,
+                                                                             part, err);
   return cudaGetLastError();
 }
 
@@ -435,6 +529,14 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
       max_rg = G * nq > max_rg ? G * nq : max_rg;
     }
     const bool rows8 = (hkv == 2 || hkv == 4) && max_rg <= 8;
+    // rows8 chunk: about one CTA per SM over this launch's keys, a multiple of a stage
+    int64_t launch_tokens = 0;
+    for (int i = 0; i < ns; ++i) launch_tokens += seqs->cu_seqlens_h[s0 + i + 1] - seqs->cu_seqlens_h[s0 + i];
+    const int64_t stage_tok = kStrmStageBytes / (static_cast<int64_t>(hkv) * 256);
+    const int64_t sms = device_sm_count();
+    int64_t chunk = (launch_tokens + sms - 1) / sms;
+    chunk = std::max<int64_t>(stage_tok, (chunk + stage_tok - 1) / stage_tok * stage_tok);
+    P.chunk = static_cast<int32_t>(std::min<int64_t>(chunk, 1 << 24));
     int units = 0, units8 = 0, max_rows = 0;
     int64_t rows_all = 0;
     for (int i = 0; i < ns; ++i) {
@@ -452,7 +554,7 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
       sq.part_base = part_base;
       sq.lse_base = lse_base;
       const int ctas = (sq.len + kThreads - 1) / kThreads;
-      const int ctas8 = (sq.len + kRows8Tokens - 1) / kRows8Tokens;
+      const int ctas8 = (sq.len + P.chunk - 1) / P.chunk;   // <= (len + 63) / 64: fits the workspace
       sq.nparts = rows8 ? ctas8 : ctas;
       units += ctas;
       units8 += ctas8;
@@ -469,13 +571,9 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
     const uint16_t *q16 = static_cast<const uint16_t *>(q);
     const uint8_t *k8 = static_cast<const uint8_t *>(k);
     if (rows8) {
-      if (hkv == 4)
-        score_narrow_rows8_kernel<2><<<units8, kThreads, 0, stream>>>(P, q16, k8, k_token_stride, seqs->modality,
-                                                                       logits, part);
-      else
-        score_narrow_rows8_kernel<1><<<units8, kThreads, 0, stream>>>(P, q16, k8, k_token_stride, seqs->modality,
-                                                                       logits, part);
-      e = cudaGetLastError();
+      DeviceError *err = reinterpret_cast<DeviceError *>(wsb + L.err_off);
+      e = hkv == 4 ? launch_rows8<2>(units8, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part, err)
+                   : launch_rows8<1>(units8, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part, err);
     } else {
       const size_t smem = static_cast<size_t>(max_rows) * 128 * sizeof(float) +
                           static_cast<size_t>(kWarps) * max_rows * sizeof(float2);
