@@ -39,3 +39,45 @@ def test_pruning_layer_runs_at_its_entering_length():
 def test_paper_reduction_figure_is_a_ratio_of_its_table_values():
     # Table main7b: 67.9 T at full tokens, 15.0 T for the 25% tier ("up to 78%").
     assert 1 - 15.0 / 67.9 == pytest.approx(0.779, abs=1e-3)
+
+
+def _golden_rows():
+    import os
+    path = os.path.join(os.path.dirname(__file__), "golden", "full_token_prefill_flops.txt")
+    rows = []
+    with open(path) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                name, T, d, m, tf = line.split()
+                rows.append((name, F.Thinker(int(T), int(d), int(m)), float(tf) * 1e12))
+    return rows
+
+
+def _length_for(total, model, phi=F.phi):
+    """n0 with T phi(n0) = total (phi is increasing in n)."""
+    lo, hi = 0.0, 1e6
+    for _ in range(200):
+        mid = 0.5 * (lo + hi)
+        if model.layers * phi(mid, model) < total:
+            lo = mid
+        else:
+            hi = mid
+    return lo
+
+
+def test_both_backbones_full_token_flops_imply_one_input_length():
+    # The 7B and 3B rows of Table main7b cost the same inputs (same encoders and benchmarks), so
+    # inverting Eq. perlayer/prefill must give the same uncompressed length for both: about 9.5k
+    # tokens.  A dropped term or a wrong constant breaks the agreement (checked below).
+    (n7, m7, f7), (n3, m3, f3) = _golden_rows()
+    assert m7 == F.QWEN25_OMNI_7B and m3 == F.QWEN25_OMNI_3B
+    len7, len3 = _length_for(f7, m7), _length_for(f3, m3)
+    assert 9000 < len7 < 10000 and 9000 < len3 < 10000
+    assert len7 / len3 == pytest.approx(1.0, abs=0.015)
+    # dropping the feed-forward or the attention term makes the two models disagree by 12-17 %
+    # (the projection coefficient is pinned by the hand-worked phi(1000) above instead)
+    no_ffn = lambda n, mo: 4 * n * mo.hidden ** 2 + 2 * n * n * mo.hidden
+    no_attn = lambda n, mo: 4 * n * mo.hidden ** 2 + 2 * n * mo.hidden * mo.ffn
+    for slip in (no_ffn, no_attn):
+        r = _length_for(f7, m7, slip) / _length_for(f3, m3, slip)
+        assert abs(r - 1.0) > 0.1
