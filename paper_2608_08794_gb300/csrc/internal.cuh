@@ -72,6 +72,10 @@ apack_status run_select(const apack_seqs *seqs, const float *scores, const int32
                         void *ws, cudaStream_t stream);
 apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes, int32_t num_groups,
                          DeviceError *err, cudaStream_t stream);
+// 3-D TMA map over a K slab [tokens][hkv][128] bf16 (token_stride bytes between tokens):
+// boxes of 64 features x 1 head x box_tokens tokens, 128-byte swizzle.
+bool make_kv_tile_map(CUtensorMap *map, const void *k, int hkv, int64_t tokens, int64_t token_stride,
+                      uint32_t box_tokens);
 apack_status counts_and_offsets(const apack_seqs *s, const float *ratio_h, const int32_t *count_h, int32_t mode,
                                 int32_t *k_out, int32_t *cu_out);
 bool ws_ok(const apack_seqs *s, const void *ws, size_t bytes);

@@ -718,6 +718,12 @@ bool g_attr_done = false;
 
 }  // namespace
 
+bool make_kv_tile_map(CUtensorMap *map, const void *k, int hkv, int64_t tokens, int64_t token_stride,
+                      uint32_t box_tokens) {
+  return make_map(map, k, static_cast<uint64_t>(hkv), static_cast<uint64_t>(tokens), 256,
+                  static_cast<uint64_t>(token_stride), 1, box_tokens);
+}
+
 apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
                        float *scores, void *ws, cudaStream_t stream) {
   int64_t T = 0, NQ = 0;

@@ -2,17 +2,14 @@
 // has few query rows: the paper's own setting scores with the last query token only
 // (Table S-hparams), i.e. G = Hq/Hkv rows per group (7 for the 7B model).
 //
-// With so few rows the step is bound by reading K from HBM, not by arithmetic, so
-// this path uses CUDA cores and reads K once:
-//   logits kernel:  log2-domain logits x * log2(e)/sqrt(D) of every (logit row, key),
-//                   stored per logit row with a row stride padded to 64 keys, and per
-//                   CTA (max, sum of exp2) of every logit row over the multimodal keys of
-//                   its tile.  Two variants:
-//                   * rows8 (Hkv = 2 or 4, at most 8 rows per head group): a warp reads
-//                     token rows coalesced, 16 lanes per KV head with 8 features each,
-//                     holds its query slice in registers, and an 8-row reduce-scatter
-//                     over the 16 lanes leaves one finished logit per lane pair;
-//                   * general: one thread per key reads its whole token row and dots it
+// With so few rows the step is bound by reading K once, so the logits are computed once and
+// kept: three launches.
+//   logits kernel:  log2-domain logits x * log2(e)/sqrt(D) of every (logit row, key), stored per
+//                   logit row with a row stride padded to 64 keys, and per CTA the (max, sum of
+//                   exp2) of every logit row over its multimodal keys.  Two variants:
+//                   * Hkv = 2 or 4 with at most 8 rows per head group: the tcgen05 kernel of
+//                     score_narrow_tc.cu (keys as M = 128, the group's rows as N = 16);
+//                   * other shapes: one thread per key reads its whole token row and dots it
 //                     with the group's query rows held in shared memory;
 //   merge kernel:   per logit row, one block combines the CTA partials into lse2;
 //   final kernel:   one thread per key sums exp2(logit - lse2) over all logit rows
@@ -23,6 +20,7 @@
 #include <cmath>
 
 #include "internal.cuh"
+#include "narrow_plan.cuh"
 #include "ptx.cuh"
 
 namespace apack {
@@ -31,49 +29,8 @@ namespace {
 
 constexpr int kThreads = 256;          // keys per CTA (general logits kernel, final kernel)
 constexpr int kWarps = kThreads / 32;
-constexpr int kRows8Tokens = 64;       // smallest key chunk of the rows8 logits kernel (sizes partials)
-constexpr int kStrmWarps = 16;         // rows8 kernel: warps per CTA (lane 0 of the last also loads)
-constexpr int kStrmThreads = kStrmWarps * 32;
-constexpr int kStrmStages = 3;
-constexpr int kStrmStageBytes = 65536; // K rows per stage: 64 tokens of 4 KV heads, 128 of 2
-constexpr size_t kStrmSmem = static_cast<size_t>(kStrmStages) * kStrmStageBytes + 2 * kStrmStages * sizeof(uint64_t) +
-                             kStrmWarps * 16 * sizeof(float2) + 16;
+constexpr int kRows8Tokens = 64;       // lower bound of the tensor-core kernel's key chunk (sizes partials)
 constexpr int kLogitPad = 64;          // logit row stride: the key count rounded up to this
-
-struct NSeq {
-  int32_t t0, len;
-  int32_t q_off, n_q;
-  int32_t unit_begin;                  // first 256-key CTA of this sequence (general logits, final)
-  int32_t unit8_begin;                 // first chunk (CTA) of this sequence in the rows8 logits kernel
-  int32_t nparts;                      // CTA partials of the logits kernel in use
-  int32_t rows;                        // logit rows R = Hq * n_q
-  int64_t lstride;                     // logit row stride: len rounded up to kLogitPad
-  int64_t logit_base;                  // float offset of this sequence's logits [R][lstride]
-  int64_t part_base;                   // float2 offset of its CTA partials [nparts][R]
-  int64_t lse_base;                    // float offset of its lse2 [R]
-};
-
-struct NarrowPlan {
-  int32_t nseq;
-  int32_t total_units;
-  int32_t total_units8;
-  int32_t chunk;                       // keys per CTA of the rows8 kernel (a multiple of a stage)
-  int32_t hq, hkv, group;
-  float scale2;
-  NSeq seq[kSeqsPerLaunch];
-};
-
-__device__ __forceinline__ int find_unit_seq(const NarrowPlan &p, int u) {
-  int s = 0;
-  while (s + 1 < p.nseq && p.seq[s + 1].unit_begin <= u) ++s;
-  return s;
-}
-
-__device__ __forceinline__ int find_unit8_seq(const NarrowPlan &p, int u) {
-  int s = 0;
-  while (s + 1 < p.nseq && p.seq[s + 1].unit8_begin <= u) ++s;
-  return s;
-}
 
 __device__ __forceinline__ bool is_mm(uint8_t m) { return m == APACK_MOD_AUDIO || m == APACK_MOD_VISUAL; }
 
@@ -178,199 +135,6 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
-// rows8 logits kernel (Hkv = 2 or 4, at most 8 rows per head group): one CTA per chunk
-// of a sequence's keys (about T / #SMs keys).  The chunk's K rows stream into a ring of
-// kStrmStages shared-memory stages by bulk async copies (64 KB per stage: 64 tokens of
-// 4 KV heads or 128 of 2); lane 0 of the last warp issues them and refills a slot once all
-// warps have released it.  Warp w takes head pair w % NPAIR and the group of 8 keys
-// (w / NPAIR) of every stage; lane l works on head 2 hp + (l >> 4) and features
-// [8 (l & 15), 8 (l & 15) + 8), with its query slice in registers.  Per CTA it writes the
-// (max, sum of exp2) of every logit row over its multimodal keys.
-template <int NPAIR>
-__global__ void __launch_bounds__(kStrmThreads, 1)
-    score_narrow_rows8_kernel(const __grid_constant__ NarrowPlan plan, const uint16_t *__restrict__ q,
-                              const uint8_t *__restrict__ k, int64_t k_stride, const uint8_t *__restrict__ modality,
-                              float *__restrict__ logits, float2 *__restrict__ part, DeviceError *err) {
-  extern __shared__ __align__(1024) uint8_t dsm[];
-  uint8_t *stage_base = dsm;
-  uint64_t *full = reinterpret_cast<uint64_t *>(dsm + kStrmStages * kStrmStageBytes);
-  uint64_t *empty = full + kStrmStages;
-  float2 *wst = reinterpret_cast<float2 *>(empty + kStrmStages);          // [warp][16]
-  int *abort_flag = reinterpret_cast<int *>(wst + kStrmWarps * 16);
-  const int c = blockIdx.x;
-  const int s = find_unit8_seq(plan, c);
-  const NSeq &sq = plan.seq[s];
-  const int G = plan.group;
-  const int rg = G * sq.n_q;
-  if (rg == 0) return;                                   // no query row: nothing to score (CTA-uniform)
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t row = static_cast<int64_t>(plan.hkv) * 256;
-  const int stage_tok = kStrmStageBytes / static_cast<int>(row);
-  const int tb = (c - sq.unit8_begin) * plan.chunk;
-  const int te = min(sq.len, tb + plan.chunk);
-  const int nst = (te - tb + stage_tok - 1) / stage_tok;
-  const bool loader = warp == kStrmWarps - 1 && lane == 0;
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < kStrmStages; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&empty[i], kStrmWarps);
-    }
-    *abort_flag = 0;
-    fence_mbar_init();
-  }
-  __syncthreads();
-  volatile int *abort_v = abort_flag;
-  const uint8_t *kseq = k + static_cast<int64_t>(sq.t0) * k_stride;
-  auto issue = [&](int n) {
-    const int slot = n % kStrmStages;
-    const int t = tb + n * stage_tok;
-    const int cnt = min(stage_tok, te - t);
-    uint8_t *dst = stage_base + static_cast<size_t>(slot) * kStrmStageBytes;
-    mbar_arrive_expect_tx(&full[slot], static_cast<uint32_t>(cnt * row));
-    if (k_stride == row) {
-      bulk_load(dst, kseq + static_cast<int64_t>(t) * k_stride, static_cast<uint32_t>(cnt * row), &full[slot]);
-    } else {
-      for (int r = 0; r < cnt; ++r)
-        bulk_load(dst + r * row, kseq + static_cast<int64_t>(t + r) * k_stride, static_cast<uint32_t>(row),
-                  &full[slot]);
-    }
-  };
-  int issued = 0;
-  if (loader)
-    for (; issued < kStrmStages && issued < nst; ++issued) issue(issued);
-
-  const int hp = warp % NPAIR, grp = warp / NPAIR;
-  const int h = 2 * hp + (lane >> 4), part16 = lane & 15;
-  // query slice: rows j < rg of head group h (logit row (j / G) Hq + h G + j % G)
-  float qf[8][8];
-  const uint4 *qrow = reinterpret_cast<const uint4 *>(q + static_cast<int64_t>(sq.q_off) * plan.hq * 128);
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    uint4 w = make_uint4(0, 0, 0, 0);
-    if (j < rg) w = __ldg(qrow + ((j / G) * plan.hq + h * G + j % G) * 16 + part16);
-    bf16x8_to_f32(w, qf[j]);
-  }
-  const int r = (lane >> 1) & 7;                       // row this lane holds after the reduce-scatter
-  const bool row_ok = r < rg;
-  const int rho = row_ok ? (r / G) * plan.hq + h * G + r % G : 0;
-  const bool b1 = lane & 8, b2 = lane & 4, b3 = lane & 2;
-  float m = -INFINITY, ssum = 0.f;
-  for (int n = 0; n < nst; ++n) {
-    const int slot = n % kStrmStages;
-    if (!__all_sync(0xffffffffu, mbar_wait(&full[slot], (n / kStrmStages) & 1u, kWaitLimitNs))) {
-      if (lane == 0) {
-        raise_device_error(err, APACK_ETIMEOUT, 71, c, n);
-        *abort_v = 1;
-      }
-      break;
-    }
-    const int t0 = tb + n * stage_tok + grp * 8;
-    const int valid = min(8, te - t0);
-    if (valid > 0) {
-      const uint8_t *ks = stage_base + static_cast<size_t>(slot) * kStrmStageBytes +
-                          static_cast<size_t>(grp) * 8 * row + h * 256 + part16 * 16;
-      const int tl = t0 + (lane & 7);
-      const unsigned mmask = __ballot_sync(0xffffffffu, lane < 8 && tl < te && is_mm(modality[sq.t0 + tl]));
-      float outv[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        float kf[8];
-        bf16x8_to_f32(i < valid ? *reinterpret_cast<const uint4 *>(ks + i * row) : make_uint4(0, 0, 0, 0), kf);
-        float acc[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          float2 a2 = make_float2(0.f, 0.f);
-#pragma unroll
-          for (int e = 0; e < 4; ++e)
-            a2 = ffma2(make_float2(kf[2 * e], kf[2 * e + 1]), make_float2(qf[j][2 * e], qf[j][2 * e + 1]), a2);
-          acc[j] = a2.x + a2.y;
-        }
-        // reduce-scatter over the 16 lanes of the head: lane bits 3, 2, 1 pick the row
-        float v4[4], v2[2];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float send = b1 ? acc[e] : acc[e + 4];
-          const float keep = b1 ? acc[e + 4] : acc[e];
-          v4[e] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
-        }
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const float send = b2 ? v4[e] : v4[e + 2];
-          const float keep = b2 ? v4[e + 2] : v4[e];
-          v2[e] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
-        }
-        float v1;
-        {
-          const float send = b3 ? v2[0] : v2[1];
-          const float keep = b3 ? v2[1] : v2[0];
-          v1 = keep + __shfl_xor_sync(0xffffffffu, send, 2);
-        }
-        v1 += __shfl_xor_sync(0xffffffffu, v1, 1);
-        outv[i] = v1 * plan.scale2;
-      }
-      // running (max, sum of exp2) of this lane's row over the group's multimodal keys
-      float cm = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-        if ((mmask >> i) & 1u) cm = fmaxf(cm, outv[i]);
-      if (cm != -INFINITY) {
-        if (cm > m) {
-          ssum *= ex2_approx(m - cm);
-          m = cm;
-        }
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          if ((mmask >> i) & 1u) ssum += ex2_approx(outv[i] - m);
-      }
-      if (row_ok) {   // the lane pair writes the group's 8 logits of its row: 4 each
-        const bool odd = lane & 1;
-        const float4 w = odd ? make_float4(outv[4], outv[5], outv[6], outv[7])
-                             : make_float4(outv[0], outv[1], outv[2], outv[3]);
-        *reinterpret_cast<float4 *>(logits + sq.logit_base + static_cast<int64_t>(rho) * sq.lstride + t0 +
-                                    (odd ? 4 : 0)) = w;
-      }
-    }
-    __syncwarp();                        // this warp is done with the stage
-    if (lane == 0) mbar_arrive(&empty[slot]);
-    if (loader && issued < nst) {
-      // every warp has released stage n: refill its slot
-      if (!mbar_wait(&empty[slot], (n / kStrmStages) & 1u, kWaitLimitNs)) {
-        raise_device_error(err, APACK_ETIMEOUT, 72, c, n);
-        *abort_v = 1;
-      } else {
-        issue(issued);
-        ++issued;
-      }
-    }
-    __syncwarp();
-    if (*abort_v) break;
-  }
-  // after an abort, stages may still be in flight: wait for them (bounded) before exit
-  if (loader && *abort_v)
-    for (int n = max(0, issued - kStrmStages); n < issued; ++n)
-      mbar_wait(&full[n % kStrmStages], (n / kStrmStages) & 1u, kWaitLimitNs / 4);
-  if ((lane & 1) == 0) wst[warp * 16 + (lane >> 1)] = make_float2(m, ssum);
-  __syncthreads();
-  if (*abort_v) return;
-  // per (head, row): combine the warps of its head pair in key order
-  if (threadIdx.x < 16 * NPAIR) {
-    const int php = threadIdx.x >> 4, slot = threadIdx.x & 15;
-    const int rr = slot & 7, hh = 2 * php + (slot >> 3);
-    if (rr < rg) {
-      float mx = -INFINITY;
-      for (int g2 = 0; g2 < kStrmWarps / NPAIR; ++g2) mx = fmaxf(mx, wst[(g2 * NPAIR + php) * 16 + slot].x);
-      float sum = 0.f;
-      if (mx != -INFINITY)
-        for (int g2 = 0; g2 < kStrmWarps / NPAIR; ++g2) {
-          const float2 v = wst[(g2 * NPAIR + php) * 16 + slot];
-          if (v.x != -INFINITY) sum += v.y * ex2_approx(v.x - mx);
-        }
-      const int rh = (rr / G) * plan.hq + hh * G + rr % G;
-      part[sq.part_base + static_cast<int64_t>(c - sq.unit8_begin) * sq.rows + rh] = make_float2(mx, sum);
-    }
-  }
-}
-
 // One block per (sequence, logit row): lse2 over the CTA partials.  Each thread
 // folds a fixed stride of partials, then a fixed-shape tree combines the
 // threads: the order never depends on timing, so lse2 is deterministic.
@@ -463,22 +227,6 @@ cudaError_t launch_logits(int grid, size_t smem, cudaStream_t stream, const Narr
   return cudaGetLastError();
 }
 
-template <int NPAIR>
-cudaError_t launch_rows8(int grid, cudaStream_t stream, const NarrowPlan &P, const uint16_t *q, const uint8_t *k,
-                         int64_t k_stride, const uint8_t *modality, float *logits, float2 *part, DeviceError *err) {
-  static bool attr = false;
-  if (!attr) {
-    const cudaError_t e = cudaFuncSetAttribute(score_narrow_rows8_kernel<NPAIR>,
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               static_cast<int>(kStrmSmem));
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
-  score_narrow_rows8_kernel<NPAIR><<<grid, kStrmThreads, kStrmSmem, stream>>>(P, q, k, k_stride, modality, logits,
-                                                                             part, err);
-  return cudaGetLastError();
-}
-
 }  // namespace
 
 bool narrow_score_applies(const apack_seqs *s) {
@@ -522,17 +270,17 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
     P.hkv = hkv;
     P.group = G;
     P.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(APACK_HEAD_DIM)));
-    // rows8 kernel: K read by whole warps, query slice in registers
+    // tensor-core logits kernel: Hkv = 2 or 4, at most 8 rows per head group
     int max_rg = 0;
     for (int i = 0; i < ns; ++i) {
       const int nq = seqs->cu_qlens_h[s0 + i + 1] - seqs->cu_qlens_h[s0 + i];
       max_rg = G * nq > max_rg ? G * nq : max_rg;
     }
     const bool rows8 = (hkv == 2 || hkv == 4) && max_rg <= 8;
-    // rows8 chunk: about one CTA per SM over this launch's keys, a multiple of a stage
+    // its chunk: about one CTA per SM over this launch's keys, whole 128-key tiles
     int64_t launch_tokens = 0;
     for (int i = 0; i < ns; ++i) launch_tokens += seqs->cu_seqlens_h[s0 + i + 1] - seqs->cu_seqlens_h[s0 + i];
-    const int64_t stage_tok = kStrmStageBytes / (static_cast<int64_t>(hkv) * 256);
+    const int64_t stage_tok = 128;     // chunks are whole 128-key tensor-core tiles
     const int64_t sms = device_sm_count();
     int64_t chunk = (launch_tokens + sms - 1) / sms;
     chunk = std::max<int64_t>(stage_tok, (chunk + stage_tok - 1) / stage_tok * stage_tok);
@@ -572,8 +320,9 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
     const uint8_t *k8 = static_cast<const uint8_t *>(k);
     if (rows8) {
       DeviceError *err = reinterpret_cast<DeviceError *>(wsb + L.err_off);
-      e = hkv == 4 ? launch_rows8<2>(units8, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part, err)
-                   : launch_rows8<1>(units8, stream, P, q16, k8, k_token_stride, seqs->modality, logits, part, err);
+      CUtensorMap kmap;
+      if (!make_kv_tile_map(&kmap, k, hkv, seqs->cu_seqlens_h[B], k_token_stride, 128)) return APACK_ECUDA;
+      e = launch_narrow_tc(units8, stream, kmap, P, q16, seqs->modality, logits, part, err);
     } else {
       const size_t smem = static_cast<size_t>(max_rows) * 128 * sizeof(float) +
                           static_cast<size_t>(kWarps) * max_rows * sizeof(float2);
