@@ -56,6 +56,7 @@ CASES = [
     (37, 16, 462, 256, 3),
     (20, 100, 250, 3584, 7),
     (9, 2, 9, 128, 1),
+    (6, 3, 6, 4104, 3),       # rows wider than one CTA: separate pooling and CKA launches
 ]
 
 
