@@ -562,9 +562,14 @@ def main():
                 stage_ms[i, st] += e[st].elapsed_time(e[st + 1])
     stage_ms /= args.steps
 
-    # end to end through the C ABI with host buffers: H2D of the step's inputs
-    # from pinned memory, the three prune steps, D2H of the result
+    # end to end through the C ABI with host buffers: every iteration copies its inputs from
+    # pinned host memory, runs the schedule and reads the result back.  Two device buffer sets
+    # let iteration i+1's upload (copy stream) run while iteration i computes and while
+    # iteration i-1's result is read back (third stream): the link carries both directions.
     e2e_steps = args.e2e_steps or max(3, min(args.steps, 20))
+    pp2 = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                           wl.prune_layers, counts, select_mode=mode)
+    sets = [pp, pp2]
     h_k = torch.empty(pp.k_in.shape, dtype=pp.k_in.dtype, pin_memory=True)
     h_v = torch.empty_like(h_k, pin_memory=True)
     h_h = torch.empty(pp.hidden_in.shape, dtype=pp.hidden_in.dtype, pin_memory=True)
@@ -574,40 +579,67 @@ def main():
     for a, b in zip(h_q, pp.q):
         a.copy_(b)
     last = nsteps - 1
-    ko, vo = pp.output_kv(last)
-    ho = pp.output_hidden(last)
-    o_k = torch.empty(ko.shape, dtype=ko.dtype, pin_memory=True)
-    o_v = torch.empty_like(o_k, pin_memory=True)
-    o_h = torch.empty(ho.shape, dtype=ho.dtype, pin_memory=True)
-    o_i = [torch.empty(int(t), dtype=torch.int32, pin_memory=True) for t in pp.t_out]
+
+    def host_outputs(p):
+        ko, vo = p.output_kv(last)
+        ho = p.output_hidden(last)
+        return ([torch.empty(ko.shape, dtype=ko.dtype, pin_memory=True),
+                 torch.empty(vo.shape, dtype=vo.dtype, pin_memory=True),
+                 torch.empty(ho.shape, dtype=ho.dtype, pin_memory=True)] +
+                [torch.empty(int(t), dtype=torch.int32, pin_memory=True) for t in p.t_out])
+
+    h_out = [host_outputs(p) for p in sets]
     h2d = sum(x.numel() * x.element_size() for x in [h_k, h_v, h_h, h_m] + h_q)
-    d2h = sum(x.numel() * x.element_size() for x in [o_k, o_v, o_h] + o_i)
+    d2h = sum(x.numel() * x.element_size() for x in h_out[0])
+    s_up, s_down = torch.cuda.Stream(), torch.cuda.Stream()
+    ev_up = [torch.cuda.Event() for _ in sets]
+    ev_comp = [torch.cuda.Event() for _ in sets]
+    ev_down = [torch.cuda.Event() for _ in sets]
+    for e in ev_down:
+        e.record(stream)
 
-    def e2e_step():
-        pp.k_in.copy_(h_k, non_blocking=True); pp.v_in.copy_(h_v, non_blocking=True)
-        pp.hidden_in.copy_(h_h, non_blocking=True); pp.modality_in.copy_(h_m, non_blocking=True)
-        for a, b in zip(pp.q, h_q):
-            a.copy_(b, non_blocking=True)
-        run_schedule()
-        o_k.copy_(ko, non_blocking=True); o_v.copy_(vo, non_blocking=True); o_h.copy_(ho, non_blocking=True)
-        for i, t in enumerate(pp.t_out):
-            o_i[i].copy_(pp.keep_idx[i][:t], non_blocking=True)
+    def e2e_iteration(j):
+        b = j % 2
+        p = sets[b]
+        with torch.cuda.stream(s_up):          # upload once the set's last result was read back
+            s_up.wait_event(ev_down[b])
+            p.k_in.copy_(h_k, non_blocking=True); p.v_in.copy_(h_v, non_blocking=True)
+            p.hidden_in.copy_(h_h, non_blocking=True); p.modality_in.copy_(h_m, non_blocking=True)
+            for a, qh in zip(p.q, h_q):
+                a.copy_(qh, non_blocking=True)
+            ev_up[b].record(s_up)
+        stream.wait_event(ev_up[b])
+        p.run(stream=stream)
+        ev_comp[b].record(stream)
+        with torch.cuda.stream(s_down):
+            s_down.wait_event(ev_comp[b])
+            ko, vo = p.output_kv(last)
+            o = h_out[b]
+            o[0].copy_(ko, non_blocking=True); o[1].copy_(vo, non_blocking=True)
+            o[2].copy_(p.output_hidden(last), non_blocking=True)
+            for i, t in enumerate(p.t_out):
+                o[3 + i].copy_(p.keep_idx[i][:t], non_blocking=True)
+            ev_down[b].record(s_down)
 
-    e2e_step()
+    for j in range(2):
+        e2e_iteration(j)
     torch.cuda.synchronize()
     barrier()
     if clocks:
         clocks.mark(True)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(e2e_steps):
-        e2e_step()
+    s_up.wait_stream(stream)
+    for j in range(e2e_steps):
+        e2e_iteration(j)
+    stream.wait_stream(s_down)
     e1.record(stream)
     barrier()
     if clocks:
         clocks.mark(False)
         clocks.stop()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dist, "cuda")
+    del pp2, sets
 
     # the pre-LLM stage of the same clip, timed on its own after the prune steps
     prellm = prellm_measure(ap, wl, args.steps, args.warmup, stream, dist)
@@ -646,7 +678,9 @@ def main():
             "stages_ms_per_iter": {"score": float(score_ms), "select": float(select_ms),
                                    "compact": float(comp_ms.sum())},
             "e2e": {"value": whole_job_value(mm_per_iter, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
-                    "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps},
+                    "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps,
+                    "pipeline": "two device buffer sets: the next iteration's upload and the previous one's read-back "
+                                "run on copy streams while the current iteration computes"},
             "clocks": clocks.summary() if clocks else None,
             "context": schedule_context(wl, pp),
         }
