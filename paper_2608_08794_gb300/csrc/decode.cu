@@ -23,6 +23,7 @@
 #include <algorithm>
 #include <cmath>
 
+#include "decode_plan.cuh"
 #include "internal.cuh"
 #include "ptx.cuh"
 
@@ -39,24 +40,6 @@ constexpr size_t kDecSmem = static_cast<size_t>(kDecStages) * 2 * kStageBytes + 
                             (kDecConsumers * 8 * kDecRows + kDecConsumers * kDecRows) * sizeof(float) + 16;
 constexpr int kDecCombineThreads = 512;
 constexpr int kDecCombineWarps = kDecCombineThreads / 32;
-
-struct DecSeq {
-  int32_t t0, len;
-  int32_t chunk_begin, nchunks;
-};
-
-struct DecPlan {
-  int32_t nseq, hq, hkv, group, chunk;   // chunk: keys per CTA, a multiple of 64
-  int32_t total_chunks;
-  float scale2;                          // log2(e) / sqrt(128)
-  DecSeq seq[kSeqsPerLaunch];
-};
-
-__device__ __forceinline__ int find_chunk_seq(const DecPlan &p, int c) {
-  int s = 0;
-  while (s + 1 < p.nseq && p.seq[s + 1].chunk_begin <= c) ++s;
-  return s;
-}
 
 __device__ __forceinline__ void bf16x4_to_f32(const uint2 &w, float (&f)[4]) {
   f[0] = __uint_as_float(w.x << 16);
@@ -341,13 +324,17 @@ __global__ void __launch_bounds__(kDecCombineThreads)
   }
 }
 
-// Keys per chunk: about one CTA per SM over the whole batch, a multiple of a stage.
+// The tensor-core chunk kernel takes Hkv = 2 or 4 with at most 8 query heads per KV head.
+bool decode_tc_applies(int32_t hq, int32_t hkv) { return (hkv == 2 || hkv == 4) && hq / hkv <= kDecRows; }
+
+// Keys per chunk: about one CTA per SM over the whole batch, whole 128-key tiles (a multiple of
+// every stage size of both chunk kernels).
 int decode_chunk_keys(int64_t total_tokens, int32_t hkv) {
-  const int64_t stage_tok = kStageBytes / (static_cast<int64_t>(hkv) * 256);
+  (void)hkv;
   const int64_t ctas = device_sm_count();
   int64_t c = (total_tokens + ctas - 1) / std::max<int64_t>(1, ctas);
-  c = (c + stage_tok - 1) / stage_tok * stage_tok;
-  return static_cast<int>(std::min<int64_t>(std::max<int64_t>(c, stage_tok), 1 << 20));
+  c = (c + 127) / 128 * 128;
+  return static_cast<int>(std::min<int64_t>(std::max<int64_t>(c, 128), 1 << 20));
 }
 
 apack_status decode_validate(int32_t num_seqs, const int32_t *cu_seqlens_h, int32_t hq, int32_t hkv,
@@ -419,6 +406,11 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const uint16_t *q16 = static_cast<const uint16_t *>(q);
+  const bool tc = decode_tc_applies(num_q_heads, num_kv_heads) && total > 0;
+  CUtensorMap kmap, vmap;
+  if (tc && (!make_kv_tile_map(&kmap, k, num_kv_heads, total, kv_token_stride, 128) ||
+             !make_kv_tile_map(&vmap, v, num_kv_heads, total, kv_token_stride, 128)))
+    return APACK_ECUDA;
   int64_t chunk_base = 0;
   for (int s0 = 0; s0 < num_seqs; s0 += kSeqsPerLaunch) {
     const int ns = std::min(num_seqs - s0, kSeqsPerLaunch);
@@ -427,7 +419,7 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
     P.hq = num_q_heads;
     P.hkv = num_kv_heads;
     P.group = num_q_heads / num_kv_heads;
-    P.chunk = chunk;                    // a multiple of the stage size
+    P.chunk = chunk;                    // whole 128-key tiles
     P.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(APACK_HEAD_DIM)));
     int chunks = 0;
     for (int i = 0; i < ns; ++i) {
@@ -443,11 +435,15 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
     float2 *mp = mlpart + chunk_base * num_q_heads;
     const uint16_t *qs = q16 + static_cast<int64_t>(s0) * num_q_heads * 128;
     if (chunks > 0) {
-      decode_chunk_kernel<<<chunks, kDecThreads, kDecSmem, s>>>(P, qs, static_cast<const uint8_t *>(k),
-                                                                static_cast<const uint8_t *>(v), kv_token_stride,
-                                                                op, mp, err);
+      if (tc) {
+        if (check_cuda(launch_decode_tc(chunks, s, kmap, vmap, P, qs, op, mp, err)) != APACK_OK) return APACK_ECUDA;
+      } else {
+        decode_chunk_kernel<<<chunks, kDecThreads, kDecSmem, s>>>(P, qs, static_cast<const uint8_t *>(k),
+                                                                  static_cast<const uint8_t *>(v), kv_token_stride,
+                                                                  op, mp, err);
+        if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+      }
       count_launches(1);
-      if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
     decode_combine_kernel<<<ns * num_q_heads, kDecCombineThreads, 0, s>>>(
         P, op, mp, out + static_cast<int64_t>(s0) * num_q_heads * 128);

@@ -1,0 +1,457 @@
+// decode_tc.cu -- decode-step attention over a (compacted) KV cache on the tensor cores
+// (Sec. 3.2, last sentence; App. G: the cost pruning shortens at every decode step).
+//
+//   out[b, h] = sum_j softmax_j(q[b, h] . k[j, g(h)] / sqrt(128)) v[j, g(h)]
+//
+// One CTA per chunk of a sequence's keys (whole 128-key tiles), all KV heads.  A stage is one
+// KV head of one tile; its K rows and its V rows (TMA boxes of 64 features x 1 head x 128 keys,
+// 128-byte swizzle, 32 KB each) are separate items of a 6-slot shared-memory ring, loaded in
+// the order K0 K1 V0 K2 V1 K3 V2 ...: the keys of a stage arrive one stage ahead of its values,
+// so its logits and probabilities are ready when V lands, and each item holds its slot only
+// until its own contraction is done (K: S, V: O^T).
+//   warp 0, one lane:  TMA loads of the items
+//   warp 1, one lane:  TMEM allocation; S = K q^T of every stage: keys as M = 128, the head
+//                      group's <= 8 query rows (zero-padded) as N = 16; S[key][row] in TMEM
+//   warp 6, one lane:  O^T += V^T P^T of every stage: features as M = 128 (V read as an MN-major
+//                      operand straight from the stage), keys as K, N = 16 columns: the 8 rows'
+//                      p split into a bf16 high part (columns 0..7) and the bf16 rounding of the
+//                      remainder (8..15); O^T of each KV head stays in TMEM for the whole chunk.
+//                      Two issuing warps, so that no stage's O^T waits for the next stage's data.
+//   warps 2..5:        softmax, one key per thread (one TMEM lane): scaled logits, p = exp2(s - m)
+//                      against a per-(head, row) reference maximum m that is only raised when a
+//                      tile's logits exceed it by more than 2^8 (then O^T's columns of that row
+//                      and the partial sums are rescaled once), p written as the bf16 pair into
+//                      the head's P tile; at the end they read O^T back (one feature per thread).
+// The result per query head is the chunk partial (m, l = sum p, o = sum p v) in log2 units,
+// merged by the combine kernel with the CUDA-core kernel's partials' rules.  hi + lo carries p
+// to about 2^-17 relative, so o matches fp32 arithmetic.  Every wait is bounded.
+#include <cmath>
+
+#include <cuda_bf16.h>
+
+#include "decode_plan.cuh"
+#include "internal.cuh"
+#include "ptx.cuh"
+
+namespace apack {
+namespace {
+
+constexpr int kDM = 128;                           // keys per tile (MMA M of S, K of O^T)
+constexpr int kDN = 16;                            // MMA N: query rows (S), hi/lo rows (O^T)
+constexpr int kDRows = 8;                          // rows handled (G <= 8)
+constexpr int kDSlots = 6;
+constexpr int kDHalf = kDM * 128;                  // 64 features x 128 keys x 2 B = 16 KB
+constexpr int kDSlotBytes = 2 * kDHalf;            // K or V of one stage, two feature halves: 32 KB
+constexpr int kDQHalf = kDN * 128;                 // 16 rows x 64 features x 2 B = 2 KB
+constexpr int kDPBytes = 2 * kDN * 128;            // P^T of one head: 16 rows x 128 keys x 2 B = 4 KB
+constexpr int kDSoftWarps = 4;
+constexpr int kDPvWarp = 2 + kDSoftWarps;
+constexpr int kDThreads = 32 * (3 + kDSoftWarps);
+constexpr float kDLazy = 8.f;                      // the reference maximum lags by at most 2^8
+constexpr uint32_t kDIdescS = idesc_bf16_f32(kDM, kDN);
+constexpr uint32_t kDIdescO = idesc_bf16_f32(128, kDN) | (1u << 15);   // A (V^T) MN-major
+constexpr uint32_t kDTmemCols = 128;               // S [2][16] at 0, O^T of head h at 32 + 16 h
+
+struct __align__(8) DBars {
+  uint64_t full[kDSlots], empty[kDSlots], s_full[2], s_empty[2], drain[2];   // drain: per issuing warp
+  uint64_t p_full[4], p_empty[4];                  // one pair per KV head: their phases are its tiles
+  uint32_t tmem_base;
+  volatile int32_t abort;
+};
+
+template <int HKV>
+struct DLay {
+  static constexpr uint32_t kOffQ = kDSlots * kDSlotBytes;                      // 1024-aligned
+  static constexpr uint32_t kOffP = kOffQ + HKV * 2 * kDQHalf;                   // [HKV] P^T tiles, 1024-aligned
+  static constexpr uint32_t kOffT = kOffP + HKV * kDPBytes;                      // tile maxima [2][4][8]
+  static constexpr uint32_t kOffM = kOffT + 2 * kDSoftWarps * kDRows * 4;        // reference max [2][HKV][8]
+  static constexpr uint32_t kOffBars = (kOffM + 2 * HKV * kDRows * 4 + 7) & ~7u;
+  static constexpr uint32_t kBytes = kOffBars + 256;
+};
+
+__device__ __forceinline__ bool d_wait(uint64_t *bar, uint32_t parity, DBars *bars, DeviceError *err, int where) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (bars->abort) return false;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      bars->abort = 1;
+      raise_device_error(err, APACK_ETIMEOUT, where);
+      return false;
+    }
+  }
+}
+
+// Named barrier over `count` threads that also ORs a predicate across them.
+__device__ __forceinline__ bool bar_red_or(uint32_t id, uint32_t count, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(v)), "r"(id), "r"(count)
+      : "memory");
+  return r != 0;
+}
+
+// byte offset of element (row, key) in a 16-row x 128-key bf16 K-major tile, 128-byte swizzle
+__device__ __forceinline__ uint32_t p_off(int row, int key) {
+  const int half = key >> 6, ch = (key & 63) >> 3;
+  return half * 2048 + (row >> 3) * 1024 + (row & 7) * 128 + ((ch ^ (row & 7)) << 4) + (key & 7) * 2;
+}
+
+// Load order of the ring's items: K0, K1, V0, K2, V1, ..., K(N-1), V(N-2), V(N-1) for N stages.
+__device__ __forceinline__ int item_of_k(int n) { return n == 0 ? 0 : 2 * n - 1; }
+__device__ __forceinline__ int item_of_v(int n, int N) { return n == N - 1 ? 2 * N - 1 : 2 * n + 2; }
+__device__ __forceinline__ void item_stage(int i, int N, bool *is_v, int *n) {
+  if (i == 0) { *is_v = false; *n = 0; }
+  else if (i == 2 * N - 1) { *is_v = true; *n = N - 1; }
+  else if (i & 1) { *is_v = false; *n = (i + 1) >> 1; }
+  else { *is_v = true; *n = (i >> 1) - 1; }
+}
+
+template <int HKV>
+__global__ void __launch_bounds__(kDThreads, 1)
+    decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                     const __grid_constant__ DecPlan plan, const uint16_t *__restrict__ q, float *__restrict__ opart,
+                     float2 *__restrict__ mlpart, DeviceError *err) {
+  using Lay = DLay<HKV>;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  if ((smem_u32(smem) & 1023u) != 0) {
+    if (threadIdx.x == 0) raise_device_error(err, APACK_EDEVICE, 90);
+    return;
+  }
+  uint8_t *ring = smem;
+  uint8_t *qs = smem + Lay::kOffQ;
+  uint8_t *ps = smem + Lay::kOffP;
+  float *tmax = reinterpret_cast<float *>(smem + Lay::kOffT);
+  float *msm = reinterpret_cast<float *>(smem + Lay::kOffM);
+  DBars *bars = reinterpret_cast<DBars *>(smem + Lay::kOffBars);
+  const int c = blockIdx.x;
+  const int s = find_chunk_seq(plan, c);
+  const DecSeq &sq = plan.seq[s];
+  const int G = plan.group;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tb = (c - sq.chunk_begin) * plan.chunk;
+  const int te = min(sq.len, tb + plan.chunk);
+  const int ntiles = (te - tb + kDM - 1) / kDM;
+  const int nstage = ntiles * HKV;
+
+  // query tiles: rows j < G of head group h, 128-byte swizzled K-major layout
+  for (int idx = threadIdx.x; idx < HKV * kDN * 16; idx += kDThreads) {
+    const int h = idx / (kDN * 16), rem = idx % (kDN * 16);
+    const int row = rem / 16, ch = rem % 16;
+    const int half = ch >> 3, cc = ch & 7;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (row < G)
+      v = __ldg(reinterpret_cast<const uint4 *>(q + (static_cast<int64_t>(s) * plan.hq + h * G + row) * 128) + ch);
+    *reinterpret_cast<uint4 *>(qs + h * 2 * kDQHalf + half * kDQHalf + (row >> 3) * 1024 + (row & 7) * 128 +
+                               ((cc ^ (row & 7)) << 4)) = v;
+  }
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kDSlots; ++i) {
+      mbar_init(&bars->full[i], 1);
+      mbar_init(&bars->empty[i], 1);                // the commit after the item's MMAs
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars->s_full[i], 1);
+      mbar_init(&bars->s_empty[i], kDSoftWarps);
+    }
+    for (int h = 0; h < HKV; ++h) {
+      mbar_init(&bars->p_full[h], kDSoftWarps);
+      mbar_init(&bars->p_empty[h], 1);
+    }
+    mbar_init(&bars->drain[0], 1);
+    mbar_init(&bars->drain[1], 1);
+    bars->abort = 0;
+    for (int i = 0; i < 2 * HKV * kDRows; ++i) msm[i] = -INFINITY;
+    fence_mbar_init();
+  }
+  fence_proxy_async_smem();
+  if (warp == 1) {
+    tmem_alloc(&bars->tmem_base, kDTmemCols);
+    tc_fence_before();
+  }
+  __syncthreads();
+  tc_fence_after();
+
+  float l_run[HKV][kDRows];                        // softmax threads: partial sums of their keys
+#pragma unroll
+  for (int h = 0; h < HKV; ++h)
+#pragma unroll
+    for (int j = 0; j < kDRows; ++j) l_run[h][j] = 0.f;
+  bool stop = false;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&kmap);
+      tma_prefetch_desc(&vmap);
+      bool pend[kDSlots] = {};
+      uint32_t pend_par[kDSlots] = {};
+      for (int i = 0; i < 2 * nstage; ++i) {
+        const int slot = i % kDSlots;
+        if (i >= kDSlots && !d_wait(&bars->empty[slot], ((i / kDSlots) - 1) & 1u, bars, err, 91)) break;
+        bool is_v;
+        int n;
+        item_stage(i, nstage, &is_v, &n);
+        const int t = n / HKV, h = n % HKV;
+        uint8_t *dst = ring + slot * kDSlotBytes;
+        const CUtensorMap *map = is_v ? &vmap : &kmap;
+        mbar_arrive_expect_tx(&bars->full[slot], kDSlotBytes);
+        const int key0 = sq.t0 + tb + t * kDM;
+        tma_load_3d(dst, map, &bars->full[slot], 0, h, key0);
+        tma_load_3d(dst + kDHalf, map, &bars->full[slot], 64, h, key0);
+        pend[slot] = true;
+        pend_par[slot] = (i / kDSlots) & 1u;
+      }
+      if (bars->abort)
+        for (int i = 0; i < kDSlots; ++i)
+          if (pend[i]) mbar_wait(&bars->full[i], pend_par[i], kWaitLimitNs / 4);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ S issuer
+    if (lane == 0) {
+      const uint32_t tmem = bars->tmem_base;
+      const uint32_t q_base = smem_u32(qs);
+      for (int n = 0; n < nstage; ++n) {
+        const int item = item_of_k(n), slot = item % kDSlots, buf = n & 1, h = n % HKV;
+        if (n >= 2 && !d_wait(&bars->s_empty[buf], ((n >> 1) - 1) & 1u, bars, err, 92)) break;
+        if (!d_wait(&bars->full[slot], (item / kDSlots) & 1u, bars, err, 93)) break;
+        tc_fence_after();
+        // K (two 64-feature halves) against the head group's query rows, 16 features per MMA
+        const uint32_t a_base = smem_u32(ring + slot * kDSlotBytes);
+        const uint32_t b_base = q_base + h * 2 * kDQHalf;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t ao = (kk >> 2) * kDHalf + (kk & 3) * 32;
+          const uint32_t bo = (kk >> 2) * kDQHalf + (kk & 3) * 32;
+          tc_mma_bf16(tmem + buf * kDN, smem_desc_sw128(a_base + ao), smem_desc_sw128(b_base + bo), kDIdescS,
+                      kk > 0 ? 1u : 0u);
+        }
+        tc_commit(&bars->s_full[buf]);
+        if (item + kDSlots < 2 * nstage) tc_commit(&bars->empty[slot]);   // K is free once S is done
+      }
+      tc_commit(&bars->drain[0]);                   // every MMA of this thread done before teardown
+      mbar_wait(&bars->drain[0], 0, kWaitLimitNs / 4);
+    }
+  } else if (warp == kDPvWarp) {
+    // ------------------------------------------------------------ O^T issuer
+    if (lane == 0) {
+      const uint32_t tmem = bars->tmem_base;
+      const uint32_t p_base = smem_u32(ps);
+      for (int n = 0; n < nstage; ++n) {
+        const int item = item_of_v(n, nstage), slot = item % kDSlots, t = n / HKV, h = n % HKV;
+        if (!d_wait(&bars->p_full[h], t & 1u, bars, err, 94)) break;
+        if (!d_wait(&bars->full[slot], (item / kDSlots) & 1u, bars, err, 98)) break;
+        tc_fence_after();
+        // O^T[feature][col] += sum_key V[key][feature] P^T[col][key]: 16 keys per MMA
+        const uint32_t v_base = smem_u32(ring + slot * kDSlotBytes);
+        const uint32_t b_base = p_base + h * kDPBytes;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t bo = (kk >> 2) * (kDPBytes / 2) + (kk & 3) * 32;
+          tc_mma_bf16(tmem + 32 + h * kDN, smem_desc_sw128_mn(v_base + kk * 2048, kDHalf, 1024),
+                      smem_desc_sw128(b_base + bo), kDIdescO, (t > 0 || kk > 0) ? 1u : 0u);
+        }
+        tc_commit(&bars->p_empty[h]);
+        if (item + kDSlots < 2 * nstage) tc_commit(&bars->empty[slot]);   // only slots that are reloaded
+      }
+      tc_commit(&bars->drain[1]);
+      mbar_wait(&bars->drain[1], 0, kWaitLimitNs / 4);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax, one key per thread (warps 2..5)
+    const int sw = warp - 2;
+    const int quad = warp & 3;                       // TMEM lanes 32 * (warp % 4) ..
+    const int kt = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    const float c2 = plan.scale2;
+    const bool odd = lane & 1;
+    for (int t = 0; t < ntiles && !stop; ++t) {
+#pragma unroll
+      for (int h = 0; h < HKV; ++h) {         // compile-time head: the partial sums stay in registers
+        const int n = t * HKV + h, buf = n & 1;
+        // every wait of the stage comes first; the group leaves only together, at a barrier
+        bool ok = __all_sync(0xffffffffu, d_wait(&bars->s_full[buf], (n >> 1) & 1u, bars, err, 95));
+        if (ok && t >= 1)   // the head's previous O^T MMAs are done: its P tile and O^T are free
+          ok = __all_sync(0xffffffffu, d_wait(&bars->p_empty[h], (t - 1) & 1u, bars, err, 96));
+        const int key = tb + t * kDM + kt;
+        const bool valid = key < te;
+        const float *m_old = msm + ((t & 1) ^ 1) * HKV * kDRows + h * kDRows;
+        float *m_new = msm + (t & 1) * HKV * kDRows + h * kDRows;
+        float x[kDRows], m[kDRows];
+        bool raise = false;
+#pragma unroll
+        for (int j = 0; j < kDRows; ++j) x[j] = -INFINITY;
+        if (ok) {
+          tc_fence_after();
+          uint32_t r[8];
+          tmem_ld8_wait(bars->tmem_base + lane_off + buf * kDN, r);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars->s_empty[buf]);
+#pragma unroll
+          for (int j = 0; j < kDRows; ++j) {
+            x[j] = (valid && j < G) ? __uint_as_float(r[j]) * c2 : -INFINITY;
+            m[j] = m_old[j];
+            raise |= x[j] > m[j] + kDLazy;           // also every finite logit against -inf
+          }
+        }
+        const bool bad = !ok || bars->abort;
+        if (bar_red_or(1, kDSoftWarps * 32, bad || raise)) {
+          // slow path (the first tile, a new maximum, or an abort): the tile's row maxima
+          float *tm = tmax + buf * kDSoftWarps * kDRows;
+#pragma unroll
+          for (int j = 0; j < kDRows; ++j) {
+            float wm = x[j];
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, off));
+            if (lane == 0) tm[sw * kDRows + j] = wm;
+          }
+          if (bar_red_or(1, kDSoftWarps * 32, bad)) {
+            stop = true;
+            break;
+          }
+          float f[kDRows];
+          bool any = false;
+#pragma unroll
+          for (int j = 0; j < kDRows; ++j) {
+            const float mt = fmaxf(fmaxf(tm[j], tm[kDRows + j]), fmaxf(tm[2 * kDRows + j], tm[3 * kDRows + j]));
+            f[j] = 1.f;
+            if (mt > m[j] + kDLazy) {               // the same decision in every thread
+              f[j] = m[j] == -INFINITY ? 0.f : ex2_approx(m[j] - mt);
+              m[j] = mt;
+              any = true;
+            }
+            l_run[h][j] *= f[j];
+          }
+          if (any && t > 0) {
+            // rescale the head's O^T columns (this thread's feature kt): hi and lo alike
+            uint32_t o[16];
+            tc_fence_after();
+            tmem_ld16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
+#pragma unroll
+            for (int j = 0; j < kDRows; ++j) {
+              o[j] = __float_as_uint(__uint_as_float(o[j]) * f[j]);
+              o[j + 8] = __float_as_uint(__uint_as_float(o[j + 8]) * f[j]);
+            }
+            tmem_st16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
+            tc_fence_before();
+          }
+        }
+        // p = exp2(s - m) as a bf16 pair into the head's P^T tile; the even lane of a key pair
+        // writes the high parts of both keys, the odd lane the low parts (rows rotated by 4 so
+        // that the two halves of the warp hit different banks)
+        uint32_t hl[kDRows];                         // (hi | lo << 16) of this key, per row
+#pragma unroll
+        for (int j = 0; j < kDRows; ++j) {
+          const float p = x[j] == -INFINITY ? 0.f : ex2_approx(x[j] - m[j]);
+          l_run[h][j] += p;
+          const __nv_bfloat16 hi = __float2bfloat16_rn(p);
+          const __nv_bfloat16 lo = __float2bfloat16_rn(p - __bfloat162float(hi));
+          hl[j] = static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
+                  (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16);
+        }
+        uint8_t *pt = ps + h * kDPBytes;
+#pragma unroll
+        for (int j = 0; j < kDRows; ++j) {
+          const int jl = (j + 4) & 7;
+          const uint32_t send = odd ? (hl[j] & 0xFFFFu) : (hl[jl] >> 16);
+          const uint32_t recv = __shfl_xor_sync(0xffffffffu, send, 1);
+          if (!odd)   // keys kt, kt + 1: high parts of row j
+            *reinterpret_cast<uint32_t *>(pt + p_off(j, kt)) = (hl[j] & 0xFFFFu) | (recv << 16);
+          else        // keys kt - 1, kt: low parts of row jl
+            *reinterpret_cast<uint32_t *>(pt + p_off(8 + jl, kt - 1)) = recv | (hl[jl] & 0xFFFF0000u);
+        }
+        if (kt == 0)
+#pragma unroll
+          for (int j = 0; j < kDRows; ++j) m_new[j] = m[j];
+        fence_proxy_async_smem();                    // the P tile is read by the tensor cores
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->p_full[h]);
+      }
+    }
+    // the head's last O^T MMAs must be complete before O^T is read
+    if (!stop)
+#pragma unroll
+      for (int h = 0; h < HKV; ++h)
+        if (!__all_sync(0xffffffffu, d_wait(&bars->p_empty[h], (ntiles - 1) & 1u, bars, err, 97))) break;
+  }
+
+  // ---------------------------------------------------------------- epilogue and teardown
+  tc_fence_before();
+  __syncthreads();                              // every stage consumed: the ring is free
+  tc_fence_after();
+  const bool ok = !bars->abort;
+  float *lsum = reinterpret_cast<float *>(ring);                         // [HKV * 8][128 keys]
+  float *mrow = lsum + kDM * HKV * kDRows;                                // [HKV][8]
+  if (ok && warp >= 2 && warp < kDPvWarp) {
+    const int quad = warp & 3, kt = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+#pragma unroll
+    for (int h = 0; h < HKV; ++h) {
+      uint32_t o[16];
+      tmem_ld16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
+#pragma unroll
+      for (int j = 0; j < kDRows; ++j)           // feature kt of row j: high plus low part
+        if (j < G)
+          opart[(static_cast<int64_t>(c) * plan.hq + h * G + j) * 128 + kt] =
+              __uint_as_float(o[j]) + __uint_as_float(o[j + 8]);
+#pragma unroll
+      for (int j = 0; j < kDRows; ++j) lsum[(h * kDRows + j) * kDM + kt] = l_run[h][j];
+    }
+    if (kt == 0)   // the last tile's copy of the reference maximum
+#pragma unroll
+      for (int h = 0; h < HKV; ++h)
+#pragma unroll
+        for (int j = 0; j < kDRows; ++j) mrow[h * kDRows + j] = msm[((ntiles - 1) & 1) * HKV * kDRows + h * kDRows + j];
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (ok) {
+    // one warp per (head, row): the 128 partial sums in a fixed order
+    for (int e = warp; e < HKV * G; e += kDThreads / 32) {
+      const int h = e / G, j = e % G;
+      const float4 l4 = *reinterpret_cast<const float4 *>(lsum + (h * kDRows + j) * kDM + lane * 4);
+      float l = (l4.x + l4.y) + (l4.z + l4.w);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
+      if (lane == 0) mlpart[static_cast<int64_t>(c) * plan.hq + h * G + j] = make_float2(mrow[h * kDRows + j], l);
+    }
+  }
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(bars->tmem_base, kDTmemCols);
+}
+
+}  // namespace
+
+cudaError_t launch_decode_tc(int grid, cudaStream_t stream, const CUtensorMap &kmap, const CUtensorMap &vmap,
+                             const DecPlan &P, const uint16_t *q, float *opart, float2 *mlpart, DeviceError *err) {
+  if (P.hkv == 4) {
+    static bool attr = false;
+    if (!attr) {
+      const cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 static_cast<int>(DLay<4>::kBytes));
+      if (e != cudaSuccess) return e;
+      attr = true;
+    }
+    decode_tc_kernel<4><<<grid, kDThreads, DLay<4>::kBytes, stream>>>(kmap, vmap, P, q, opart, mlpart, err);
+  } else {
+    static bool attr = false;
+    if (!attr) {
+      const cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 static_cast<int>(DLay<2>::kBytes));
+      if (e != cudaSuccess) return e;
+      attr = true;
+    }
+    decode_tc_kernel<2><<<grid, kDThreads, DLay<2>::kBytes, stream>>>(kmap, vmap, P, q, opart, mlpart, err);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace apack

@@ -119,3 +119,31 @@ def test_decode_attention_batch_beyond_one_launch(ap):
     k = bits(rng, (T, 4, 128), 1.5)
     v = bits(rng, (T, 4, 128))
     check(run(ap, cu, q, k, v, 28, 4), oracle.decode_attention(q, k, v, cu, 28, 4))
+
+
+@pytest.mark.parametrize("hq,hkv", [(28, 4), (16, 2)])
+def test_decode_attention_rising_and_falling_maxima(ap, hq, hkv):
+    # Row j of every head group reads feature j of the keys (q = 8 e_j, so a key value x gives
+    # a logit of about 1.02 x in log2 units).  Feature j steps by 12 every 128 keys with period
+    # 5 blocks: up for even rows (a new maximum about 2^12 above the previous one at every
+    # block of a chunk), down for odd rows (the first block holds the maximum), plus one spike
+    # late in row 1.  Long sequences, so that every chunk of keys spans several blocks.
+    G = hq // hkv
+    rng = np.random.default_rng(11 + hq)
+    lens = [40000, 9001]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = int(cu[-1])
+    qf = np.zeros((len(lens), hq, 128), np.float32)
+    for h in range(hq):
+        qf[:, h, h % G] = 8.0
+    kf = rng.standard_normal((T, hkv, 128)).astype(np.float32) * 0.25
+    for b, n in enumerate(lens):
+        step = (np.arange(n) // 128) % 5
+        for j in range(G):
+            kf[cu[b]:cu[b + 1], :, j] = (12.0 * step if j % 2 == 0 else 12.0 * (4 - step))[:, None]
+        kf[cu[b] + n - 5, :, 1] = 70.0
+    q = f32_to_bf16_bits(qf)
+    k = f32_to_bf16_bits(kf)
+    v = bits(rng, (T, hkv, 128))
+    got = run(ap, cu, q, k, v, hq, hkv)
+    check(got, oracle.decode_attention(q, k, v, cu, hq, hkv))
