@@ -460,15 +460,18 @@ def decode_measure(ap, wl, pp, steps, warmup, stream, dist):
     ms_full, T_full, launches, calls = res["full"]
     alg = T_full * hkv * 128 * 2 * 2 + hq * 128 * (2 + 4)
     achieved = alg / (ms_full / 1e3) / 1e9
+    prof = profiled_traffic("decode_tc.cu", "decode_traffic.json") if hkv in (2, 4) and hq // hkv <= 8 else None
+    traffic = int(prof["traffic_over_algorithmic"] * alg) if prof is not None else None
+    kern = ("decode_tc_kernel + decode_combine_kernel" if hkv in (2, 4) and hq // hkv <= 8
+            else "decode_chunk_kernel + decode_combine_kernel")
     return {"metric": "decode-step attention time per layer, uncompressed vs compacted cache",
             "layers": f"{l_last}..{wl.num_layers - 1}", "tokens": [T_full, res["compacted"][1]],
             "full_ms_per_layer": ms_full, "compacted_ms_per_layer": res["compacted"][0],
             "speedup": ms_full / res["compacted"][0], "calls_timed": calls,
             "gpu_launches_per_call": launches / calls,
-            "roofline": {"bound": "hbm", "kernel": "apack_decode_attention call on the uncompressed cache "
-                                                   "(decode_chunk_kernel + decode_combine_kernel)",
+            "roofline": {"bound": "hbm", "kernel": f"apack_decode_attention call on the uncompressed cache ({kern})",
                          "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                         "traffic": None, "peak_source": peak_kind, "algorithmic_bytes_per_launch": alg,
+                         "traffic": traffic, "peak_source": peak_kind, "algorithmic_bytes_per_launch": alg,
                          "note": "K and V of one layer read once, q read and out written once"}}
 
 
