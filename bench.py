@@ -46,6 +46,10 @@ def parse():
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=None)
+    p.add_argument("--part", default="all", choices=["all", "decode"],
+                   help="decode: time only the decode-step attention on a synthetic cache")
+    p.add_argument("--decode-tokens", type=int, default=135272)
+    p.add_argument("--decode-layers", type=int, default=8)
     return p.parse_args()
 
 
@@ -475,6 +479,51 @@ def decode_measure(ap, wl, pp, steps, warmup, stream, dist):
                          "note": "K and V of one layer read once, q read and out written once"}}
 
 
+def decode_only(args):
+    """Decode-step attention alone: one decode token of a single sequence over a synthetic
+    cache of `--decode-tokens` keys (7B heads, 28 query / 4 KV), rotating over
+    `--decode-layers` layers.  Prints one JSON line (time per layer, roofline)."""
+    import torch
+    import paper_2608_08794_gb300 as ap
+    from synth.gen import TID_Q
+    from synth.device import fill_normal_bf16
+    hq, hkv, T, nl = 28, 4, args.decode_tokens, args.decode_layers
+    stream = torch.cuda.current_stream()
+    ks = [torch.empty(T, hkv * 128, dtype=torch.bfloat16, device="cuda") for _ in range(nl)]
+    vs = [torch.empty(T, hkv * 128, dtype=torch.bfloat16, device="cuda") for _ in range(nl)]
+    for j in range(nl):
+        fill_normal_bf16(ks[j], 17, 2 * j, stream=stream)
+        fill_normal_bf16(vs[j], 17, 2 * j + 1, stream=stream)
+    q = torch.empty(1, hq, 128, dtype=torch.bfloat16, device="cuda")
+    fill_normal_bf16(q, 17, TID_Q, stream=stream)
+    out = torch.empty(1, hq, 128, dtype=torch.float32, device="cuda")
+    cu = [0, T]
+    ws = torch.zeros(max(256, ap.apack_decode_workspace_size(cu, hq, hkv)), dtype=torch.uint8, device="cuda")
+    for j in range(args.warmup * nl):
+        ap.apack_decode_attention(cu, q, ks[j % nl], vs[j % nl], hkv * 256, hq, hkv, out, ws, stream=stream)
+    torch.cuda.synchronize()
+    n = args.steps * nl
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for j in range(n):
+        ap.apack_decode_attention(cu, q, ks[j % nl], vs[j % nl], hkv * 256, hq, hkv, out, ws, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if ap.apack_device_error(ws) != ap.APACK_OK:
+        raise RuntimeError("decode attention reported a device error")
+    ms = e0.elapsed_time(e1) / n
+    peak, peak_kind = measured_peaks()
+    alg = T * hkv * 128 * 2 * 2 + hq * 128 * (2 + 4)
+    achieved = alg / (ms / 1e3) / 1e9
+    print(json.dumps({"metric": "decode-step attention time per layer", "value": ms, "unit": "ms",
+                      "higher_is_better": False, "steps": args.steps, "warmup": args.warmup,
+                      "config": {"workload": f"one sequence, {T} cached tokens, 28 query / 4 KV heads, "
+                                             f"{nl} layers rotated", "dtype": "bf16"},
+                      "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                                   "frac": achieved / peak, "peak_source": peak_kind,
+                                   "algorithmic_bytes_per_launch": alg}}))
+
+
 # ----------------------------------------------------------------------------- GPU leg
 
 def main():
@@ -484,6 +533,9 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         reference_arm(args, rank, world)
+        return
+    if args.part == "decode":
+        decode_only(args)
         return
 
     import numpy as np
