@@ -243,6 +243,27 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
                                   int32_t num_steps, float *scores, void *ws, size_t ws_bytes,
                                   void *const *stage_events_h, void *stream);
 
+/* ---- The schedule as a CUDA graph.
+   apack_prune_schedule_graph makes the same checks and host planning as
+   apack_prune_schedule (same arguments, no stage events) once, and captures its
+   launches into an executable CUDA graph; it launches nothing itself.  It
+   writes steps_h[i].new_cu_seqlens_h as the direct call does.
+   apack_graph_launch replays those launches on `stream`, with the same
+   pointers, sizes and keep counts: one graph launch instead of one launch per
+   kernel, for a schedule that repeats with fixed shapes (a serving bucket).
+   Every device buffer named at capture must stay allocated while the graph is
+   used; the host-side arguments are not read again after the capture returns.
+   apack_graph_destroy frees the graph.  Errors: the capture's own checks
+   (as apack_prune_schedule), APACK_ECUDA if the driver refuses the capture. */
+typedef struct apack_graph_s *apack_graph;
+apack_status apack_prune_schedule_graph(const apack_seqs *seqs, int32_t num_layers, const void *k_cache,
+                                        const void *v_cache, int64_t kv_layer_stride, const void *hidden,
+                                        int64_t hidden_dim, int32_t select_mode, const apack_step *steps_h,
+                                        int32_t num_steps, float *scores, void *ws, size_t ws_bytes,
+                                        apack_graph *graph_out);
+apack_status apack_graph_launch(apack_graph graph, void *stream);
+apack_status apack_graph_destroy(apack_graph graph);
+
 /* ---- Decode-step attention over a (compacted) KV cache.
    Sec. 3.2 (last sentence) and App. G: pruning shortens the cache that every
    autoregressive decode step attends to.  One decode token per sequence:

@@ -28,7 +28,8 @@ APACK_HEAD_DIM = 128
 EXPORTED = ("apack_workspace_size", "apack_keep_counts", "apack_score", "apack_select", "apack_compact",
             "apack_prune_step", "apack_device_error", "apack_launch_count", "apack_status_string",
             "apack_score_static", "apack_frame_alignment_workspace_size", "apack_frame_alignment",
-            "apack_decode_workspace_size", "apack_decode_attention", "apack_prune_schedule")
+            "apack_decode_workspace_size", "apack_decode_attention", "apack_prune_schedule",
+            "apack_prune_schedule_graph", "apack_graph_launch", "apack_graph_destroy")
 
 
 class ApackError(RuntimeError):
@@ -88,6 +89,10 @@ def _load():
     lib.apack_decode_attention.argtypes = [I32, PI32, VP, VP, VP, I64, I32, I32, VP, VP, SZ, VP]
     lib.apack_prune_schedule.argtypes = [P(apack_seqs), I32, VP, VP, I64, VP, I64, I32, P(apack_step), I32, VP, VP,
                                          SZ, P(VP), VP]
+    lib.apack_prune_schedule_graph.argtypes = [P(apack_seqs), I32, VP, VP, I64, VP, I64, I32, P(apack_step), I32,
+                                               VP, VP, SZ, P(VP)]
+    lib.apack_graph_launch.argtypes = [VP, VP]
+    lib.apack_graph_destroy.argtypes = [VP]
     lib.apack_launch_count.argtypes = []
     lib.apack_launch_count.restype = ctypes.c_uint64
     lib.apack_status_string.argtypes = [I32]
@@ -250,7 +255,8 @@ def _event_handles(events, n, what):
 
 
 def apack_prune_schedule(seqs, num_layers, k_cache, v_cache, kv_layer_stride, hidden, hidden_dim, steps,
-                         select_mode=APACK_SELECT_PER_MODALITY, scores=None, ws=None, stage_events=None, stream=None):
+                         select_mode=APACK_SELECT_PER_MODALITY, scores=None, ws=None, stage_events=None, stream=None,
+                         capture=False):
     """A whole progressive schedule (one apack_prune_step per entry of `steps`, each
     reading the previous step's outputs).  steps: dicts with layer, q, keep_count or
     keep_ratio, k_out, v_out, kv_out_layer_stride, hidden_out, modality_out, keep_idx
@@ -289,12 +295,46 @@ def apack_prune_schedule(seqs, num_layers, k_cache, v_cache, kv_layer_stride, hi
         new_cus.append(cu)
         st.new_cu_seqlens_h = cu.ctypes.data_as(I32P)
         st.new_cu_seqlens = _ptr(d.get("new_cu_seqlens"))
+    head = (seqs.ref(), int(num_layers), _ptr(k_cache), _ptr(v_cache), int(kv_layer_stride), _ptr(hidden),
+            int(hidden_dim), int(select_mode), arr, n, _ptr(scores), _ptr(ws),
+            0 if ws is None else ws.numel() * ws.element_size())
+    if capture:
+        g = ctypes.c_void_p()
+        _check(_lib.apack_prune_schedule_graph(*head, ctypes.byref(g)), "apack_prune_schedule_graph")
+        return new_cus, ScheduleGraph(g)
     stage = _event_handles(stage_events, 4 * n, "stage_events")
-    _check(_lib.apack_prune_schedule(
-        seqs.ref(), int(num_layers), _ptr(k_cache), _ptr(v_cache), int(kv_layer_stride), _ptr(hidden),
-        int(hidden_dim), int(select_mode), arr, n, _ptr(scores), _ptr(ws),
-        0 if ws is None else ws.numel() * ws.element_size(), stage, _stream(stream)), "apack_prune_schedule")
+    _check(_lib.apack_prune_schedule(*head, stage, _stream(stream)), "apack_prune_schedule")
     return new_cus
+
+
+class ScheduleGraph:
+    """An executable CUDA graph of one schedule (apack_prune_schedule_graph);
+    launch() replays it, the graph is freed with the object."""
+
+    def __init__(self, handle):
+        self._h = handle
+
+    def launch(self, stream=None):
+        _check(_lib.apack_graph_launch(self._h, _stream(stream)), "apack_graph_launch")
+
+    def close(self):
+        if self._h is not None and self._h.value:
+            _check(_lib.apack_graph_destroy(self._h), "apack_graph_destroy")
+        self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def apack_prune_schedule_graph(seqs, num_layers, k_cache, v_cache, kv_layer_stride, hidden, hidden_dim, steps,
+                               select_mode=APACK_SELECT_PER_MODALITY, scores=None, ws=None):
+    """Captures the schedule of apack_prune_schedule (same arguments) into a CUDA
+    graph.  Returns (new host offsets of every step, ScheduleGraph)."""
+    return apack_prune_schedule(seqs, num_layers, k_cache, v_cache, kv_layer_stride, hidden, hidden_dim, steps,
+                                select_mode=select_mode, scores=scores, ws=ws, capture=True)
 
 
 def apack_score_static(seqs, q, k, k_token_stride, scores, device_error_out=None, stream=None):

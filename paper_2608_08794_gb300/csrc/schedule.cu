@@ -6,6 +6,7 @@
 // the hidden states and any extra planes to the kept tokens; step i+1 reads step i's
 // outputs.  All steps are planned and checked on the host before the first launch, then
 // run in order on one stream: the outputs are those of one apack_prune_step per step.
+#include <new>
 #include <vector>
 
 #include "internal.cuh"
@@ -138,6 +139,64 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
     mark(i, 3);
   }
   return APACK_OK;
+}
+
+struct apack_graph_s {
+  cudaGraphExec_t exec;
+  uint64_t launches;     // kernels per replay
+};
+
+apack_status apack_prune_schedule_graph(const apack_seqs *seqs, int32_t num_layers, const void *k_cache,
+                                        const void *v_cache, int64_t kv_layer_stride, const void *hidden,
+                                        int64_t hidden_dim, int32_t select_mode, const apack_step *steps_h,
+                                        int32_t num_steps, float *scores, void *ws, size_t ws_bytes,
+                                        apack_graph *graph_out) {
+  if (!graph_out) return APACK_EINVAL;
+  *graph_out = nullptr;
+  cudaStream_t cs = nullptr;
+  if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) return APACK_ECUDA;
+  const uint64_t before = apack_launch_count();
+  if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+    cudaStreamDestroy(cs);
+    return APACK_ECUDA;
+  }
+  apack_status st = apack_prune_schedule(seqs, num_layers, k_cache, v_cache, kv_layer_stride, hidden, hidden_dim,
+                                         select_mode, steps_h, num_steps, scores, ws, ws_bytes, nullptr, cs);
+  cudaGraph_t g = nullptr;
+  const cudaError_t ce = cudaStreamEndCapture(cs, &g);
+  const uint64_t captured = apack_launch_count() - before;
+  count_launches(0 - captured);                 // nothing ran: captured launches count when replayed
+  cudaStreamDestroy(cs);
+  if (st == APACK_OK && (ce != cudaSuccess || !g)) st = APACK_ECUDA;
+  cudaGraphExec_t exec = nullptr;
+  if (st == APACK_OK && cudaGraphInstantiate(&exec, g, 0) != cudaSuccess) st = APACK_ECUDA;
+  if (g) cudaGraphDestroy(g);
+  cudaGetLastError();                           // a refused capture leaves no sticky error behind
+  if (st != APACK_OK) {
+    if (exec) cudaGraphExecDestroy(exec);
+    return st;
+  }
+  apack_graph h = new (std::nothrow) apack_graph_s{exec, captured};
+  if (!h) {
+    cudaGraphExecDestroy(exec);
+    return APACK_ECUDA;
+  }
+  *graph_out = h;
+  return APACK_OK;
+}
+
+apack_status apack_graph_launch(apack_graph graph, void *stream) {
+  if (!graph) return APACK_EINVAL;
+  if (cudaGraphLaunch(graph->exec, static_cast<cudaStream_t>(stream)) != cudaSuccess) return APACK_ECUDA;
+  count_launches(graph->launches);
+  return APACK_OK;
+}
+
+apack_status apack_graph_destroy(apack_graph graph) {
+  if (!graph) return APACK_OK;
+  const cudaError_t e = cudaGraphExecDestroy(graph->exec);
+  delete graph;
+  return e == cudaSuccess ? APACK_OK : APACK_ECUDA;
 }
 
 }  // extern "C"

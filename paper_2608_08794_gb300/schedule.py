@@ -15,7 +15,8 @@ Only buffer management and argument marshalling happen here.
 import numpy as np
 import torch
 
-from . import (Seqs, apack_plane, apack_prune_step, apack_prune_schedule, apack_workspace_size, apack_keep_counts,
+from . import (Seqs, apack_plane, apack_prune_step, apack_prune_schedule, apack_prune_schedule_graph,
+               apack_workspace_size, apack_keep_counts,
                APACK_HEAD_DIM, APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT)
 
 
@@ -135,25 +136,35 @@ class ProgressivePrune:
         v = self.v_out[prev][off:]
         return (self._step_seqs(i), k, v, t_prev * self.row, self.h_out[prev])
 
-    def run(self, events=None, stream=None):
-        """Runs every step through apack_prune_schedule.  events: None or 4 CUDA
-        events per step (before scoring, after scoring, after selection, after
-        compaction)."""
-        n = len(self.layers)
+    def _schedule_steps(self):
         steps = []
-        for i in range(n):
+        for i in range(len(self.layers)):
             o = i % 2
             steps.append(dict(layer=self.layers[i], q=self.q[i], keep_count=self.counts[i], k_out=self.k_out[o],
                               v_out=self.v_out[o], kv_out_layer_stride=self.t_out[i] * self.row,
                               hidden_out=self.h_out[o], modality_out=self.mod_out[o], keep_idx=self.keep_idx[i],
                               extra_planes=self._below_planes(i)))
+        return steps
+
+    def run(self, events=None, stream=None):
+        """Runs every step through apack_prune_schedule.  events: None or 4 CUDA
+        events per step (before scoring, after scoring, after selection, after
+        compaction)."""
         flat = None
         if events is not None:
             flat = [e for per_step in events for e in per_step]
         self.new_cu = apack_prune_schedule(
             self._step_seqs(0), self.L, self.k_in.view(-1), self.v_in.view(-1), self.T0 * self.row,
-            self.hidden_in, self.H, steps, select_mode=self.mode, scores=self.scores, ws=self.ws,
+            self.hidden_in, self.H, self._schedule_steps(), select_mode=self.mode, scores=self.scores, ws=self.ws,
             stage_events=flat, stream=stream)
+
+    def capture(self):
+        """The schedule of run() as a CUDA graph (apack_prune_schedule_graph):
+        graph.launch(stream) replays every launch with these buffers."""
+        self.new_cu, graph = apack_prune_schedule_graph(
+            self._step_seqs(0), self.L, self.k_in.view(-1), self.v_in.view(-1), self.T0 * self.row,
+            self.hidden_in, self.H, self._schedule_steps(), select_mode=self.mode, scores=self.scores, ws=self.ws)
+        return graph
 
     def run_steps(self, events=None, stream=None):
         """Runs every step with one apack_prune_step call each; events[i] = 4 CUDA

@@ -170,6 +170,45 @@ def test_schedule_runner_is_bit_identical_to_single_steps(ap, name):
     same(ref, snapshot(pp))
 
 
+@pytest.mark.parametrize("name", ["7b_2min", "7b_ragged16", "7b_10min_paper"])
+def test_schedule_graph_replay_is_bit_identical(ap, name):
+    """apack_prune_schedule_graph captures the schedule once; every replay leaves
+    exactly the outputs of apack_prune_schedule (also after the outputs were
+    wiped), and counts the captured kernels as launched per replay only."""
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+
+    wl = workload(name)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod_d = torch.from_numpy(wl.modality()).cuda()
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_d,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
+    pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                          wl.prune_layers, counts, select_mode=mode)
+    fill_progressive_inputs(pp, wl)
+    c0 = ap.apack_launch_count()
+    pp.run()
+    torch.cuda.synchronize()
+    per_run = ap.apack_launch_count() - c0
+    ref = snapshot(pp)
+    c1 = ap.apack_launch_count()
+    graph = pp.capture()
+    assert ap.apack_launch_count() == c1          # capturing runs nothing
+    for buf in pp.k_out + pp.v_out + pp.h_out + pp.mod_out + pp.keep_idx:
+        if buf is not None:
+            buf.zero_()
+    for _ in range(2):
+        graph.launch()
+    torch.cuda.synchronize()
+    assert ap.apack_launch_count() - c1 == 2 * per_run
+    assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+    same(ref, snapshot(pp))
+    graph.close()
+
+
 @pytest.mark.parametrize("name", ["7b_2min", "7b_10min_paper"])
 def test_slicing_below_the_pruning_layers_keeps_every_layer_consistent(ap, name):
     """With slice_below, every step also compacts the caches of the layers below its
