@@ -1,7 +1,8 @@
 // select.cu -- per-(sequence, modality) top-k of Eq. inner (Sec. 3.2) and the stable keep map.
 //
-// One thread-block cluster of kCluster CTAs per sequence; CTA c owns a
-// contiguous slice of the sequence's tokens.
+// One thread-block cluster of CL CTAs per sequence (16 when the launch's clusters
+// still fit the GPU that way, else 8); CTA c owns a contiguous slice of the
+// sequence's tokens.
 //
 //  1. Radix select (4 passes of 8 bits, most significant first) of the k-th
 //     largest score of every segment.  Scores are >= 0, so the order of their
@@ -29,7 +30,7 @@ namespace apack {
 
 namespace {
 
-constexpr int kCluster = 8;
+constexpr int kClusterSmall = 8, kClusterLarge = 16;
 constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxCached = 40960;               // tokens per CTA slice cached in shared memory (200 KB)
@@ -96,14 +97,15 @@ __device__ __forceinline__ void add_bin(uint32_t *h, int bin, int lane) {
   }
 }
 
-__global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
+template <int CL>
+__global__ void __cluster_dims__(CL, 1, 1) __launch_bounds__(kThreads)
     select_kernel(const __grid_constant__ SelectPlan plan, const float *__restrict__ scores,
                   const uint8_t *__restrict__ modality, int32_t *__restrict__ keep_idx,
                   uint8_t *__restrict__ modality_out, int32_t *__restrict__ dst_of_src,
                   int32_t *__restrict__ new_cu, DeviceError *err) {
   __shared__ uint32_t hist[2][2][256];
   __shared__ uint32_t tot[2][256];            // cluster-wide histogram of the current pass
-  __shared__ uint32_t rcnt[kCluster][5];      // per-CTA counts of the cluster
+  __shared__ uint32_t rcnt[CL][5];            // per-CTA counts of the cluster
   __shared__ uint32_t st_prefix[2], st_mask[2], st_krem[2], st_total[2];
   __shared__ uint32_t wcnt[kWarps][5];        // per warp chunk: other, gt0, gt1, eq0, eq1
   __shared__ uint32_t cnt[5];                 // per CTA (read by the cluster)
@@ -115,7 +117,7 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const uint32_t lt_mask = (1u << lane) - 1u;
   const int nsegs = plan.nsegs;
-  const int chunk = (sq.len + kCluster - 1) / kCluster;
+  const int chunk = (sq.len + CL - 1) / CL;
   const int lo = sq.t0 + min(sq.len, static_cast<int>(crank) * chunk);
   const int hi = sq.t0 + min(sq.len, static_cast<int>(crank + 1) * chunk);
   // each warp owns a contiguous run of the slice (a multiple of 32 tokens)
@@ -167,14 +169,14 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
     cluster_sync();
     for (int j = tid; j < 2 * 256; j += kThreads) (&hist[hb ^ 1][0][0])[j] = 0u;
     // cluster-wide histogram: thread (seg, bin) adds the bin of every CTA, its
-    // kCluster remote loads issued back to back
+    // CL remote loads issued back to back
     for (int j = tid; j < nsegs * 256; j += kThreads) {
-      uint32_t v[kCluster];
+      uint32_t v[CL];
 #pragma unroll
-      for (int r = 0; r < kCluster; ++r) v[r] = ld_shared_cluster_u32(map_shared_rank(&(&hist[hb][0][0])[j], r));
+      for (int r = 0; r < CL; ++r) v[r] = ld_shared_cluster_u32(map_shared_rank(&(&hist[hb][0][0])[j], r));
       uint32_t sum = 0;
 #pragma unroll
-      for (int r = 0; r < kCluster; ++r) sum += v[r];
+      for (int r = 0; r < CL; ++r) sum += v[r];
       (&tot[0][0])[j] = sum;
     }
     __syncthreads();
@@ -263,14 +265,14 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
   }
   __syncthreads();
   cluster_sync();
-  if (tid < kCluster * 5) rcnt[tid / 5][tid % 5] = ld_shared_cluster_u32(map_shared_rank(&cnt[tid % 5], tid / 5));
+  if (tid < CL * 5) rcnt[tid / 5][tid % 5] = ld_shared_cluster_u32(map_shared_rank(&cnt[tid % 5], tid / 5));
   __syncthreads();
   if (tid == 0) {
     // Walk the CTAs of the cluster, then the warps of this CTA, in token order:
     // ties are granted until the quota runs out.
     uint32_t kept_before = 0, kept_all = 0, seg_dev[2] = {0, 0};
     uint32_t eq_prefix[2] = {0, 0}, eqb[2] = {0, 0};
-    for (int r = 0; r < kCluster; ++r) {
+    for (int r = 0; r < CL; ++r) {
       const uint32_t *c = rcnt[r];
       uint32_t kept = c[0] + c[1] + c[2];
       for (int s = 0; s < 2; ++s) {
@@ -400,25 +402,54 @@ apack_status run_select(const apack_seqs *seqs, const float *scores, const int32
       q.out_base = out_base;
       out_base += q.out_len;
     }
+    // 16-CTA clusters while every sequence of the launch still gets its own 16 SMs
+    static int large_ok = -1;
+    if (large_ok < 0) {
+      large_ok = cudaFuncSetAttribute(select_kernel<kClusterLarge>, cudaFuncAttributeNonPortableClusterSizeAllowed,
+                                      1) == cudaSuccess &&
+                 cudaFuncSetAttribute(select_kernel<kClusterLarge>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(kCacheBytes)) == cudaSuccess &&
+                 cudaFuncSetAttribute(select_kernel<kClusterSmall>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(kCacheBytes)) == cudaSuccess;
+      if (large_ok) {   // can a 16-CTA cluster of this kernel be resident at all?
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = kClusterLarge;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(kClusterLarge, 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = kCacheBytes;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        int nclusters = 0;
+        large_ok = cudaOccupancyMaxActiveClusters(&nclusters, select_kernel<kClusterLarge>, &cfg) == cudaSuccess &&
+                   nclusters > 0;
+      }
+      cudaGetLastError();
+      if (!large_ok &&
+          check_cuda(cudaFuncSetAttribute(select_kernel<kClusterSmall>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          static_cast<int>(kCacheBytes))) != APACK_OK)
+        return APACK_ECUDA;
+    }
+    const int CL = (large_ok && ns * kClusterLarge <= device_sm_count()) ? kClusterLarge : kClusterSmall;
     // cache each CTA's slice in shared memory when the longest slice of the launch fits
     int max_len = 0;
     for (int i = 0; i < ns; ++i) max_len = P.seq[i].len > max_len ? P.seq[i].len : max_len;
-    const int slice = (max_len + kCluster - 1) / kCluster;
+    const int slice = (max_len + CL - 1) / CL;
     size_t smem = 0;
     if (slice <= kMaxCached) {
       P.cache_tokens = slice;
       smem = static_cast<size_t>(slice) * 5;
     }
-    static bool attr_done = false;
-    if (!attr_done) {
-      if (check_cuda(cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          static_cast<int>(kCacheBytes))) != APACK_OK)
-        return APACK_ECUDA;
-      attr_done = true;
-    }
-    dim3 grid(kCluster, ns, 1);
-    select_kernel<<<grid, kThreads, smem, stream>>>(P, scores, seqs->modality, keep_idx, modality_out, dst_of_src,
-                                                    new_cu_seqlens, err);
+    dim3 grid(CL, ns, 1);
+    if (CL == kClusterLarge)
+      select_kernel<kClusterLarge><<<grid, kThreads, smem, stream>>>(P, scores, seqs->modality, keep_idx, modality_out,
+                                                                     dst_of_src, new_cu_seqlens, err);
+    else
+      select_kernel<kClusterSmall><<<grid, kThreads, smem, stream>>>(P, scores, seqs->modality, keep_idx, modality_out,
+                                                                     dst_of_src, new_cu_seqlens, err);
     count_launches(1);
     if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
   }
