@@ -27,6 +27,13 @@ loop; Table S-hparams "Query score"):
    layers, hidden states, metadata) is copied so that output row j is input
    row keep_idx[j].
 
+A second softmax domain is offered as a reading of the north star's "full
+key row": the denominator of Eq. (inner_score) then runs over the decoder's
+causal attention row of the query token, i.e. every token at or before the
+query row's position (system, text, audio, visual and query tokens), with the
+query rows taken as the last n_q tokens of the sequence; a token of S after a
+row's position gets nothing from that row.
+
 The arithmetic is fp64 from exactly widened bf16 inputs; numpy's matmul,
 exp and stable argsort are the only library steps.
 """
@@ -36,6 +43,7 @@ import math
 import numpy as np
 
 MOD_OTHER, MOD_AUDIO, MOD_VISUAL = 0, 1, 2
+SOFTMAX_MM, SOFTMAX_CAUSAL_ROW = 0, 1
 
 
 def bf16_to_f64(bits):
@@ -45,14 +53,18 @@ def bf16_to_f64(bits):
 
 
 def relevance_scores(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads,
-                     row_chunk=512):
+                     row_chunk=512, softmax_domain=SOFTMAX_MM):
     """Eq. (inner_score), averaged over query heads and query rows.
 
     q_bits: uint16 [sum n_q, Hq, D] (bf16) query rows, packed per sequence by cu_qlens.
     k_bits: uint16 [T, Hkv, D] (bf16) keys of the pruning layer, packed by cu_seqlens.
     modality: uint8 [T]; 1 = audio, 2 = visual form S, anything else is outside S.
+    softmax_domain: SOFTMAX_MM (the denominator over S, as Eq. inner_score prints it) or
+    SOFTMAX_CAUSAL_ROW (over the causal attention row; see the module docstring).
     Returns float64 [T]; 0 outside S.
     """
+    if softmax_domain == SOFTMAX_CAUSAL_ROW:
+        return _relevance_causal(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads)
     q_bits = np.asarray(q_bits)
     k_bits = np.asarray(k_bits)
     T = k_bits.shape[0]
@@ -79,6 +91,37 @@ def relevance_scores(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads
                 p /= p.sum(axis=1, keepdims=True)
                 acc += p.sum(axis=0)
         scores[mm] = acc / (num_q_heads * n_q)                   # mean over heads and rows
+    return scores
+
+
+def _relevance_causal(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads):
+    """Eq. (inner_score) with the causal-row denominator: query row r of a
+    sequence of length L with n_q query rows is token p_r = L - n_q + r; its
+    softmax runs over the tokens 0..p_r of the sequence, and the score of a token
+    i of S averages that row's probability of i (0 when i > p_r) over heads and rows."""
+    q_bits = np.asarray(q_bits)
+    k_bits = np.asarray(k_bits)
+    T = k_bits.shape[0]
+    D = k_bits.shape[2]
+    group = num_q_heads // num_kv_heads
+    scores = np.zeros(T, dtype=np.float64)
+    for s in range(len(cu_seqlens) - 1):
+        t0, t1 = int(cu_seqlens[s]), int(cu_seqlens[s + 1])
+        r0, r1 = int(cu_qlens[s]), int(cu_qlens[s + 1])
+        n_q, L = r1 - r0, t1 - t0
+        in_s = (modality[t0:t1] == MOD_AUDIO) | (modality[t0:t1] == MOD_VISUAL)
+        if not in_s.any() or n_q == 0:
+            continue
+        acc = np.zeros(L, dtype=np.float64)
+        for h in range(num_q_heads):
+            keys = bf16_to_f64(k_bits[t0:t1, h // group, :])     # [L, D], every token
+            for r in range(n_q):
+                p = L - n_q + r                                   # position of query row r
+                qv = bf16_to_f64(q_bits[r0 + r, h, :])
+                x = (keys[:p + 1] @ qv) / math.sqrt(D)            # the row's visible logits
+                e = np.exp(x - x.max())
+                acc[:p + 1] += e / e.sum()
+        scores[t0:t1] = np.where(in_s, acc / (num_q_heads * n_q), 0.0)
     return scores
 
 
@@ -139,10 +182,11 @@ def compact_rows(plane, keep_idx):
 
 
 def prune_step(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads,
-               keep_counts, planes=(), joint=False):
+               keep_counts, planes=(), joint=False, softmax_domain=SOFTMAX_MM):
     """One inner-LLM pruning step: scores, kept indices, new offsets and the
     compacted planes (each a per-token array, first axis = token)."""
-    scores = relevance_scores(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads)
+    scores = relevance_scores(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads,
+                              softmax_domain=softmax_domain)
     keep_idx = select_keep(scores, modality, cu_seqlens, keep_counts, joint=joint)
     return dict(scores=scores, keep_idx=keep_idx,
                 cu_seqlens=new_cu_seqlens(keep_idx, cu_seqlens),

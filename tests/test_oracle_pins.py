@@ -317,3 +317,103 @@ def test_compaction_row_by_row_and_progressive_composition():
     k2 = oracle.select_keep(scores[k1], mod1, cu1, [(1, 2), (1, 1)])
     out2 = oracle.compact_rows(out1, k2)
     np.testing.assert_array_equal(out2, oracle.compact_rows(plane, k1[k2]))
+
+
+# ---------------------------------------------------------------- causal-row softmax domain
+
+def brute_scores_causal(q_bits, k_bits, cu, cuq, mod, Hq, Hkv):
+    """Arbitrary-precision reference of the causal-row domain: query row r of a
+    sequence of length L is token L - n_q + r; its softmax runs over tokens
+    0..L - n_q + r of the sequence (every modality), explicit loops at 40 digits."""
+    mpmath.mp.dps = 40
+    q = oracle.bf16_to_f64(q_bits)
+    k = oracle.bf16_to_f64(k_bits)
+    T = k.shape[0]
+    out = [mpmath.mpf(0)] * T
+    g = Hq // Hkv
+    for s in range(len(cu) - 1):
+        t0, t1 = int(cu[s]), int(cu[s + 1])
+        nq = int(cuq[s + 1] - cuq[s])
+        if nq == 0 or not any(mod[i] in (1, 2) for i in range(t0, t1)):
+            continue
+        for h in range(Hq):
+            for r in range(nq):
+                pos = t1 - t0 - nq + r
+                vis = range(t0, t0 + pos + 1)
+                logits = {i: mpmath.fsum(mpmath.mpf(float(a)) * mpmath.mpf(float(b))
+                                         for a, b in zip(q[cuq[s] + r, h], k[i, h // g])) / mpmath.sqrt(D)
+                          for i in vis}
+                z = mpmath.fsum(mpmath.exp(x) for x in logits.values())
+                for i in vis:
+                    if mod[i] in (1, 2):
+                        out[i] += mpmath.exp(logits[i]) / z
+        for i in range(t0, t1):
+            out[i] /= Hq * nq
+    return np.array([float(v) for v in out])
+
+
+@pytest.mark.parametrize("Hq,Hkv,nq", [(4, 2, 3), (2, 2, 1), (6, 1, 4)])
+def test_causal_scores_match_arbitrary_precision_brute_force(Hq, Hkv, nq):
+    rng = np.random.default_rng(100 + Hq * 10 + Hkv)
+    # the second sequence has tokens of S among its last rows (inside the query span)
+    mod = np.array([0, 0, 1, 2, 2, 1, 2, 2, 2, 1, 0, 2, 1, 1, 0, 0], np.uint8)
+    mod2 = np.array([0, 2, 2, 1, 2, 1, 0, 2, 0, 1], np.uint8)
+    modality = np.concatenate([mod, mod2])
+    cu = np.array([0, mod.size, modality.size], np.int32)
+    cuq = np.array([0, nq, 2 * nq], np.int32)
+    k = rand_bf16(rng, (modality.size, Hkv, D))
+    q = rand_bf16(rng, (2 * nq, Hq, D), 0.3)
+    got = oracle.relevance_scores(q, k, cu, cuq, modality, Hq, Hkv, softmax_domain=oracle.SOFTMAX_CAUSAL_ROW)
+    ref = brute_scores_causal(q, k, cu, cuq, modality, Hq, Hkv)
+    np.testing.assert_allclose(got, ref, rtol=1e-12, atol=1e-15)
+    assert np.all(got[modality == 0] == 0)
+
+
+def test_causal_identical_keys_closed_form():
+    # Identical keys: every visible token has the same logit, so row r spreads its
+    # mass uniformly over the p_r + 1 tokens it sees (every modality, itself
+    # included), p_r = L - n_q + r; a token of S at position i collects
+    # (1/n_q) sum over rows with p_r >= i of 1/(p_r + 1).
+    rng = np.random.default_rng(5)
+    L, nq, Hq, Hkv = 23, 5, 4, 2
+    mod = np.zeros(L, np.uint8)
+    mod[[1, 2, 5, 8, 9, 13]] = 1
+    mod[[3, 4, 10, 11, 16]] = 2
+    mod[[19, 21]] = 2                       # inside the query span (positions 18..22)
+    k = np.repeat(rand_bf16(rng, (1, Hkv, D)), L, axis=0)
+    q = rand_bf16(rng, (nq, Hq, D))
+    cu, _ = one_seq(mod)
+    got = oracle.relevance_scores(q, k, cu, np.array([0, nq]), mod, Hq, Hkv,
+                                  softmax_domain=oracle.SOFTMAX_CAUSAL_ROW)
+    for i in range(L):
+        want = 0.0
+        if mod[i]:
+            want = sum(1.0 / (L - nq + r + 1) for r in range(nq) if L - nq + r >= i) / nq
+        assert got[i] == pytest.approx(want, rel=1e-13, abs=0.0), i
+    # the mass on the non-S tokens (system, text, query rows) is what S loses
+    assert got.sum() < 1.0
+
+
+def test_causal_domain_reduces_to_the_S_domain_when_other_keys_are_negligible():
+    # One head, one query row (the last token).  Keys outside S point against the
+    # query (logit about -40, against logits of order 1 on S), so their share is
+    # below 1e-16: the causal-row scores equal the S-domain scores, which equal
+    # scipy's softmax over S.
+    rng = np.random.default_rng(6)
+    L = 40
+    mod = np.full(L, 1, np.uint8)
+    mod[[0, 1, 2, 20, 39]] = 0
+    q = np.zeros((1, 1, D), np.float32)
+    q[0, 0, :] = rng.standard_normal(D).astype(np.float32)
+    k = rng.standard_normal((L, 1, D)).astype(np.float32) * 0.5
+    u = q[0, 0] / np.linalg.norm(q[0, 0])
+    k[mod == 0, 0, :] = -40.0 * u
+    qb, kb = bf16(q), bf16(k)
+    cu, _ = one_seq(mod)
+    causal = oracle.relevance_scores(qb, kb, cu, np.array([0, 1]), mod, 1, 1,
+                                     softmax_domain=oracle.SOFTMAX_CAUSAL_ROW)
+    mm = oracle.relevance_scores(qb, kb, cu, np.array([0, 1]), mod, 1, 1)
+    np.testing.assert_allclose(causal, mm, rtol=1e-12, atol=0)
+    S = np.nonzero(mod)[0]
+    ref = scipy.special.softmax(oracle.bf16_to_f64(kb)[S, 0, :] @ oracle.bf16_to_f64(qb)[0, 0, :] / np.sqrt(D))
+    np.testing.assert_allclose(causal[S], ref, rtol=1e-12)
