@@ -54,6 +54,16 @@ enum { APACK_MOD_OTHER = 0, APACK_MOD_AUDIO = 1, APACK_MOD_VISUAL = 2 };
    JOINT takes one top-k over all of S, the literal form of Eq. inner. */
 enum { APACK_SELECT_PER_MODALITY = 0, APACK_SELECT_JOINT = 1 };
 
+/* Softmax domain of the relevance scores (apack_seqs.softmax_domain).
+   MM: Eq. inner_score as printed, the denominator runs over the cached
+   multimodal tokens S of the sequence only.
+   CAUSAL_ROW: the denominator is the decoder's own attention row, every token
+   the query row attends to causally (system, text, audio, visual and the
+   query tokens up to and including its own position); the query rows are the
+   last n_q tokens of the sequence, row r at position len - n_q + r, and a token
+   of S that a row cannot see contributes 0 for that row. */
+enum { APACK_SOFTMAX_MM = 0, APACK_SOFTMAX_CAUSAL_ROW = 1 };
+
 /* Maximum sizes of this build. */
 #define APACK_HEAD_DIM 128
 #define APACK_MAX_SEQS 4096
@@ -71,6 +81,8 @@ typedef struct apack_seqs {
   int32_t num_q_heads;          /* Hq */
   int32_t num_kv_heads;         /* Hkv; Hq % Hkv == 0, query head h reads key head h / (Hq/Hkv) */
   int32_t head_dim;             /* D; must be APACK_HEAD_DIM */
+  int32_t softmax_domain;       /* APACK_SOFTMAX_MM (0, zero-initialised default) or
+                                   APACK_SOFTMAX_CAUSAL_ROW (needs n_q <= len per sequence) */
 } apack_seqs;
 
 /* One group of per-token planes to compact (e.g. the K cache of layers l..L-1).
@@ -108,7 +120,10 @@ apack_status apack_keep_counts(const apack_seqs *seqs, const float *keep_ratio_h
    heads and all query rows of each sequence:
      I_i = 1/(Hq * n_q) * sum_h sum_r  exp(q_{r,h}.k_{i,g(h)} / sqrt(D))
                                       / sum_{j in S} exp(q_{r,h}.k_{j,g(h)} / sqrt(D))
-   for i in S of the sequence, and I_i = 0 for tokens outside S.
+   for i in S of the sequence, and I_i = 0 for tokens outside S.  With
+   seqs->softmax_domain = APACK_SOFTMAX_CAUSAL_ROW the sum in the denominator
+   runs over every token j <= p_r (p_r = len - n_q + r, the row's position)
+   and row r adds to I_i only when i <= p_r.
    q: bf16 [sum n_q][Hq][D], contiguous (the query rows at the pruning layer).
    k: bf16 keys of the pruning layer, token t at k + t*k_token_stride, laid
       out [Hkv][D] within the row; k_token_stride a multiple of 16 bytes.

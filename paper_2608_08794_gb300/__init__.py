@@ -23,6 +23,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libapack.so")
 APACK_OK, APACK_EINVAL, APACK_ECUDA, APACK_EWORKSPACE, APACK_ETIMEOUT, APACK_EDEVICE, APACK_EUNSUPPORTED = range(7)
 APACK_MOD_OTHER, APACK_MOD_AUDIO, APACK_MOD_VISUAL = 0, 1, 2
 APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT = 0, 1
+APACK_SOFTMAX_MM, APACK_SOFTMAX_CAUSAL_ROW = 0, 1
 APACK_HEAD_DIM = 128
 
 EXPORTED = ("apack_workspace_size", "apack_keep_counts", "apack_score", "apack_select", "apack_compact",
@@ -47,7 +48,8 @@ class apack_seqs(ctypes.Structure):
                 ("modality", ctypes.c_void_p),
                 ("num_q_heads", ctypes.c_int32),
                 ("num_kv_heads", ctypes.c_int32),
-                ("head_dim", ctypes.c_int32)]
+                ("head_dim", ctypes.c_int32),
+                ("softmax_domain", ctypes.c_int32)]
 
 
 class apack_plane(ctypes.Structure):
@@ -139,7 +141,7 @@ class Seqs:
     Keeps the host arrays alive for as long as the ``apack_seqs`` struct is used."""
 
     def __init__(self, cu_seqlens, cu_qlens, n_audio, n_visual, modality, num_q_heads, num_kv_heads,
-                 head_dim=APACK_HEAD_DIM):
+                 head_dim=APACK_HEAD_DIM, softmax_domain=0):
         self.cu_seqlens = _i32(cu_seqlens)
         self.cu_qlens = _i32(cu_qlens)
         self.n_audio = _i32(n_audio)
@@ -153,7 +155,9 @@ class Seqs:
             n_audio_h=self.n_audio.ctypes.data_as(I32P),
             n_visual_h=self.n_visual.ctypes.data_as(I32P),
             modality=None if modality is None else modality.data_ptr(),
-            num_q_heads=num_q_heads, num_kv_heads=num_kv_heads, head_dim=head_dim)
+            num_q_heads=num_q_heads, num_kv_heads=num_kv_heads, head_dim=head_dim,
+            softmax_domain=int(softmax_domain))
+        self.softmax_domain = int(softmax_domain)
 
     @property
     def num_seqs(self):

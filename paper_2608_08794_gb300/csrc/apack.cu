@@ -34,10 +34,12 @@ apack_status validate_seqs(const apack_seqs *s, int64_t *total_tokens, int64_t *
   if (s->head_dim != APACK_HEAD_DIM) return APACK_EUNSUPPORTED;
   if (s->num_q_heads < 1 || s->num_kv_heads < 1 || s->num_q_heads % s->num_kv_heads != 0) return APACK_EINVAL;
   if (s->cu_seqlens_h[0] != 0 || s->cu_qlens_h[0] != 0) return APACK_EINVAL;
+  if (s->softmax_domain != APACK_SOFTMAX_MM && s->softmax_domain != APACK_SOFTMAX_CAUSAL_ROW) return APACK_EINVAL;
   for (int b = 0; b < s->num_seqs; ++b) {
     const int64_t len = static_cast<int64_t>(s->cu_seqlens_h[b + 1]) - s->cu_seqlens_h[b];
     const int64_t nq = static_cast<int64_t>(s->cu_qlens_h[b + 1]) - s->cu_qlens_h[b];
     if (len < 0 || nq < 0) return APACK_EINVAL;
+    if (s->softmax_domain == APACK_SOFTMAX_CAUSAL_ROW && nq > len) return APACK_EINVAL;   // rows are tokens
     if (s->n_audio_h[b] < 0 || s->n_visual_h[b] < 0 ||
         static_cast<int64_t>(s->n_audio_h[b]) + s->n_visual_h[b] > len)
       return APACK_EINVAL;

@@ -26,6 +26,7 @@ struct NarrowPlan {
   int32_t total_units8;
   int32_t chunk;                       // keys per CTA of the rows8 kernel (a multiple of the kernel's tile)
   int32_t hq, hkv, group;
+  int32_t causal;                      // APACK_SOFTMAX_CAUSAL_ROW: row r of n_q sees keys <= len - n_q + r
   float scale2;
   NSeq seq[kSeqsPerLaunch];
 };

@@ -69,6 +69,7 @@ struct ScorePlan {
   int32_t hq, hkv, group;
   int32_t total_qrows;     // sum n_q over the whole batch
   int32_t total_tokens;    // T
+  int32_t causal;          // APACK_SOFTMAX_CAUSAL_ROW: rows see every token up to their own position
   float scale2;            // log2(e) / sqrt(D)
   SeqPlan seq[kSeqsPerLaunch];
 };
@@ -364,13 +365,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int key = sp.t0 + w.b0 * kKeysPerBlock1 + h * 64 + c * 32 + lane;
         mod_next[c] = (active && key < t_end) ? modality[key] : 0;
       }
+      // causal rows: this lane's row (token r of the query span) sees keys up to len - n_q + r
+      const int see = sp.len - sp.n_q + (w.qp * 256 + row) / G;
       for (int b = w.b0; b < w.b1; ++b) {
-        uint32_t mask[2];
+        uint32_t mask[2], rmask[2];   // keys of the chunk (warp-uniform); and those this lane's row sees
         const int key_base = sp.t0 + b * kKeysPerBlock1 + h * 64;
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
           const int key = key_base + c * 32 + lane;
-          mask[c] = __ballot_sync(0xffffffffu, key < t_end && is_mm(mod_next[c]));
+          mask[c] = __ballot_sync(0xffffffffu, key < t_end && (plan.causal || is_mm(mod_next[c])));
+          rmask[c] = mask[c];
+          if (plan.causal) {   // keys at local index <= see
+            const int lim = see - (key_base - sp.t0 + c * 32);
+            rmask[c] &= lim >= 31 ? 0xffffffffu : (lim < 0 ? 0u : (2u << lim) - 1u);
+          }
         }
         if (active && b + 1 < w.b1) {
 #pragma unroll
@@ -388,8 +396,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->acc_empty[ci]);   // registers hold the data: release early
-          online_chunk<0>(rr, mask[0], c2, m, sum);
-          online_chunk<32>(rr, mask[1], c2, m, sum);
+          online_chunk<0>(rr, rmask[0], c2, m, sum);
+          online_chunk<32>(rr, rmask[1], c2, m, sum);
         } else {
           tc_fence_before();
           __syncwarp();
@@ -505,6 +513,16 @@ __device__ __forceinline__ void colsum_chunk(const uint32_t (&r)[64], const floa
   }
 }
 
+// The same over the columns OFF + i >= first only (causal rows that cannot see the key drop out;
+// taken only by keys inside the query span).
+template <int OFF>
+__device__ __forceinline__ void colsum_chunk_from(const uint32_t (&r)[64], const float *nl, float c2, int first,
+                                                  float2 (&a)[4]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i)
+    if (OFF + i >= first) a[i & 3].x += ex2_approx(fmaf(__uint_as_float(r[OFF + i]), c2, nl[i]));
+}
+
 // Work unit = (256-key pair, KV head group g); writes the group's sum for each
 // key to gsum[g][key]; the final kernel adds the groups.
 __global__ void __launch_bounds__(kThreads, 1)
@@ -614,6 +632,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (nch == 0) continue;
       const bool active = t < w.ntiles;
       float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+      // causal rows: only packed rows rho >= rho_min (tokens r >= key - (len - n_q)) see this key
+      const int rho_min = plan.causal ? max(0, w.kp * kKeysPerUnit2 + klane - (sp.len - sp.n_q)) * G : 0;
       for (int c = 0; c < nch; ++c) {
         if (!wait_or_abort(&bars->acc_full[ci], cph, bars, err, 26)) { ok = false; break; }
         tc_fence_after();
@@ -625,8 +645,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->acc_empty[ci]);   // registers hold the data: release early
-          colsum_chunk<0>(rr, nl, c2, a);
-          colsum_chunk<32>(rr, nl + 32, c2, a);
+          const int first = rho_min - (c * kBRows + h * 64);
+          if (first <= 0) {
+            colsum_chunk<0>(rr, nl, c2, a);
+            colsum_chunk<32>(rr, nl + 32, c2, a);
+          } else if (first < 64) {
+            colsum_chunk_from<0>(rr, nl, c2, first, a);
+            colsum_chunk_from<32>(rr, nl + 32, c2, first, a);
+          }
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->l_empty[li]);
         } else {
@@ -776,6 +802,7 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
     P.total_qrows = static_cast<int32_t>(NQ);
     P.total_tokens = static_cast<int32_t>(T);
     P.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(APACK_HEAD_DIM)));
+    P.causal = seqs->softmax_domain == APACK_SOFTMAX_CAUSAL_ROW;
     int64_t chunks = 0, qrows = 0, work = 0;
     for (int i = 0; i < ns; ++i) {
       const int b = s0 + i;

@@ -114,9 +114,11 @@ __global__ void __launch_bounds__(kThreads)
         const int rho = qoff[l] / 128;
         const float y = acc[l] * plan.scale2;
         if (in) logits[lbase + static_cast<int64_t>(rho) * sq.lstride] = y;
-        // this warp's (max, sum of exp2) of the row over its multimodal keys
-        const float wm = warp_max(mm ? y : -INFINITY);
-        const float ws = warp_sum(mm && wm != -INFINITY ? ex2_approx(y - wm) : 0.f);
+        // this warp's (max, sum of exp2) of the row over the keys in its denominator: the
+        // multimodal keys, or (causal rows) every key up to the row's own position
+        const bool use = plan.causal ? (in && key - sq.t0 <= sq.len - sq.n_q + l / G) : mm;
+        const float wm = warp_max(use ? y : -INFINITY);
+        const float ws = warp_sum(use && wm != -INFINITY ? ex2_approx(y - wm) : 0.f);
         if (lane == 0) wpart[warp * R + rho] = make_float2(wm, ws);
       }
     }
@@ -200,11 +202,14 @@ __global__ void __launch_bounds__(kThreads)
     // eight independent sums, the loads of a block of 8 rows issued together
     const float *lp = logits + sq.logit_base + (key - sq.t0);
     float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    // causal rows: logit row rho = token * Hq + head sees this key when token >= key - (len - n_q)
+    const int rho_min = plan.causal ? max(0, key - sq.t0 - (sq.len - sq.n_q)) * plan.hq : 0;
     for (int r0 = 0; r0 < R; r0 += 8) {
       float x[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u)
-        x[u] = r0 + u < R ? lp[static_cast<int64_t>(r0 + u) * sq.lstride] - ls[r0 + u] : -INFINITY;
+        x[u] = (r0 + u < R && r0 + u >= rho_min) ? lp[static_cast<int64_t>(r0 + u) * sq.lstride] - ls[r0 + u]
+                                                 : -INFINITY;
 #pragma unroll
       for (int u = 0; u < 8; ++u) a[u] += ex2_approx(x[u]);
     }
@@ -270,6 +275,7 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
     P.hkv = hkv;
     P.group = G;
     P.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(APACK_HEAD_DIM)));
+    P.causal = seqs->softmax_domain == APACK_SOFTMAX_CAUSAL_ROW;
     // tensor-core logits kernel: Hkv = 2 or 4, at most 8 rows per head group
     int max_rg = 0;
     for (int i = 0; i < ns; ++i) {

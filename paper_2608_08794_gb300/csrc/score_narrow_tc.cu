@@ -227,7 +227,8 @@ __global__ void __launch_bounds__(tc_threads<HKV>(), 1)
           const float y = __uint_as_float(r[hh * kTcN + j]) * c2;
           const int rho = (j / G) * plan.hq + h * G + j % G;
           if (valid) logits[sq.logit_base + static_cast<int64_t>(rho) * sq.lstride + key] = y;
-          if (mm) {
+          // the row's denominator: multimodal keys, or (causal rows) every key up to its position
+          if (plan.causal ? (valid && key <= sq.len - sq.n_q + j / G) : mm) {
             const float mn = fmaxf(m[hh][j], y);
             sum[hh][j] = sum[hh][j] * ex2_approx(m[hh][j] - mn) + ex2_approx(y - mn);
             m[hh][j] = mn;

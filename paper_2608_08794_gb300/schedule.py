@@ -52,7 +52,7 @@ def schedule_keep_counts(cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, n
 class ProgressivePrune:
     def __init__(self, cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, num_kv_heads, num_layers, hidden_dim,
                  prune_layers, keep_counts, device="cuda", select_mode=APACK_SELECT_PER_MODALITY,
-                 with_hidden=True, slice_below=False):
+                 with_hidden=True, slice_below=False, softmax_domain=0):
         """keep_counts[i]: int array [B, 2] of the tokens each segment keeps after step i.
 
         slice_below: also compact, at every step, the K/V of the layers below its
@@ -60,6 +60,7 @@ class ProgressivePrune:
         kept tokens (for decoding).  The caches of layers [0, l_0) are then inputs
         too (``k_low_in`` / ``v_low_in``); ``output_low_kv`` gives layers [0, l_i)."""
         self.dev = torch.device(device)
+        self.softmax_domain = int(softmax_domain)
         self.cu0 = np.asarray(cu_seqlens, np.int32)
         self.cuq = np.asarray(cu_qlens, np.int32)
         self.na0 = np.asarray(n_audio, np.int32)
@@ -120,7 +121,7 @@ class ProgressivePrune:
             cu = np.concatenate([[0], np.cumsum(other + k[:, 0] + k[:, 1])]).astype(np.int32)
             na, nv = k[:, 0], k[:, 1]
             mod = self.mod_out[(i - 1) % 2]
-        s = Seqs(cu, self.cuq, na, nv, mod, self.hq, self.hkv)
+        s = Seqs(cu, self.cuq, na, nv, mod, self.hq, self.hkv, softmax_domain=self.softmax_domain)
         self._seqs.append(s)
         return s
 

@@ -61,9 +61,9 @@ def random_batch(rng, lens, nqs, hq, hkv, p_other=0.05, scale_k=1.0, scale_q=1.0
     return mod, cu, cuq, k, q, na, nv
 
 
-def gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv):
+def gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv, softmax_domain=0):
     mod_d = dev(mod)
-    seqs = ap.Seqs(cu, cuq, na, nv, mod_d, hq, hkv)
+    seqs = ap.Seqs(cu, cuq, na, nv, mod_d, hq, hkv, softmax_domain=softmax_domain)
     ws = aligned_ws(ap, seqs)
     T = int(cu[-1])
     scores = torch.full((max(T, 1),), float("nan"), dtype=torch.float32, device="cuda")
@@ -123,6 +123,57 @@ def test_scores_match_oracle(ap, lens, nqs, hq, hkv):
         S = ((mod[cu[s]:cu[s + 1]] == 1) | (mod[cu[s]:cu[s + 1]] == 2)).sum()
         tot = got[cu[s]:cu[s + 1]].astype(np.float64).sum()
         assert tot == pytest.approx(1.0 if S and nqs[s] else 0.0, abs=1e-4)
+
+
+# ------------------------------------------------------------------------------ causal-row domain
+
+CAUSAL_SHAPES = [
+    # tensor-core passes (more than 32 rows per head group)
+    ([1000], [32], 28, 4),
+    ([300, 77, 1290], [5, 1, 40], 28, 4),
+    ([700], [64], 16, 2),
+    ([513], [40], 4, 4),
+    ([129, 257, 40], [7, 19, 2], 12, 2),
+    ([40, 600], [0, 30], 28, 4),
+    # narrow path: tensor-core logits (<= 8 rows per group, Hkv 2 / 4) and the general kernel
+    ([1000], [1], 28, 4),
+    ([3000, 700, 1, 90, 64, 65], [1, 1, 1, 0, 1, 1], 28, 4),
+    ([5000, 333], [1, 1], 16, 2),
+    ([4100], [2], 8, 4),
+    ([3000, 700, 2, 90], [1, 4, 2, 0], 28, 4),
+    ([2049], [4], 8, 1),
+]
+
+
+@pytest.mark.parametrize("query_text", [False, True])
+@pytest.mark.parametrize("lens,nqs,hq,hkv", CAUSAL_SHAPES)
+def test_causal_row_scores_match_oracle(ap, lens, nqs, hq, hkv, query_text):
+    """APACK_SOFTMAX_CAUSAL_ROW: the denominator is the query token's causal row (every
+    token up to the row's position).  query_text: the last n_q tokens (the query rows) are
+    text, as in a prompt; otherwise most of them are audio/visual tokens, which then get
+    credit only from the rows at or after their position."""
+    rng = np.random.default_rng(sum(lens) * 5 + hq + int(query_text))
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, lens, nqs, hq, hkv, scale_k=1.3)
+    if query_text:
+        for s in range(len(lens)):
+            mod[cu[s + 1] - nqs[s]:cu[s + 1]] = 0
+        na = [int((mod[cu[s]:cu[s + 1]] == 1).sum()) for s in range(len(lens))]
+        nv = [int((mod[cu[s]:cu[s + 1]] == 2).sum()) for s in range(len(lens))]
+    got = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv, softmax_domain=ap.APACK_SOFTMAX_CAUSAL_ROW)
+    ref = oracle.relevance_scores(q, k, cu, cuq, mod, hq, hkv, softmax_domain=oracle.SOFTMAX_CAUSAL_ROW)
+    check_scores(got, ref, strict_rel=2e-3)
+    mm = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv)
+    for s in range(len(lens)):      # the causal row spends mass outside S: never more than the S domain's 1
+        if nqs[s]:
+            assert got[cu[s]:cu[s + 1]].astype(np.float64).sum() <= mm[cu[s]:cu[s + 1]].astype(np.float64).sum() + 1e-4
+
+
+def test_causal_row_domain_rejects_more_rows_than_tokens(ap):
+    mod = np.full(10, 1, np.uint8)
+    seqs = ap.Seqs(np.array([0, 10], np.int32), np.array([0, 11], np.int32), [10], [0], dev(mod), 28, 4,
+                   softmax_domain=ap.APACK_SOFTMAX_CAUSAL_ROW)
+    with pytest.raises(ap.ApackError):
+        ap.apack_workspace_size(seqs)
 
 
 def test_scores_large_logits_and_sequence_without_S(ap):

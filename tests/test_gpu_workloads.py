@@ -46,8 +46,12 @@ def oracle_counts(wl):
     return out, True
 
 
-@pytest.mark.parametrize("name", ["tiny", "3b_60s", "7b_2min", "7b_10min", "7b_ragged16", "7b_10min_paper"])
-def test_workload_parity(ap, name):
+@pytest.mark.parametrize("name,domain", [(n, 0) for n in ["tiny", "3b_60s", "7b_2min", "7b_10min", "7b_ragged16",
+                                                          "7b_10min_paper"]] +
+                         [(n, 1) for n in ["tiny", "3b_60s", "7b_2min", "7b_10min_paper"]])
+def test_workload_parity(ap, name, domain):
+    """domain 1: the causal-row softmax domain (the text-query rows are the last n_q
+    tokens of every synthetic sequence)."""
     from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
     from synth import workload
     from synth.device import fill_progressive_inputs
@@ -64,7 +68,7 @@ def test_workload_parity(ap, name):
     ref_counts, joint = oracle_counts(wl)
     assert [c.tolist() for c in counts] == [[list(x) for x in r] for r in ref_counts]
     pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
-                          wl.prune_layers, counts, select_mode=mode)
+                          wl.prune_layers, counts, select_mode=mode, softmax_domain=domain)
     qs = fill_progressive_inputs(pp, wl)
 
     composite = np.arange(wl.total_tokens)
@@ -79,7 +83,8 @@ def test_workload_parity(ap, name):
         T_in, t_out = int(cu_cur[-1]), pp.t_out[i]
         # scores
         k_host = key_slab(wl, layer, qs[i])[composite]
-        ref_scores = oracle.relevance_scores(qs[i], k_host, cu_cur, cuq, mod_cur, wl.num_q_heads, wl.num_kv_heads)
+        ref_scores = oracle.relevance_scores(qs[i], k_host, cu_cur, cuq, mod_cur, wl.num_q_heads, wl.num_kv_heads,
+                                             softmax_domain=domain)
         got = pp.scores[:T_in].cpu().numpy()
         check_scores(got, ref_scores)
         # selection
@@ -113,7 +118,7 @@ def test_workload_parity(ap, name):
         cu_cur = new_cu
     tok, _ = planted_tokens(wl)
     assert np.isin(tok, composite).all(), "a planted token was dropped"
-    print(f"{name}: tie-exempt tokens {exempt_total}")
+    print(f"{name} (softmax domain {domain}): tie-exempt tokens {exempt_total}")
 
 
 def snapshot(pp):
