@@ -50,8 +50,9 @@ def parse():
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=None)
-    p.add_argument("--part", default="all", choices=["all", "decode"],
-                   help="decode: time only the decode-step attention on a synthetic cache")
+    p.add_argument("--part", default="all", choices=["all", "decode", "compact"],
+                   help="decode: time only the decode-step attention on a synthetic cache; compact: only "
+                        "the first step's compaction of the 10-minute 7B cache, out of place and in place")
     p.add_argument("--decode-tokens", type=int, default=135272)
     p.add_argument("--decode-layers", type=int, default=8)
     return p.parse_args()
@@ -528,6 +529,44 @@ def decode_only(args):
                                    "algorithmic_bytes_per_launch": alg}}))
 
 
+def compact_only(args):
+    """The first prune step's compaction of the 10-minute 7B sequence alone: K and V of layers
+    4..27 (48 planes of 135272 rows of 1024 B, 58772 kept), out of place (ping-pong buffers)
+    and in place (src == dst), through apack_compact.  Prints one JSON line."""
+    import numpy as np
+    import torch
+    import paper_2608_08794_gb300 as ap
+    T, n_keep, planes, rb = 135272, 58772, 48, 1024
+    rng = np.random.default_rng(4)
+    keep = torch.from_numpy(np.sort(rng.choice(T, n_keep, replace=False)).astype(np.int32)).cuda()
+    src = torch.empty((planes, T, rb), dtype=torch.uint8, device="cuda")
+    dst = torch.empty((planes, n_keep, rb), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    alg = 2 * n_keep * rb * planes + 4 * n_keep
+    peak, peak_kind = measured_peaks()
+    out = {}
+    for name, plane in (("out_of_place", ap.make_plane(src, dst, rb, planes, T * rb, n_keep * rb)),
+                        ("in_place", ap.make_plane(src, src, rb, planes, T * rb, T * rb))):
+        for _ in range(args.warmup):
+            ap.apack_compact(keep, n_keep, [plane], ws=ws)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(args.steps):
+            ap.apack_compact(keep, n_keep, [plane], ws=ws)
+        e1.record()
+        torch.cuda.synchronize()
+        if ap.apack_device_error(ws) != ap.APACK_OK:
+            raise RuntimeError("compaction reported a device error")
+        ms = e0.elapsed_time(e1) / args.steps
+        out[name] = {"ms": ms, "GB/s": alg / ms / 1e6, "frac": alg / ms / 1e6 / peak}
+    print(json.dumps({"metric": "compaction time of the first 10-minute 7B prune step", "unit": "ms",
+                      "higher_is_better": False, "steps": args.steps, "warmup": args.warmup,
+                      "config": {"workload": f"{planes} planes x {T} rows of {rb} B, {n_keep} kept (random)",
+                                 "l2": "inputs larger than L2 (%.1f GB)" % (planes * T * rb / 1e9)},
+                      "peak": peak, "peak_source": peak_kind, "algorithmic_bytes": alg, **out}))
+
+
 # ----------------------------------------------------------------------------- GPU leg
 
 def main():
@@ -540,6 +579,9 @@ def main():
         return
     if args.part == "decode":
         decode_only(args)
+        return
+    if args.part == "compact":
+        compact_only(args)
         return
 
     import numpy as np

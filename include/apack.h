@@ -149,10 +149,17 @@ apack_status apack_select(const apack_seqs *seqs, const float *scores, const int
 /* KV-cache and hidden-state slicing (Sec. 3.2, last sentence; Algorithm 1,
    "slice their KV-cache entries"): for every plane of every group,
    dst row j = src row keep_idx[j], j < n_out, bit for bit.
-   planes_h: host array of num_groups descriptors.  Out of place only in this
-   build (src == dst returns APACK_EUNSUPPORTED).
-   ws: NULL, or a 256-byte aligned workspace (e.g. the one of apack_score)
-   whose error word receives APACK_ETIMEOUT if a bounded wait gives up. */
+   planes_h: host array of num_groups descriptors.
+   In place: a group with src == dst (and equal plane and row strides) is
+   compacted within its own buffer.  Output row j reads row keep_idx[j] >= j,
+   so each store waits (bounded) until every load that reads the rows it
+   overwrites is done; the rows must be 16-byte multiples of at most 32 KB,
+   16-byte aligned (APACK_EUNSUPPORTED otherwise), planes must not overlap,
+   and ws is required: the launch keeps per-CTA progress words in its bytes
+   256..1023 (the workspace of apack_workspace_size has them).
+   ws: NULL (out of place only), or a 256-byte aligned workspace (e.g. the
+   one of apack_score, at least 1024 bytes) whose error word receives
+   APACK_ETIMEOUT if a bounded wait gives up. */
 apack_status apack_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes_h,
                            int32_t num_groups, void *ws, void *stream);
 
@@ -162,8 +169,11 @@ apack_status apack_compact(const int32_t *keep_idx, int64_t n_out, const apack_p
    layers [layer, num_layers), of the hidden states and of any extra planes.
    k_cache / v_cache: bf16, slab 0 = layer `layer`, slab i at
      + i*kv_layer_stride bytes, token t at + t*Hkv*D*2 bytes within a slab.
-   k_out / v_out: the same layout with kv_out_layer_stride (out of place).
-   hidden / hidden_out: bf16 [T][hidden_dim] / [T_out][hidden_dim] (hidden may be NULL).
+   k_out / v_out: the same layout with kv_out_layer_stride; k_out == k_cache
+     and v_out == v_cache with equal strides compact in place (the first T_out
+     token rows of every slab, see apack_compact).
+   hidden / hidden_out: bf16 [T][hidden_dim] / [T_out][hidden_dim] (hidden may be NULL;
+     hidden_out == hidden compacts in place).
    keep_count_h: [B][2] counts (e.g. cumulative schedules); when NULL they
    come from keep_ratio_h as in apack_keep_counts.
    new_cu_seqlens_h (host, [B+1]) receives the new offsets before the call

@@ -218,6 +218,9 @@ apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num
     return APACK_EINVAL;
   if (hidden && (!hidden_out || hidden_dim <= 0)) return APACK_EINVAL;
   if (!ws_ok(seqs, ws, ws_bytes)) return ws ? APACK_EWORKSPACE : APACK_EINVAL;
+  // in place: both caches together, with the input's slab stride (checked before any launch)
+  if ((k_out == k_cache) != (v_out == v_cache) || (k_out == k_cache && kv_out_layer_stride != kv_layer_stride))
+    return APACK_EINVAL;
   const int64_t row = static_cast<int64_t>(seqs->num_kv_heads) * APACK_HEAD_DIM * 2;
   const int32_t n_layers = num_layers - layer;
   if (n_layers > 1 && (kv_layer_stride < T * row || kv_out_layer_stride < row)) return APACK_EINVAL;

@@ -10,6 +10,15 @@
 //    CTA, so a handful of threads keep the whole HBM pipe busy.
 //  - Rows that are not 16-byte multiples (or misaligned) take the narrow
 //    kernel, one thread per row.
+//  - In place (src == dst): output row j reads row keep_idx[j] >= j, so the
+//    store of output rows [r0, r0 + n) of a plane may only start once every
+//    load of that plane that reads a row in [r0, r0 + n) is done.  Those loads
+//    belong to output rows below r0 + n: earlier items of the same plane.
+//    The in-place kernel runs two CTAs per SM (cooperative launch, so
+//    all are resident), items round-robin as in the out-of-place kernel; each
+//    CTA publishes how many of its items' loads are complete, and waits
+//    (bounded) for the owners of those earlier items before each store.
+//    Loads never wait on stores of later items, so the waits always end.
 #include "internal.cuh"
 #include "ptx.cuh"
 
@@ -31,6 +40,8 @@ struct TmaGroup {
   uint32_t chunks_per_plane;    // ceil(n_out / rows_per_slot)
   uint32_t item_begin;          // first slot-sized item of this group
   uint32_t contiguous;          // output rows are back to back (one bulk store per slot)
+  uint32_t chunk_major;         // items ordered (chunk, plane) instead of (plane, chunk): in place
+  uint32_t num_planes;
   uint32_t pad;
 };
 
@@ -38,6 +49,7 @@ struct TmaPlan {
   int32_t ngroups;
   uint32_t total_items;
   uint32_t n_out;
+  uint32_t dep_period;          // in place: owners of a plane's items repeat after this many chunks
   TmaGroup g[kMaxGroups];
 };
 
@@ -53,8 +65,15 @@ __device__ __forceinline__ Item decode_item(const TmaPlan &p, uint32_t item) {
   const uint32_t local = item - G.item_begin;
   Item it;
   it.grp = &G;
-  it.plane = local / G.chunks_per_plane;
-  it.r0 = (local - it.plane * G.chunks_per_plane) * G.rows_per_slot;
+  uint32_t chunk;
+  if (G.chunk_major) {
+    chunk = local / G.num_planes;
+    it.plane = local - chunk * G.num_planes;
+  } else {
+    it.plane = local / G.chunks_per_plane;
+    chunk = local - it.plane * G.chunks_per_plane;
+  }
+  it.r0 = chunk * G.rows_per_slot;
   it.nrows = min(G.rows_per_slot, p.n_out - it.r0);
   return it;
 }
@@ -97,7 +116,8 @@ __global__ void __launch_bounds__(32) gather_tma_kernel(const __grid_constant__ 
   // this CTA's items: blockIdx.x, blockIdx.x + gridDim.x, ...
   const uint32_t first = blockIdx.x, stride = gridDim.x;
   const uint32_t n_mine = first < plan.total_items ? (plan.total_items - first + stride - 1) / stride : 0;
-  for (uint32_t j = 0; j < n_mine && j < kSlots; ++j)
+  uint32_t issued = n_mine < kSlots ? n_mine : kSlots;   // positions whose loads were issued
+  for (uint32_t j = 0; j < issued; ++j)
     load_item(decode_item(plan, first + j * stride), slots + j * kSlotBytes, &full[j], keep_idx, lane);
   bool ok = true;
   uint32_t j = 0;
@@ -117,11 +137,180 @@ __global__ void __launch_bounds__(32) gather_tma_kernel(const __grid_constant__ 
       const uint32_t k = j - 1 + kSlots;
       const int ks = k % kSlots;
       load_item(decode_item(plan, first + k * stride), slots + ks * kSlotBytes, &full[ks], keep_idx, lane);
+      issued = k + 1;
     }
   }
   if (!ok) {
-    // loads of items j .. j+kSlots-1 may still be in flight: wait for them (bounded)
-    for (uint32_t k = j; k < n_mine && k < j + kSlots; ++k) mbar_wait(&full[k % kSlots], (k / kSlots) & 1u, kWaitLimitNs / 4);
+    // loads of items j .. issued - 1 may still be in flight: wait for them (bounded)
+    for (uint32_t k = j; k < issued; ++k) mbar_wait(&full[k % kSlots], (k / kSlots) & 1u, kWaitLimitNs / 4);
+  }
+  bulk_wait_all();
+}
+
+// ------------------------------------------------------------------ in place
+constexpr int kInSlots = 3;                      // two CTAs per SM, 3 slots of 32 KB each
+constexpr uint32_t kInSmem = kInSlots * kSlotBytes;
+constexpr int kMaxInCtas = 384;                  // 16-bit progress words at ws + 256 .. ws + 1024
+constexpr int kInChecks = 384;                   // progress words one dependency check may read
+constexpr size_t kProgressOff = 256;
+
+// Progress words.  A word is written after the CTA has observed its loads complete (the rows are
+// already in shared memory, so no later write can change what they read), and a reader only
+// issues its store after the loop that reads the word has seen the value it needs: relaxed
+// gpu-scope accesses carry all the ordering the stores need.
+__device__ __forceinline__ uint32_t ld_progress(const uint16_t *p) {
+  uint16_t v;
+  asm volatile("ld.relaxed.gpu.global.u16 %0, [%1];" : "=h"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_progress(uint16_t *p, uint32_t v) {
+  asm volatile("st.relaxed.gpu.global.u16 [%0], %1;" ::"l"(p), "h"(static_cast<uint16_t>(v)) : "memory");
+}
+
+// First index j >= lo with a[j] >= x (n if none); a ascending and a[lo - 1] < x (or lo == 0).
+// The warp gallops (lane l probes lo + 2^l - 1), then probes 32 evenly spaced rows of the bracket
+// per round: two rounds when the answer is near lo, as it is for successive chunks of a CTA.
+__device__ __forceinline__ uint32_t warp_lower_bound(const int32_t *__restrict__ a, uint32_t n, uint32_t lo,
+                                                     int64_t x, int lane) {
+  if (lo >= n) return n;
+  uint32_t hi = n;
+  {
+    const uint64_t p = static_cast<uint64_t>(lo) + (1ull << lane) - 1;
+    const bool valid = p < n;
+    const uint32_t vm = __ballot_sync(0xffffffffu, valid);
+    const uint32_t b = __ballot_sync(0xffffffffu, valid && a[p] >= x);
+    if (b) {
+      const int f = __ffs(b) - 1;
+      hi = lo + (1u << f) - 1;                              // a[hi] >= x
+      if (f > 0) lo += 1u << (f - 1);                       // a[lo - 1] < x
+    } else {
+      lo += 1u << (31 - __clz(vm));                         // past the last probe inside [lo, n)
+    }
+  }
+  while (hi > lo) {                                         // a[lo - 1] < x <= a[hi] (or hi == n)
+    const uint32_t span = hi - lo;
+    const uint32_t step = (span + 31) / 32;
+    const uint32_t p = lo + lane * step;
+    const uint32_t b = __ballot_sync(0xffffffffu, p < hi && a[p] >= x);
+    if (b) {
+      const int f = __ffs(b) - 1;
+      hi = lo + f * step;
+      if (f > 0) lo += (f - 1) * step + 1;
+    } else {
+      lo += ((span - 1) / step) * step + 1;                 // past the last probe inside [lo, hi)
+    }
+  }
+  return hi;
+}
+
+__global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constant__ TmaPlan plan,
+                                                            const int32_t *__restrict__ keep_idx,
+                                                            uint16_t *progress, DeviceError *err) {
+  extern __shared__ __align__(1024) uint8_t slots[];
+  __shared__ __align__(8) uint64_t full[kInSlots];
+  __shared__ uint16_t seen[kMaxInCtas];          // last progress read of every CTA
+  const int lane = threadIdx.x;
+  if (lane == 0) {
+    for (int i = 0; i < kInSlots; ++i) mbar_init(&full[i], 1);
+    fence_mbar_init();
+  }
+  for (int i = lane; i < kMaxInCtas; i += 32) seen[i] = 0;
+  __syncwarp();
+  const uint32_t me = blockIdx.x, P = gridDim.x;
+  const uint32_t n_mine = me < plan.total_items ? (plan.total_items - me + P - 1) / P : 0;
+  uint32_t issued = n_mine < kInSlots ? n_mine : kInSlots;   // positions whose loads were issued
+  for (uint32_t j = 0; j < issued; ++j)
+    load_item(decode_item(plan, me + j * P), slots + j * kSlotBytes, &full[j], keep_idx, lane);
+  bool ok = true;
+  uint32_t waited = 0;                                        // positions whose loads were observed
+  uint32_t hint_row = 0;                                      // search hint: previous answer (same group)
+  int64_t hint_limit = 0;
+  for (uint32_t j = 0; ok && j < n_mine; ++j) {
+    const int slot = j % kInSlots;
+    const uint32_t item = me + j * P;
+    const Item it = decode_item(plan, item);
+    if (j >= waited && !mbar_wait(&full[slot], (j / kInSlots) & 1u, kWaitLimitNs)) {
+      if (lane == 0 && err) raise_device_error(err, APACK_ETIMEOUT, 42);
+      ok = false;
+      break;
+    }
+    // publish as far as the loads are complete: this item, and the next ones already landed
+    if (j >= waited) {
+      uint32_t w = j + 1;
+      if (lane == 0) {
+        while (w < issued && mbar_try_wait(&full[w % kInSlots], (w / kInSlots) & 1u)) ++w;
+        st_progress(progress + me, w);
+      }
+      waited = __shfl_sync(0xffffffffu, w, 0);              // the same count in every lane
+    }
+    // items of this plane whose loads read rows [r0, r0 + n) hold the output rows whose source is
+    // below r0 + n: chunks <= c_hi, the chunk of the last such row (far behind c once rows are
+    // dropped, so these waits are mostly met already).  Those are items item - k * num_planes,
+    // k >= c - c_hi; their owners repeat with period P / gcd(num_planes, P) in k and an owner's
+    // progress is monotonic, so the first period covers them all (at most kInChecks words).
+    const TmaGroup &G = *it.grp;
+    const uint32_t c = it.r0 / G.rows_per_slot;
+    const int64_t limit = static_cast<int64_t>(it.r0) + it.nrows;
+    if (limit < hint_limit) hint_row = 0;                 // a new group: the search starts over
+    hint_row = warp_lower_bound(keep_idx, plan.n_out, hint_row, limit, lane);
+    hint_limit = limit;
+    uint32_t kmin = 1, kmax = 0;                          // no dependency unless some row reads below limit
+    if (hint_row > 0) {
+      const uint32_t c_hi = (hint_row - 1) / G.rows_per_slot;
+      kmin = c > c_hi ? c - c_hi : 1;
+      kmax = min(c, kmin + plan.dep_period - 1);
+    }
+    uint32_t owner[kInChecks / 32], need[kInChecks / 32];
+#pragma unroll
+    for (int u = 0; u < kInChecks / 32; ++u) {
+      const uint32_t k = kmin + lane + 32 * u;
+      owner[u] = me;                                      // no check: my own items are waited in order
+      need[u] = 0;
+      if (k <= kmax) {
+        const uint32_t other = item - k * G.num_planes;
+        owner[u] = other % P;
+        need[u] = other / P + 1;
+      }
+    }
+    // each lane owns distinct owners (k differ by less than the period), so the cache needs no sync
+    bool mine_ok = true;
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+      bool all = true;
+#pragma unroll
+      for (int u = 0; u < kInChecks / 32; ++u) {
+        if (owner[u] != me && seen[owner[u]] < need[u]) {
+          const uint32_t v = ld_progress(progress + owner[u]);
+          seen[owner[u]] = v;
+          all &= v >= need[u];
+        }
+      }
+      if (__all_sync(0xffffffffu, all)) break;
+      if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > kWaitLimitNs)) {   // the warp gives up together
+        mine_ok = false;
+        break;
+      }
+    }
+    if (!__all_sync(0xffffffffu, mine_ok)) {
+      if (lane == 0 && err) raise_device_error(err, APACK_ETIMEOUT, 43);
+      ok = false;
+      break;
+    }
+    asm volatile("fence.proxy.async.global;" ::: "memory");   // the observed loads before the bulk store
+    fence_proxy_async_smem();
+    store_item(it, slots + slot * kSlotBytes, lane);
+    if (j >= 1 && j - 1 + kInSlots < n_mine) {
+      bulk_wait_read<1>();
+      const uint32_t k = j - 1 + kInSlots;
+      const int ks = k % kInSlots;
+      load_item(decode_item(plan, me + k * P), slots + ks * kSlotBytes, &full[ks], keep_idx, lane);
+      issued = k + 1;
+    }
+  }
+  if (!ok) {
+    // loads issued but not observed may still be in flight: wait for them (bounded)
+    for (uint32_t k = waited; k < issued; ++k) mbar_wait(&full[k % kInSlots], (k / kInSlots) & 1u, kWaitLimitNs / 4);
   }
   bulk_wait_all();
 }
@@ -183,9 +372,9 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
   if (n_out == 0 || num_groups == 0) return APACK_OK;
   if (!keep_idx || n_out > INT32_MAX) return APACK_EINVAL;
   // validate and plan every group before anything touches the device
-  TmaPlan tp{};
-  tp.n_out = static_cast<uint32_t>(n_out);
-  uint64_t items = 0;
+  TmaPlan tp{}, ip{};           // out-of-place groups, in-place groups
+  tp.n_out = ip.n_out = static_cast<uint32_t>(n_out);
+  uint64_t items = 0, in_items = 0;
   int narrow[kMaxGroups * 4];
   int n_narrow = 0;
   for (int i = 0; i < num_groups; ++i) {
@@ -195,11 +384,20 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
     if (!p.src || !p.dst || p.src_row_stride < p.row_bytes || p.dst_row_stride < p.row_bytes ||
         p.src_plane_stride < 0 || p.dst_plane_stride < 0)
       return APACK_EINVAL;
-    if (p.src == p.dst) return APACK_EUNSUPPORTED;   // in-place compaction is not offered by this build
-    if (ranges_overlap(p, n_out, n_out)) return APACK_EINVAL;
-    if (widest_unit(p) == 16 && p.row_bytes <= static_cast<int64_t>(kSlotBytes)) {
-      if (tp.ngroups == kMaxGroups) return APACK_EINVAL;
-      TmaGroup &g = tp.g[tp.ngroups++];
+    const bool tma_rows = widest_unit(p) == 16 && p.row_bytes <= static_cast<int64_t>(kSlotBytes);
+    if (p.src == p.dst) {
+      // in place: same layout on both sides, vector rows, and the progress words of the workspace
+      if (p.src_plane_stride != p.dst_plane_stride || p.src_row_stride != p.dst_row_stride) return APACK_EINVAL;
+      if (!tma_rows) return APACK_EUNSUPPORTED;
+      if (!err) return APACK_EINVAL;
+    } else if (ranges_overlap(p, n_out, n_out)) {
+      return APACK_EINVAL;
+    }
+    if (tma_rows) {
+      TmaPlan &pl = p.src == p.dst ? ip : tp;
+      uint64_t &cnt = p.src == p.dst ? in_items : items;
+      if (pl.ngroups == kMaxGroups) return APACK_EINVAL;
+      TmaGroup &g = pl.g[pl.ngroups++];
       g.src = static_cast<const uint8_t *>(p.src);
       g.dst = static_cast<uint8_t *>(p.dst);
       g.sps = p.src_plane_stride;
@@ -209,10 +407,12 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
       g.row_bytes = static_cast<uint32_t>(p.row_bytes);
       g.rows_per_slot = kSlotBytes / g.row_bytes;
       g.chunks_per_plane = static_cast<uint32_t>((n_out + g.rows_per_slot - 1) / g.rows_per_slot);
-      g.item_begin = static_cast<uint32_t>(items);
+      g.item_begin = static_cast<uint32_t>(cnt);
       g.contiguous = p.dst_row_stride == p.row_bytes;
-      items += static_cast<uint64_t>(g.chunks_per_plane) * p.num_planes;
-      if (items > 0x7FFFFFFFull) return APACK_EINVAL;
+      g.chunk_major = p.src == p.dst;
+      g.num_planes = static_cast<uint32_t>(p.num_planes);
+      cnt += static_cast<uint64_t>(g.chunks_per_plane) * p.num_planes;
+      if (cnt > 0x7FFFFFFFull) return APACK_EINVAL;
     } else {
       if (n_narrow == kMaxGroups * 4) return APACK_EINVAL;
       narrow[n_narrow++] = i;
@@ -242,6 +442,41 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
     gather_tma_kernel<<<static_cast<unsigned>(blocks), 32, kTmaSmem, stream>>>(tp, keep_idx, err);
     count_launches(1);
     if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+  }
+  if (ip.ngroups > 0) {
+    static bool in_attr_done = false;
+    if (!in_attr_done) {
+      if (check_cuda(cudaFuncSetAttribute(gather_inplace_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          kInSmem)) != APACK_OK)
+        return APACK_ECUDA;
+      in_attr_done = true;
+    }
+    ip.total_items = static_cast<uint32_t>(in_items);
+    uint64_t blocks = static_cast<uint64_t>(device_sm_count()) * 2;   // two CTAs per SM, all resident
+    if (blocks > kMaxInCtas) blocks = kMaxInCtas;
+    if (blocks > in_items) blocks = in_items;
+    if (in_items > blocks * 65535) return APACK_EUNSUPPORTED;           // 16-bit progress words
+    // the dependency check covers P / gcd(num_planes, P) chunks of every group (at most P <= kInChecks)
+    uint32_t period = 1;
+    for (int gi = 0; gi < ip.ngroups; ++gi) {
+      uint32_t a = ip.g[gi].num_planes, b = static_cast<uint32_t>(blocks);
+      while (b) {
+        const uint32_t t = a % b;
+        a = b;
+        b = t;
+      }
+      const uint32_t per = static_cast<uint32_t>(blocks) / a;
+      if (per > period) period = per;
+    }
+    ip.dep_period = period;
+    uint16_t *progress = reinterpret_cast<uint16_t *>(reinterpret_cast<uint8_t *>(err) + kProgressOff);
+    if (check_cuda(cudaMemsetAsync(progress, 0, blocks * sizeof(uint16_t), stream)) != APACK_OK) return APACK_ECUDA;
+    void *args[] = {&ip, const_cast<int32_t **>(&keep_idx), &progress, &err};
+    if (check_cuda(cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(gather_inplace_kernel),
+                                               dim3(static_cast<unsigned>(blocks)), dim3(32), args, kInSmem,
+                                               stream)) != APACK_OK)
+      return APACK_ECUDA;
+    count_launches(1);
   }
   return APACK_OK;
 }

@@ -105,6 +105,9 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
     const int64_t n_out = sp.new_cu_seqlens_h[B];
     const int32_t n_layers = num_layers - sp.layer;
     if (n_layers > 1 && (p.kv_layer_stride < Ti * row || sp.kv_out_layer_stride < n_out * row)) return APACK_EINVAL;
+    // in place: both caches together, with the input's slab stride
+    if ((sp.k_out == p.k) != (sp.v_out == p.v) || (sp.k_out == p.k && sp.kv_out_layer_stride != p.kv_layer_stride))
+      return APACK_EINVAL;
   }
 
   cudaStream_t M = static_cast<cudaStream_t>(stream);

@@ -320,6 +320,130 @@ def test_compact_many_groups_and_strided_rows(ap):
         np.testing.assert_array_equal(d.cpu().numpy(), r)
 
 
+IN_PLACE_CASES = [
+    # T, kept, row bytes, planes, which rows are kept
+    (3001, 1237, 1024, 3, "random"),
+    (3001, 3001, 1024, 2, "all"),             # every row stays where it is
+    (5000, 1, 512, 2, "last"),                # one row moves from the end to row 0
+    (20000, 7000, 7168, 1, "random"),         # hidden-state rows, 4 per 32 KB slot
+    (40000, 30000, 2048, 3, "tail"),          # a few early rows, then the whole tail: long dependency ranges
+    (135272, 58772, 1024, 4, "random"),       # the 10-minute 7B step: thousands of items on every CTA
+]
+
+
+@pytest.mark.parametrize("T,n_keep,row_bytes,planes,pattern", IN_PLACE_CASES)
+def test_compact_in_place_is_bitexact(ap, T, n_keep, row_bytes, planes, pattern):
+    """src == dst: the first n_keep rows of every plane become the kept rows (oracle
+    compact_rows), the rows after them are left as they were."""
+    rng = np.random.default_rng(T + row_bytes + planes)
+    src = rng.integers(0, 256, (planes, T, row_bytes), dtype=np.uint8)
+    if pattern == "all":
+        keep = np.arange(T, dtype=np.int32)
+    elif pattern == "last":
+        keep = np.array([T - 1], np.int32)
+    elif pattern == "tail":
+        head = np.sort(rng.choice(T // 2, n_keep - (T - T // 2), replace=False))
+        keep = np.concatenate([head, np.arange(T // 2, T)]).astype(np.int32)
+    else:
+        keep = np.sort(rng.choice(T, n_keep, replace=False)).astype(np.int32)
+    assert keep.size == n_keep
+    buf = dev(src)
+    ws = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    p = ap.make_plane(buf, buf, row_bytes, planes, src_plane_stride=T * row_bytes, dst_plane_stride=T * row_bytes)
+    ap.apack_compact(dev(keep), n_keep, [p], ws=ws)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(ws) == ap.APACK_OK
+    got = buf.cpu().numpy()
+    for pl in range(planes):
+        np.testing.assert_array_equal(got[pl, :n_keep], oracle.compact_rows(src[pl], keep))
+        np.testing.assert_array_equal(got[pl, n_keep:], src[pl, n_keep:])
+    # twice in a row on the same workspace: the progress words start from zero again
+    buf2 = dev(src)
+    p2 = ap.make_plane(buf2, buf2, row_bytes, planes, src_plane_stride=T * row_bytes,
+                       dst_plane_stride=T * row_bytes)
+    ap.apack_compact(dev(keep), n_keep, [p2], ws=ws)
+    torch.cuda.synchronize()
+    assert torch.equal(buf2, buf)
+
+
+def test_compact_in_place_mixed_with_out_of_place_groups(ap):
+    rng = np.random.default_rng(31)
+    T, rb = 9000, 1024
+    keep = np.sort(rng.choice(T, 4100, replace=False)).astype(np.int32)
+    a = rng.integers(0, 256, (2, T, rb), dtype=np.uint8)
+    b = rng.integers(0, 256, (T, 3584 * 2), dtype=np.uint8)
+    ad, bd = dev(a), dev(b)
+    bo = torch.zeros((keep.size, 3584 * 2), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    groups = [ap.make_plane(ad, ad, rb, 2, src_plane_stride=T * rb, dst_plane_stride=T * rb),
+              ap.make_plane(bd, bo, 3584 * 2, 1)]
+    ap.apack_compact(dev(keep), keep.size, groups, ws=ws)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(ws) == ap.APACK_OK
+    np.testing.assert_array_equal(ad.cpu().numpy()[:, :keep.size], a[:, keep])
+    np.testing.assert_array_equal(bo.cpu().numpy(), b[keep])
+
+
+def test_compact_in_place_argument_checks(ap):
+    T = 100
+    keep = dev(np.arange(0, T, 2, dtype=np.int32))
+    ws = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    buf = torch.zeros((2, T, 40), dtype=torch.uint8, device="cuda")
+    with pytest.raises(ap.ApackError):      # rows that are not 16-byte multiples
+        ap.apack_compact(keep, T // 2, [ap.make_plane(buf, buf, 40, 2, T * 40, T * 40)], ws=ws)
+    buf = torch.zeros((2, T, 64), dtype=torch.uint8, device="cuda")
+    with pytest.raises(ap.ApackError):      # no workspace for the progress words
+        ap.apack_compact(keep, T // 2, [ap.make_plane(buf, buf, 64, 2, T * 64, T * 64)])
+    with pytest.raises(ap.ApackError):      # different layouts on the two sides of one buffer
+        ap.apack_compact(keep, T // 2, [ap.make_plane(buf, buf, 64, 2, T * 64, (T // 2) * 64)], ws=ws)
+
+
+def test_prune_step_in_place_equals_out_of_place(ap):
+    rng = np.random.default_rng(44)
+    hq, hkv, L, layer, H = 28, 4, 6, 2, 3584
+    lens, nqs = [3000, 1500], [40, 3]
+    mod, cu, cuq, k0, q, na, nv = random_batch(rng, lens, nqs, hq, hkv)
+    T = int(cu[-1])
+    nl = L - layer
+    row = hkv * D
+    kc = torch.from_numpy(rng.integers(-30000, 30000, (nl, T, row), dtype=np.int16)).cuda()
+    kc[0] = dev(k0).view(T, row)
+    vc = torch.from_numpy(rng.integers(-30000, 30000, (nl, T, row), dtype=np.int16)).cuda()
+    hid = torch.from_numpy(rng.integers(-30000, 30000, (T, H), dtype=np.int16)).cuda()
+    counts = np.array([[na[0] // 2, nv[0] // 3], [na[1] // 4, nv[1] // 2]], np.int32)
+    mod_d = dev(mod)
+    seqs = ap.Seqs(cu, cuq, na, nv, mod_d, hq, hkv)
+    ws = aligned_ws(ap, seqs)
+    n_out = int(T - sum(na) - sum(nv) + counts.sum())
+
+    def outs():
+        return (torch.empty(max(n_out, 1), dtype=torch.int32, device="cuda"),
+                torch.empty(max(n_out, 1), dtype=torch.uint8, device="cuda"),
+                torch.empty(T, dtype=torch.float32, device="cuda"))
+
+    keep1, mo1, sc1 = outs()
+    ko = torch.empty((nl, n_out, row), dtype=torch.int16, device="cuda")
+    vo = torch.empty_like(ko)
+    ho = torch.empty((n_out, H), dtype=torch.int16, device="cuda")
+    cu1 = ap.apack_prune_step(seqs, layer, L, dev(q), kc, vc, T * row * 2, hid, H, keep_count=counts,
+                              k_out=ko, v_out=vo, kv_out_layer_stride=n_out * row * 2, hidden_out=ho,
+                              modality_out=mo1, keep_idx=keep1, scores=sc1, ws=ws)
+    keep2, mo2, sc2 = outs()
+    kc2, vc2, hid2 = kc.clone(), vc.clone(), hid.clone()
+    cu2 = ap.apack_prune_step(seqs, layer, L, dev(q), kc2, vc2, T * row * 2, hid2, H, keep_count=counts,
+                              k_out=kc2, v_out=vc2, kv_out_layer_stride=T * row * 2, hidden_out=hid2,
+                              modality_out=mo2, keep_idx=keep2, scores=sc2, ws=ws)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(ws) == ap.APACK_OK
+    np.testing.assert_array_equal(cu1, cu2)
+    assert torch.equal(keep1[:n_out], keep2[:n_out]) and torch.equal(mo1[:n_out], mo2[:n_out])
+    assert torch.equal(kc2[:, :n_out], ko) and torch.equal(vc2[:, :n_out], vo) and torch.equal(hid2[:n_out], ho)
+    with pytest.raises(ap.ApackError):      # in place needs both caches in place, at the input's slab stride
+        ap.apack_prune_step(seqs, layer, L, dev(q), kc2, vc2, T * row * 2, hid2, H, keep_count=counts,
+                            k_out=kc2, v_out=vo, kv_out_layer_stride=T * row * 2, hidden_out=hid2,
+                            modality_out=mo2, keep_idx=keep2, scores=sc2, ws=ws)
+
+
 def test_device_fill_matches_host_generator(ap):
     from synth.device import fill_normal_bf16
     from synth.gen import normal_bf16_bits
