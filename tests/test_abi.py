@@ -109,10 +109,16 @@ def test_calls_reject_bad_arguments_before_the_device(ap):
     with pytest.raises(ap.ApackError) as e:
         ap.apack_select(s, ws_small, np.array([[11, 0], [0, 0]]), ws_small, ws, stream=0)
     assert e.value.status == ap.APACK_EINVAL
-    # in-place compaction is refused
+    # in-place compaction: needs the workspace's progress words, vector rows and one layout
     t = torch.zeros(4096, dtype=torch.uint8)
     p = ap.make_plane(t, t, 256)
     with pytest.raises(ap.ApackError) as e:
         ap.apack_compact(t, 4, [p], stream=0)
+    assert e.value.status == ap.APACK_EINVAL
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_compact(t, 4, [ap.make_plane(t, t, 40)], ws=ws, stream=0)
     assert e.value.status == ap.APACK_EUNSUPPORTED
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_compact(t, 4, [ap.make_plane(t, t, 256, 2, 1024, 512)], ws=ws, stream=0)
+    assert e.value.status == ap.APACK_EINVAL
     assert ap.status_string(ap.APACK_ETIMEOUT) == "device wait timed out"
