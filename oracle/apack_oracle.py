@@ -27,8 +27,8 @@ loop; Table S-hparams "Query score"):
    layers, hidden states, metadata) is copied so that output row j is input
    row keep_idx[j].
 
-A second softmax domain is offered as a reading of the north star's "full
-key row": the denominator of Eq. (inner_score) then runs over the decoder's
+A second softmax domain reads "the full key row" as the decoder's own
+attention row: the denominator of Eq. (inner_score) then runs over the
 causal attention row of the query token, i.e. every token at or before the
 query row's position (system, text, audio, visual and query tokens), with the
 query rows taken as the last n_q tokens of the sequence; a token of S after a
