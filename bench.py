@@ -407,12 +407,15 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
 
 def scoring_roofline(wl, pp, cuq, score_ms_per_step):
     """Useful tensor work of the scoring stage: one Q K^T over the multimodal keys per
-    step (2 n_q Hq |S| D flop).  The two-pass softmax computes Q K^T twice and every
+    step and sequence (2 n_q Hq |S| D flop, summed over the sequences of the batch).  The two-pass softmax computes Q K^T twice and every
     logit also needs one exp2 per pass (the SFU is the second ceiling), so this
     fraction understates how busy the tensor pipe is."""
     import numpy as np
-    nq = int(cuq[-1])
-    flops = [2.0 * nq * wl.num_q_heads * s * wl.head_dim for s in pp.mm_tokens_per_step()]
+    nq = np.diff(np.asarray(cuq, np.int64))                   # query rows per sequence
+    # |S| per sequence entering each step: the original counts, then the previous step's kept counts
+    s_seq = [np.asarray(pp.na0, np.int64) + np.asarray(pp.nv0, np.int64)]
+    s_seq += [np.asarray(c, np.int64).reshape(len(nq), 2).sum(axis=1) for c in pp.counts[:-1]]
+    flops = [2.0 * wl.num_q_heads * wl.head_dim * float((nq * sq).sum()) for sq in s_seq]
     ms = float(np.sum(score_ms_per_step))
     achieved = sum(flops) / (ms / 1e3) / 1e12
     peak, kind = measured_tensor_peak()
