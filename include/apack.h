@@ -128,7 +128,8 @@ apack_status apack_keep_counts(const apack_seqs *seqs, const float *keep_ratio_h
    k: bf16 keys of the pruning layer, token t at k + t*k_token_stride, laid
       out [Hkv][D] within the row; k_token_stride a multiple of 16 bytes.
    scores: fp32 [T].  Computed in fp32 from bf16 products on the tensor
-   cores; deterministic (fixed reduction order, no atomics). */
+   cores; deterministic (fixed reduction order, no atomics).  q and k must be
+   device memory (they are read by TMA; host memory gives APACK_EINVAL). */
 apack_status apack_score(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
                          float *scores, void *ws, size_t ws_bytes, void *stream);
 
@@ -157,6 +158,10 @@ apack_status apack_select(const apack_seqs *seqs, const float *scores, const int
    16-byte aligned (APACK_EUNSUPPORTED otherwise), planes must not overlap,
    and ws is required: the launch keeps per-CTA progress words in its bytes
    256..1023 (the workspace of apack_workspace_size has them).
+   Host source: a group whose src is pinned host memory (cudaHostAlloc or
+   cudaHostRegister) is gathered over the host link by plain loads (zero
+   copy): only the kept rows cross the link.  Its dst must be device memory,
+   and it cannot be in place (APACK_EINVAL).
    ws: NULL (out of place only), or a 256-byte aligned workspace (e.g. the
    one of apack_score, at least 1024 bytes) whose error word receives
    APACK_ETIMEOUT if a bounded wait gives up. */

@@ -18,6 +18,16 @@ void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_rela
 
 apack_status check_cuda(cudaError_t e) { return e == cudaSuccess ? APACK_OK : APACK_ECUDA; }
 
+bool in_host_memory(const void *p) {
+  if (!p) return false;
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeHost;
+}
+
 int device_sm_count() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
@@ -181,6 +191,7 @@ apack_status apack_score(const apack_seqs *seqs, const void *q, const void *k, i
   const apack_status st = validate_seqs(seqs, &T, &NQ);
   if (st != APACK_OK) return st;
   if (!ws_ok(seqs, ws, ws_bytes)) return ws ? APACK_EWORKSPACE : APACK_EINVAL;
+  if (in_host_memory(k) || in_host_memory(q)) return APACK_EINVAL;   // read by TMA: device memory only
   return run_score(seqs, q, k, k_token_stride, scores, ws, static_cast<cudaStream_t>(stream));
 }
 
@@ -218,6 +229,7 @@ apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num
     return APACK_EINVAL;
   if (hidden && (!hidden_out || hidden_dim <= 0)) return APACK_EINVAL;
   if (!ws_ok(seqs, ws, ws_bytes)) return ws ? APACK_EWORKSPACE : APACK_EINVAL;
+  if (in_host_memory(k_cache) || in_host_memory(q)) return APACK_EINVAL;   // scored by TMA: device memory
   // in place: both caches together, with the input's slab stride (checked before any launch)
   if ((k_out == k_cache) != (v_out == v_cache) || (k_out == k_cache && kv_out_layer_stride != kv_layer_stride))
     return APACK_EINVAL;

@@ -315,6 +315,53 @@ __global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constan
   bulk_wait_all();
 }
 
+// ------------------------------------------------------------------ host source
+// Source rows in pinned host memory (zero copy): only the kept rows cross the host link.
+// Consecutive threads take consecutive 16-byte pieces of a row (coalesced link reads); each
+// thread issues U loads before its U stores so that enough reads are in flight.
+constexpr int kHostUnroll = 4;
+
+__global__ void __launch_bounds__(256) gather_host_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst,
+                                                          int64_t sps, int64_t dps, int64_t srs, int64_t drs,
+                                                          int64_t row_bytes, int64_t n_planes, int64_t n_out,
+                                                          const int32_t *__restrict__ keep_idx) {
+  const int64_t vec_per_row = row_bytes / 16;
+  const int64_t total = n_planes * n_out * vec_per_row;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t base = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; base < total;
+       base += stride * kHostUnroll) {
+    uint4 v[kHostUnroll];
+#pragma unroll
+    for (int u = 0; u < kHostUnroll; ++u) {
+      const int64_t e = base + u * stride;
+      if (e < total) {
+        const int64_t row = e / vec_per_row, c = e - row * vec_per_row;
+        const int64_t plane = row / n_out, j = row - plane * n_out;
+        v[u] = *reinterpret_cast<const uint4 *>(src + plane * sps + static_cast<int64_t>(keep_idx[j]) * srs + c * 16);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kHostUnroll; ++u) {
+      const int64_t e = base + u * stride;
+      if (e < total) {
+        const int64_t row = e / vec_per_row, c = e - row * vec_per_row;
+        const int64_t plane = row / n_out, j = row - plane * n_out;
+        *reinterpret_cast<uint4 *>(dst + plane * dps + j * drs + c * 16) = v[u];
+      }
+    }
+  }
+}
+
+// Device address of a pinned host buffer, or nullptr when src is not host memory.
+const void *host_source(const void *src) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, src) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return at.type == cudaMemoryTypeHost ? at.devicePointer : nullptr;
+}
+
 // One thread per (plane, row); copies with the widest access the row allows.
 __global__ void gather_narrow_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst, int64_t sps,
                                      int64_t dps, int64_t srs, int64_t drs, int64_t row_bytes, int unit,
@@ -377,6 +424,8 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
   uint64_t items = 0, in_items = 0;
   int narrow[kMaxGroups * 4];
   int n_narrow = 0;
+  apack_plane host_groups[kMaxGroups * 4];
+  int n_host = 0;
   for (int i = 0; i < num_groups; ++i) {
     const apack_plane &p = planes[i];
     if (p.num_planes < 0 || p.row_bytes < 0) return APACK_EINVAL;
@@ -385,6 +434,15 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
         p.src_plane_stride < 0 || p.dst_plane_stride < 0)
       return APACK_EINVAL;
     const bool tma_rows = widest_unit(p) == 16 && p.row_bytes <= static_cast<int64_t>(kSlotBytes);
+    if (const void *hs = host_source(p.src)) {
+      // pinned host source: zero-copy gather (destination in device memory, never in place)
+      if (p.src == p.dst || host_source(p.dst)) return APACK_EINVAL;
+      if (n_host == kMaxGroups * 4) return APACK_EINVAL;
+      host_groups[n_host] = p;
+      host_groups[n_host].src = hs;
+      ++n_host;
+      continue;
+    }
     if (p.src == p.dst) {
       // in place: same layout on both sides, vector rows, and the progress words of the workspace
       if (p.src_plane_stride != p.dst_plane_stride || p.src_row_stride != p.dst_row_stride) return APACK_EINVAL;
@@ -417,6 +475,25 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
       if (n_narrow == kMaxGroups * 4) return APACK_EINVAL;
       narrow[n_narrow++] = i;
     }
+  }
+  for (int k = 0; k < n_host; ++k) {
+    const apack_plane &p = host_groups[k];
+    if (widest_unit(p) == 16) {
+      const int64_t n = static_cast<int64_t>(p.num_planes) * n_out * (p.row_bytes / 16);
+      int64_t blocks = (n + 256 * kHostUnroll - 1) / (256 * kHostUnroll);
+      const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
+      if (blocks > cap) blocks = cap;
+      gather_host_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
+          static_cast<const uint8_t *>(p.src), static_cast<uint8_t *>(p.dst), p.src_plane_stride, p.dst_plane_stride,
+          p.src_row_stride, p.dst_row_stride, p.row_bytes, p.num_planes, n_out, keep_idx);
+    } else {
+      const int64_t n = static_cast<int64_t>(p.num_planes) * n_out;
+      gather_narrow_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, stream>>>(
+          static_cast<const uint8_t *>(p.src), static_cast<uint8_t *>(p.dst), p.src_plane_stride, p.dst_plane_stride,
+          p.src_row_stride, p.dst_row_stride, p.row_bytes, widest_unit(p), p.num_planes, n_out, keep_idx);
+    }
+    count_launches(1);
+    if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
   }
   for (int k = 0; k < n_narrow; ++k) {
     const apack_plane &p = planes[narrow[k]];

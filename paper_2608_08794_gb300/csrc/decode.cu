@@ -382,6 +382,7 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
   if (st != APACK_OK) return st;
   if (num_seqs == 0) return APACK_OK;
   if (!q || !k || !v || !out || !ws) return APACK_EINVAL;
+  if (in_host_memory(k) || in_host_memory(v)) return APACK_EINVAL;   // read by TMA / bulk copies
   if ((reinterpret_cast<uintptr_t>(q) & 7) || (reinterpret_cast<uintptr_t>(k) & 15) ||
       (reinterpret_cast<uintptr_t>(v) & 15) || (reinterpret_cast<uintptr_t>(out) & 15) ||
       (reinterpret_cast<uintptr_t>(ws) & 255) || (kv_token_stride & 15) ||

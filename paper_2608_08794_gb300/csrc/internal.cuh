@@ -58,6 +58,7 @@ WsLayout workspace_layout(const apack_seqs *seqs);
 int device_sm_count();
 void count_launches(uint64_t n);
 apack_status check_cuda(cudaError_t e);
+bool in_host_memory(const void *p);   // pinned or registered host memory (cudaMemoryTypeHost)
 
 apack_status validate_seqs(const apack_seqs *seqs, int64_t *total_tokens, int64_t *total_qrows);
 

@@ -51,6 +51,7 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
   apack_status st = validate_seqs(seqs, &T, &NQ);
   if (st != APACK_OK) return st;
   if (num_steps < 1 || !steps_h || !k_cache || !v_cache || !scores) return APACK_EINVAL;
+  if (in_host_memory(k_cache)) return APACK_EINVAL;   // scored by TMA: device memory
   if (hidden && hidden_dim <= 0) return APACK_EINVAL;
   const int B = seqs->num_seqs;
   const int64_t row = static_cast<int64_t>(seqs->num_kv_heads) * APACK_HEAD_DIM * 2;

@@ -16,7 +16,7 @@ import numpy as np
 import torch
 
 from . import (Seqs, apack_plane, apack_prune_step, apack_prune_schedule, apack_prune_schedule_graph,
-               apack_workspace_size, apack_keep_counts,
+               apack_workspace_size, apack_keep_counts, apack_score, apack_select, apack_compact, make_plane,
                APACK_HEAD_DIM, APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT)
 
 
@@ -166,6 +166,32 @@ class ProgressivePrune:
             self._step_seqs(0), self.L, self.k_in.view(-1), self.v_in.view(-1), self.T0 * self.row,
             self.hidden_in, self.H, self._schedule_steps(), select_mode=self.mode, scores=self.scores, ws=self.ws)
         return graph
+
+    def run_first_step_from_host(self, k_host, v_host, hidden_host=None, stream=None):
+        """Step 0 with the K/V caches of layers [l_0, L) (and the hidden states) in pinned host
+        memory, laid out like k_in / v_in / hidden_in.  Only the scored layer's keys must be on
+        the device: the caller copies slab 0 of k_in.  Scoring and selection run on the device;
+        the compaction reads only the kept rows over the host link (apack_compact from a host
+        source).  Leaves exactly what run_step(0) leaves; continue with run_step(1), ..."""
+        if self.slice_below:
+            raise ValueError("run_first_step_from_host: slice_below is not supported")
+        seqs = self._step_seqs(0)
+        t_out, lc = self.t_out[0], self.L - self.layers[0]
+        new_cu = np.zeros(self.B + 1, np.int32)
+        apack_score(seqs, self.q[0], self.k_in.view(-1), self.row, self.scores, self.ws, stream=stream)
+        apack_select(seqs, self.scores, self.counts[0], self.keep_idx[0], self.ws, select_mode=self.mode,
+                     modality_out=self.mod_out[0], stream=stream)
+        planes = [make_plane(k_host, self.k_out[0], self.row, lc, self.T0 * self.row, t_out * self.row),
+                  make_plane(v_host, self.v_out[0], self.row, lc, self.T0 * self.row, t_out * self.row)]
+        if hidden_host is not None and self.h_out[0] is not None:
+            planes.append(make_plane(hidden_host, self.h_out[0], self.H * 2, 1))
+        apack_compact(self.keep_idx[0], t_out, planes, ws=self.ws, stream=stream)
+        other = np.diff(self.cu0) - self.na0 - self.nv0
+        k = self.counts[0]
+        new_cu[1:] = np.cumsum(other + k[:, 0] + k[:, 1])
+        if len(self.new_cu) != len(self.layers):
+            self.new_cu = [None] * len(self.layers)
+        self.new_cu[0] = new_cu
 
     def run_steps(self, events=None, stream=None):
         """Runs every step with one apack_prune_step call each; events[i] = 4 CUDA

@@ -444,6 +444,41 @@ def test_prune_step_in_place_equals_out_of_place(ap):
                             modality_out=mo2, keep_idx=keep2, scores=sc2, ws=ws)
 
 
+@pytest.mark.parametrize("row_bytes,planes", [(1024, 3), (7168, 1), (48, 2)])
+def test_compact_from_pinned_host_memory(ap, row_bytes, planes):
+    """A group whose source is pinned host memory is gathered over the host link (zero
+    copy): only kept rows are read; the result is the same bytes as from device memory."""
+    rng = np.random.default_rng(row_bytes + 5)
+    T = 20011
+    src = rng.integers(0, 256, (planes, T, row_bytes), dtype=np.uint8)
+    keep = np.sort(rng.choice(T, 8123, replace=False)).astype(np.int32)
+    h = torch.from_numpy(src).pin_memory()
+    d = torch.zeros((planes, keep.size, row_bytes), dtype=torch.uint8, device="cuda")
+    p = ap.make_plane(h, d, row_bytes, planes, src_plane_stride=T * row_bytes, dst_plane_stride=keep.size * row_bytes)
+    ap.apack_compact(dev(keep), keep.size, [p])
+    torch.cuda.synchronize()
+    got = d.cpu().numpy()
+    for pl in range(planes):
+        np.testing.assert_array_equal(got[pl], oracle.compact_rows(src[pl], keep))
+
+
+def test_host_memory_is_refused_where_tma_reads_it(ap):
+    rng = np.random.default_rng(3)
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, [300], [4], 28, 4)
+    seqs = ap.Seqs(cu, cuq, na, nv, dev(mod), 28, 4)
+    ws = aligned_ws(ap, seqs)
+    scores = torch.zeros(300, dtype=torch.float32, device="cuda")
+    k_host = torch.from_numpy(k.view(np.int16)).pin_memory()
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_score(seqs, dev(q), k_host, 4 * D * 2, scores, ws)
+    assert e.value.status == ap.APACK_EINVAL
+    h = torch.zeros((2, 64, 64), dtype=torch.uint8).pin_memory()
+    with pytest.raises(ap.ApackError) as e:      # a host buffer cannot be compacted in place
+        ap.apack_compact(dev(np.arange(0, 64, 2, dtype=np.int32)), 32, [ap.make_plane(h, h, 64, 2, 4096, 4096)],
+                         ws=ws)
+    assert e.value.status == ap.APACK_EINVAL
+
+
 def test_device_fill_matches_host_generator(ap):
     from synth.device import fill_normal_bf16
     from synth.gen import normal_bf16_bits

@@ -214,6 +214,44 @@ def test_schedule_graph_replay_is_bit_identical(ap, name):
     graph.close()
 
 
+@pytest.mark.parametrize("name", ["7b_2min", "7b_ragged16"])
+def test_first_step_from_host_caches_is_bit_identical(ap, name):
+    """Step 0 with the K/V caches and hidden states in pinned host memory (only the scored
+    layer's keys on the device; the compaction reads the kept rows over the host link),
+    then the remaining steps on the device: the same outputs as the all-device schedule."""
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+
+    wl = workload(name)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod_d = torch.from_numpy(wl.modality()).cuda()
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_d,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
+    pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                          wl.prune_layers, counts, select_mode=mode)
+    fill_progressive_inputs(pp, wl)
+    pp.run()
+    torch.cuda.synchronize()
+    ref = snapshot(pp)
+    h_k = pp.k_in.cpu().pin_memory()
+    h_v = pp.v_in.cpu().pin_memory()
+    h_h = pp.hidden_in.cpu().pin_memory()
+    for buf in pp.k_out + pp.v_out + pp.h_out + pp.mod_out + pp.keep_idx:
+        buf.zero_()
+    pp.k_in[1:].zero_()                          # only the scored layer's keys stay on the device
+    pp.v_in.zero_()
+    pp.hidden_in.zero_()
+    pp.run_first_step_from_host(h_k, h_v, h_h)
+    for i in range(1, len(pp.layers)):
+        pp.run_step(i)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+    same(ref, snapshot(pp))
+
+
 @pytest.mark.parametrize("name", ["7b_2min", "7b_10min_paper"])
 def test_slicing_below_the_pruning_layers_keeps_every_layer_consistent(ap, name):
     """With slice_below, every step also compacts the caches of the layers below its
