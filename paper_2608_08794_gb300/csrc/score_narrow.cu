@@ -204,14 +204,24 @@ __global__ void __launch_bounds__(kThreads)
     float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     // causal rows: logit row rho = token * Hq + head sees this key when token >= key - (len - n_q)
     const int rho_min = plan.causal ? max(0, key - sq.t0 - (sq.len - sq.n_q)) * plan.hq : 0;
-    for (int r0 = 0; r0 < R; r0 += 8) {
-      float x[8];
+    if (R <= 32) {
+      // all rows' logits requested at once: one round trip (the paper's one query token: R = Hq)
+      float x[32];
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
-        x[u] = (r0 + u < R && r0 + u >= rho_min) ? lp[static_cast<int64_t>(r0 + u) * sq.lstride] - ls[r0 + u]
-                                                 : -INFINITY;
+      for (int u = 0; u < 32; ++u)
+        x[u] = (u < R && u >= rho_min) ? lp[static_cast<int64_t>(u) * sq.lstride] - ls[u] : -INFINITY;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) a[u] += ex2_approx(x[u]);
+      for (int u = 0; u < 32; ++u) a[u & 7] += ex2_approx(x[u]);
+    } else {
+      for (int r0 = 0; r0 < R; r0 += 8) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          x[u] = (r0 + u < R && r0 + u >= rho_min) ? lp[static_cast<int64_t>(r0 + u) * sq.lstride] - ls[r0 + u]
+                                                   : -INFINITY;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) a[u] += ex2_approx(x[u]);
+      }
     }
     out = (((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]))) / static_cast<float>(plan.hq * sq.n_q);
   }

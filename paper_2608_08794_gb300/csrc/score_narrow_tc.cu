@@ -247,20 +247,33 @@ __global__ void __launch_bounds__(tc_threads<HKV>(), 1)
           red[kt * (HKV * kTcRows) + (hg * HH + hh) * kTcRows + j] = make_float2(m[hh][j], sum[hh][j]);
     }
     asm volatile("bar.sync 1, %0;" ::"n"(tc_epi_warps<HKV>() * 32) : "memory");
-    if (!bars->abort && threadIdx.x - 64 < HKV * kTcRows) {
-      const int e = threadIdx.x - 64, h = e / kTcRows, j = e % kTcRows;
-      if (j < rg) {
-        const float2 *red = reinterpret_cast<const float2 *>(ring);
+    if (!bars->abort) {
+      // one warp per (head, row): each lane folds 4 of the 128 per-key states, then a fixed
+      // shuffle tree combines the lanes (deterministic order)
+      const float2 *red = reinterpret_cast<const float2 *>(ring);
+      for (int e = ew; e < HKV * kTcRows; e += tc_epi_warps<HKV>()) {
+        const int h = e / kTcRows, j = e % kTcRows;
+        if (j >= rg) continue;                          // uniform over the warp
+        float2 v[kTcM / 32];
         float mx = -INFINITY;
-        for (int k2 = 0; k2 < kTcM; ++k2) mx = fmaxf(mx, red[k2 * (HKV * kTcRows) + e].x);
+#pragma unroll
+        for (int i = 0; i < kTcM / 32; ++i) {
+          v[i] = red[(lane + 32 * i) * (HKV * kTcRows) + e];
+          mx = fmaxf(mx, v[i].x);
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
         float tot = 0.f;
         if (mx != -INFINITY)
-          for (int k2 = 0; k2 < kTcM; ++k2) {
-            const float2 v = red[k2 * (HKV * kTcRows) + e];
-            if (v.x != -INFINITY) tot += v.y * ex2_approx(v.x - mx);
-          }
-        const int rho = (j / G) * plan.hq + h * G + j % G;
-        part[sq.part_base + static_cast<int64_t>(c - sq.unit8_begin) * sq.rows + rho] = make_float2(mx, tot);
+#pragma unroll
+          for (int i = 0; i < kTcM / 32; ++i)
+            if (v[i].x != -INFINITY) tot += v[i].y * ex2_approx(v[i].x - mx);
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, off);
+        if (lane == 0) {
+          const int rho = (j / G) * plan.hq + h * G + j % G;
+          part[sq.part_base + static_cast<int64_t>(c - sq.unit8_begin) * sq.rows + rho] = make_float2(mx, tot);
+        }
       }
     }
     // teardown below
