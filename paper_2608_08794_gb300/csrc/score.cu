@@ -263,6 +263,7 @@ __device__ __forceinline__ void online_chunk(const uint32_t (&r)[64], uint32_t m
   sum += t;
 }
 
+template <bool CAUSAL>
 __global__ void __launch_bounds__(kThreads, 1)
     score_rowstats_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                           const __grid_constant__ ScorePlan plan, const uint8_t *__restrict__ modality,
@@ -373,9 +374,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
           const int key = key_base + c * 32 + lane;
-          mask[c] = __ballot_sync(0xffffffffu, key < t_end && (plan.causal || is_mm(mod_next[c])));
+          mask[c] = __ballot_sync(0xffffffffu, key < t_end && (CAUSAL || is_mm(mod_next[c])));
           rmask[c] = mask[c];
-          if (plan.causal) {   // keys at local index <= see
+          if (CAUSAL) {        // keys at local index <= see
             const int lim = see - (key_base - sp.t0 + c * 32);
             rmask[c] &= lim >= 31 ? 0xffffffffu : (lim < 0 ? 0u : (2u << lim) - 1u);
           }
@@ -525,6 +526,7 @@ __device__ __forceinline__ void colsum_chunk_from(const uint32_t (&r)[64], const
 
 // Work unit = (256-key pair, KV head group g); writes the group's sum for each
 // key to gsum[g][key]; the final kernel adds the groups.
+template <bool CAUSAL>
 __global__ void __launch_bounds__(kThreads, 1)
     score_colsum_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                         const __grid_constant__ ScorePlan plan, const float *__restrict__ nlse2,
@@ -633,7 +635,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool active = t < w.ntiles;
       float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
       // causal rows: only packed rows rho >= rho_min (tokens r >= key - (len - n_q)) see this key
-      const int rho_min = plan.causal ? max(0, w.kp * kKeysPerUnit2 + klane - (sp.len - sp.n_q)) * G : 0;
+      const int rho_min = CAUSAL ? max(0, w.kp * kKeysPerUnit2 + klane - (sp.len - sp.n_q)) * G : 0;
       for (int c = 0; c < nch; ++c) {
         if (!wait_or_abort(&bars->acc_full[ci], cph, bars, err, 26)) { ok = false; break; }
         tc_fence_after();
@@ -646,7 +648,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->acc_empty[ci]);   // registers hold the data: release early
           const int first = rho_min - (c * kBRows + h * 64);
-          if (first <= 0) {
+          if (!CAUSAL || first <= 0) {
             colsum_chunk<0>(rr, nl, c2, a);
             colsum_chunk<32>(rr, nl + 32, c2, a);
           } else if (first < 64) {
@@ -774,9 +776,13 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
   float *gsum = reinterpret_cast<float *>(wsb + L.gsum_off);
 
   if (!g_attr_done) {
-    if (check_cuda(cudaFuncSetAttribute(score_rowstats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (check_cuda(cudaFuncSetAttribute(score_rowstats_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         kSmemBytes)) != APACK_OK ||
-        check_cuda(cudaFuncSetAttribute(score_colsum_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        check_cuda(cudaFuncSetAttribute(score_rowstats_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        kSmemBytes)) != APACK_OK ||
+        check_cuda(cudaFuncSetAttribute(score_colsum_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        kSmemBytes)) != APACK_OK ||
+        check_cuda(cudaFuncSetAttribute(score_colsum_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         kSmemBytes)) != APACK_OK)
       return APACK_ECUDA;
     g_attr_done = true;
@@ -844,7 +850,10 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
     P.total_units = units1;
     if (units1 > 0) {
       const int grid = units1 < sms ? units1 : sms;
-      score_rowstats_kernel<<<grid, kThreads, kSmemBytes, stream>>>(qmap1, kmap1, P, seqs->modality, part, err);
+      if (P.causal)
+        score_rowstats_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap1, kmap1, P, seqs->modality, part, err);
+      else
+        score_rowstats_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap1, kmap1, P, seqs->modality, part, err);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
@@ -863,7 +872,10 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
     P.total_units = units2;
     if (units2 > 0) {
       const int grid = units2 < sms ? units2 : sms;
-      score_colsum_kernel<<<grid, kThreads, kSmemBytes, stream>>>(qmap2, kmap2, P, nlse2, gsum, err);
+      if (P.causal)
+        score_colsum_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap2, kmap2, P, nlse2, gsum, err);
+      else
+        score_colsum_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap2, kmap2, P, nlse2, gsum, err);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
