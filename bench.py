@@ -722,14 +722,17 @@ def main():
     h2d = (h_k[0].numel() * h_k.element_size() + h_m.numel() + sum(x.numel() * x.element_size() for x in h_q) +
            pp.t_out[0] * (2 * h_k.shape[0] * pp.row + pp.H * 2))
     d2h = sum(x.numel() * x.element_size() for x in h_out[0])
-    s_up, s_down = torch.cuda.Stream(), torch.cuda.Stream()
+    s_up, s_gather, s_down = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
     ev_up = [torch.cuda.Event() for _ in sets]
+    ev_sel = [torch.cuda.Event() for _ in sets]
+    ev_gath = [torch.cuda.Event() for _ in sets]
     ev_comp = [torch.cuda.Event() for _ in sets]
     ev_down = [torch.cuda.Event() for _ in sets]
     for e in ev_down:
         e.record(stream)
 
-    def e2e_iteration(j):
+    def front(j):
+        """Upload, score, select and start the host-source compaction of iteration j."""
         b = j % 2
         p = sets[b]
         with torch.cuda.stream(s_up):          # upload once the set's last result was read back
@@ -740,7 +743,18 @@ def main():
                 a.copy_(qh, non_blocking=True)
             ev_up[b].record(s_up)
         stream.wait_event(ev_up[b])
-        p.run_first_step_from_host(h_k, h_v, h_h, stream=stream)
+        p.select_first_step(stream=stream)
+        ev_sel[b].record(stream)
+        with torch.cuda.stream(s_gather):      # the link-bound gather runs beside the device work
+            s_gather.wait_event(ev_sel[b])
+            p.compact_first_step_from_host(h_k, h_v, h_h, stream=s_gather)
+            ev_gath[b].record(s_gather)
+
+    def back(j):
+        """The later steps and the read-back of iteration j."""
+        b = j % 2
+        p = sets[b]
+        stream.wait_event(ev_gath[b])
         for i in range(1, nsteps):
             p.run_step(i, stream=stream)
         ev_comp[b].record(stream)
@@ -754,8 +768,16 @@ def main():
                 o[3 + i].copy_(p.keep_idx[i][:t], non_blocking=True)
             ev_down[b].record(s_down)
 
-    for j in range(2):
-        e2e_iteration(j)
+    def e2e_run(n):
+        # software pipeline: iteration j+1's upload, scoring and selection are queued before
+        # iteration j's later steps, so that they run while iteration j's gather holds the link
+        front(0)
+        for j in range(n):
+            if j + 1 < n:
+                front(j + 1)
+            back(j)
+
+    e2e_run(2)
     torch.cuda.synchronize()
     barrier()
     if clocks:
@@ -763,8 +785,8 @@ def main():
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     s_up.wait_stream(stream)
-    for j in range(e2e_steps):
-        e2e_iteration(j)
+    s_gather.wait_stream(stream)
+    e2e_run(e2e_steps)
     stream.wait_stream(s_down)
     e1.record(stream)
     barrier()
@@ -821,8 +843,9 @@ def main():
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps,
                     "pipeline": "caches and hidden states in pinned host memory; per iteration the scored layer's "
                                 "keys, the queries and the modality are copied, the first compaction reads only the "
-                                "kept rows over the host link, the later steps run on the device; two device buffer "
-                                "sets overlap the next upload and the previous read-back with the current compute",
+                                "kept rows over the host link (its own stream), the later steps run on the device; "
+                                "two device buffer sets let the next iteration's upload, scoring and selection and "
+                                "the previous read-back run while the current gather holds the link",
                     "h2d_note": "h2d_bytes_per_step counts the copies and the kept rows read from host memory"},
             "clocks": clocks.summary() if clocks else None,
             "context": schedule_context(wl, pp),

@@ -173,14 +173,24 @@ class ProgressivePrune:
         the device: the caller copies slab 0 of k_in.  Scoring and selection run on the device;
         the compaction reads only the kept rows over the host link (apack_compact from a host
         source).  Leaves exactly what run_step(0) leaves; continue with run_step(1), ..."""
+        self.select_first_step(stream=stream)
+        self.compact_first_step_from_host(k_host, v_host, hidden_host, stream=stream)
+
+    def select_first_step(self, stream=None):
+        """Scoring and selection of step 0 on the device (slab 0 of k_in holds the scored keys):
+        the first half of run_first_step_from_host."""
         if self.slice_below:
             raise ValueError("run_first_step_from_host: slice_below is not supported")
         seqs = self._step_seqs(0)
-        t_out, lc = self.t_out[0], self.L - self.layers[0]
-        new_cu = np.zeros(self.B + 1, np.int32)
         apack_score(seqs, self.q[0], self.k_in.view(-1), self.row, self.scores, self.ws, stream=stream)
         apack_select(seqs, self.scores, self.counts[0], self.keep_idx[0], self.ws, select_mode=self.mode,
                      modality_out=self.mod_out[0], stream=stream)
+
+    def compact_first_step_from_host(self, k_host, v_host, hidden_host=None, stream=None):
+        """The compaction of step 0 from host-resident caches (after select_first_step on the
+        stream order): only the kept rows cross the host link."""
+        t_out, lc = self.t_out[0], self.L - self.layers[0]
+        new_cu = np.zeros(self.B + 1, np.int32)
         planes = [make_plane(k_host, self.k_out[0], self.row, lc, self.T0 * self.row, t_out * self.row),
                   make_plane(v_host, self.v_out[0], self.row, lc, self.T0 * self.row, t_out * self.row)]
         if hidden_host is not None and self.h_out[0] is not None:
