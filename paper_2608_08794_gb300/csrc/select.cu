@@ -1,8 +1,8 @@
 // select.cu -- per-(sequence, modality) top-k of Eq. inner (Sec. 3.2) and the stable keep map.
 //
-// One thread-block cluster of CL CTAs per sequence (16 when the launch's clusters
-// still fit the GPU that way, else 8); CTA c owns a contiguous slice of the
-// sequence's tokens.
+// One thread-block cluster of CL CTAs per sequence (16 for long sequences when the
+// launch's clusters still fit the GPU that way, else 8); CTA c owns a contiguous
+// slice of the sequence's tokens.
 //
 //  1. Radix select (4 passes of 8 bits, most significant first) of the k-th
 //     largest score of every segment.  Scores are >= 0, so the order of their
@@ -30,7 +30,6 @@ namespace apack {
 
 namespace {
 
-constexpr int kClusterSmall = 8, kClusterLarge = 16;
 constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxCached = 40960;               // tokens per CTA slice cached in shared memory (200 KB)
@@ -350,6 +349,53 @@ __global__ void __cluster_dims__(CL, 1, 1) __launch_bounds__(kThreads)
 
 }  // namespace
 
+template <int CL>
+cudaError_t launch_select(const SelectPlan &P, int ns, size_t smem, const float *scores, const uint8_t *modality,
+                          int32_t *keep_idx, uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu,
+                          DeviceError *err, cudaStream_t stream) {
+  select_kernel<CL><<<dim3(CL, ns, 1), kThreads, smem, stream>>>(P, scores, modality, keep_idx, modality_out,
+                                                                   dst_of_src, new_cu, err);
+  return cudaGetLastError();
+}
+
+// Cluster size per sequence: 8 CTAs, or 16 for sequences longer than kWideFrom tokens where such
+// clusters can be resident and every sequence of the launch still gets its own 16 SMs.  Measured
+// on GB300 (graph replays, joint top-k): 16 CTAs win from about 30k tokens (26.8 vs 37.2 us at
+// 135k), 8 win below (13.3 vs 14.1 us at 16k; 1, 2 or 4 CTAs never win by more than 0.5 us and
+// lose up to 11x on long sequences).  0 when the attributes cannot be set.
+constexpr int kWideFrom = 24576;
+
+int select_cluster_size(int max_len, int ns) {
+  static int ready = -1, large_ok = 0;
+  if (ready < 0) {
+    ready = cudaFuncSetAttribute(select_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(kCacheBytes)) == cudaSuccess;
+    large_ok = ready &&
+               cudaFuncSetAttribute(select_kernel<16>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
+                   cudaSuccess &&
+               cudaFuncSetAttribute(select_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    static_cast<int>(kCacheBytes)) == cudaSuccess;
+    if (large_ok) {   // can a 16-CTA cluster of this kernel be resident at all?
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = 16;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      cfg.gridDim = dim3(16, 1, 1);
+      cfg.blockDim = dim3(kThreads, 1, 1);
+      cfg.dynamicSmemBytes = kCacheBytes;
+      cfg.attrs = at;
+      cfg.numAttrs = 1;
+      int nclusters = 0;
+      large_ok = cudaOccupancyMaxActiveClusters(&nclusters, select_kernel<16>, &cfg) == cudaSuccess && nclusters > 0;
+    }
+    cudaGetLastError();
+  }
+  if (!ready) return 0;
+  return (max_len > kWideFrom && large_ok && ns * 16 <= device_sm_count()) ? 16 : 8;
+}
+
 apack_status run_select(const apack_seqs *seqs, const float *scores, const int32_t *keep_count_h, int32_t mode,
                         int32_t *keep_idx, uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu_seqlens,
                         void *ws, cudaStream_t stream) {
@@ -402,54 +448,25 @@ apack_status run_select(const apack_seqs *seqs, const float *scores, const int32
       q.out_base = out_base;
       out_base += q.out_len;
     }
-    // 16-CTA clusters while every sequence of the launch still gets its own 16 SMs
-    static int large_ok = -1;
-    if (large_ok < 0) {
-      large_ok = cudaFuncSetAttribute(select_kernel<kClusterLarge>, cudaFuncAttributeNonPortableClusterSizeAllowed,
-                                      1) == cudaSuccess &&
-                 cudaFuncSetAttribute(select_kernel<kClusterLarge>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      static_cast<int>(kCacheBytes)) == cudaSuccess &&
-                 cudaFuncSetAttribute(select_kernel<kClusterSmall>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      static_cast<int>(kCacheBytes)) == cudaSuccess;
-      if (large_ok) {   // can a 16-CTA cluster of this kernel be resident at all?
-        cudaLaunchConfig_t cfg = {};
-        cudaLaunchAttribute at[1];
-        at[0].id = cudaLaunchAttributeClusterDimension;
-        at[0].val.clusterDim.x = kClusterLarge;
-        at[0].val.clusterDim.y = 1;
-        at[0].val.clusterDim.z = 1;
-        cfg.gridDim = dim3(kClusterLarge, 1, 1);
-        cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = kCacheBytes;
-        cfg.attrs = at;
-        cfg.numAttrs = 1;
-        int nclusters = 0;
-        large_ok = cudaOccupancyMaxActiveClusters(&nclusters, select_kernel<kClusterLarge>, &cfg) == cudaSuccess &&
-                   nclusters > 0;
-      }
-      cudaGetLastError();
-      if (!large_ok &&
-          check_cuda(cudaFuncSetAttribute(select_kernel<kClusterSmall>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          static_cast<int>(kCacheBytes))) != APACK_OK)
-        return APACK_ECUDA;
-    }
-    const int CL = (large_ok && ns * kClusterLarge <= device_sm_count()) ? kClusterLarge : kClusterSmall;
-    // cache each CTA's slice in shared memory when the longest slice of the launch fits
     int max_len = 0;
     for (int i = 0; i < ns; ++i) max_len = P.seq[i].len > max_len ? P.seq[i].len : max_len;
+    const int CL = select_cluster_size(max_len, ns);
+    if (CL == 0) return APACK_ECUDA;
+    // cache each CTA's slice in shared memory when the longest slice of the launch fits
     const int slice = (max_len + CL - 1) / CL;
     size_t smem = 0;
     if (slice <= kMaxCached) {
       P.cache_tokens = slice;
       smem = static_cast<size_t>(slice) * 5;
     }
-    dim3 grid(CL, ns, 1);
-    if (CL == kClusterLarge)
-      select_kernel<kClusterLarge><<<grid, kThreads, smem, stream>>>(P, scores, seqs->modality, keep_idx, modality_out,
-                                                                     dst_of_src, new_cu_seqlens, err);
+    cudaError_t e = cudaSuccess;
+    if (CL == 16)
+      e = launch_select<16>(P, ns, smem, scores, seqs->modality, keep_idx, modality_out, dst_of_src, new_cu_seqlens,
+                            err, stream);
     else
-      select_kernel<kClusterSmall><<<grid, kThreads, smem, stream>>>(P, scores, seqs->modality, keep_idx, modality_out,
-                                                                     dst_of_src, new_cu_seqlens, err);
+      e = launch_select<8>(P, ns, smem, scores, seqs->modality, keep_idx, modality_out, dst_of_src, new_cu_seqlens,
+                           err, stream);
+    if (check_cuda(e) != APACK_OK) return APACK_ECUDA;
     count_launches(1);
     if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
   }
