@@ -52,13 +52,18 @@ def schedule_keep_counts(cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, n
 class ProgressivePrune:
     def __init__(self, cu_seqlens, cu_qlens, n_audio, n_visual, num_q_heads, num_kv_heads, num_layers, hidden_dim,
                  prune_layers, keep_counts, device="cuda", select_mode=APACK_SELECT_PER_MODALITY,
-                 with_hidden=True, slice_below=False, softmax_domain=0):
+                 with_hidden=True, slice_below=False, softmax_domain=0, in_place=False):
         """keep_counts[i]: int array [B, 2] of the tokens each segment keeps after step i.
 
         slice_below: also compact, at every step, the K/V of the layers below its
         pruning layer, so that after the schedule every layer's cache holds only the
         kept tokens (for decoding).  The caches of layers [0, l_0) are then inputs
-        too (``k_low_in`` / ``v_low_in``); ``output_low_kv`` gives layers [0, l_i)."""
+        too (``k_low_in`` / ``v_low_in``); ``output_low_kv`` gives layers [0, l_i).
+
+        in_place: every step compacts within the input buffers (k_in, v_in, hidden_in keep their
+        slab stride; step i's result is the first t_out_i rows of slabs l_i - l_0 ..), so no
+        output caches are allocated: a third of the memory, at the in-place gather's speed.
+        softmax_domain: APACK_SOFTMAX_MM (default) or APACK_SOFTMAX_CAUSAL_ROW."""
         self.dev = torch.device(device)
         self.softmax_domain = int(softmax_domain)
         self.cu0 = np.asarray(cu_seqlens, np.int32)
@@ -83,12 +88,19 @@ class ProgressivePrune:
         nq = int(self.cuq[-1])
         self.q = [torch.empty((nq, num_q_heads, APACK_HEAD_DIM), dtype=torch.bfloat16, device=dev)
                   for _ in self.layers]
-        # outputs, sized for the largest step
+        # outputs, sized for the largest step (ping-pong), or the inputs themselves (in place: every
+        # step compacts its slabs of k_in / v_in and hidden_in within their own rows)
         t1 = self.t_out[0]
-        self.k_out = [torch.empty(Lc0 * t1 * self.row // 2, dtype=torch.bfloat16, device=dev) for _ in range(2)]
-        self.v_out = [torch.empty_like(self.k_out[0]) for _ in range(2)]
-        self.h_out = [torch.empty((t1, hidden_dim), dtype=torch.bfloat16, device=dev) if with_hidden else None
-                      for _ in range(2)]
+        self.in_place = bool(in_place)
+        if self.in_place and slice_below:
+            raise ValueError("in_place and slice_below cannot be combined")
+        if self.in_place:
+            self.k_out = self.v_out = self.h_out = None
+        else:
+            self.k_out = [torch.empty(Lc0 * t1 * self.row // 2, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+            self.v_out = [torch.empty_like(self.k_out[0]) for _ in range(2)]
+            self.h_out = [torch.empty((t1, hidden_dim), dtype=torch.bfloat16, device=dev) if with_hidden else None
+                          for _ in range(2)]
         self.mod_out = [torch.empty(t1, dtype=torch.uint8, device=dev) for _ in range(2)]
         self.slice_below = slice_below
         if slice_below:
@@ -129,21 +141,29 @@ class ProgressivePrune:
         """(seqs, k_in, v_in, in_layer_stride, hidden_in) entering step i; K/V as flat bf16 views."""
         if i == 0:
             return (self._step_seqs(0), self.k_in.view(-1), self.v_in.view(-1), self.T0 * self.row, self.hidden_in)
-        prev = (i - 1) % 2
-        t_prev = self.t_out[i - 1]
-        skip = self.layers[i] - self.layers[i - 1]
-        off = skip * t_prev * self.row // 2          # bf16 elements
-        k = self.k_out[prev][off:]
-        v = self.v_out[prev][off:]
-        return (self._step_seqs(i), k, v, t_prev * self.row, self.h_out[prev])
+        k_prev, v_prev, stride = self.step_outputs(i - 1)
+        off = (self.layers[i] - self.layers[i - 1]) * stride // 2     # bf16 elements
+        return (self._step_seqs(i), k_prev[off:], v_prev[off:], stride, self.step_hidden_out(i - 1))
+
+    def step_outputs(self, i):
+        """(k_out, v_out, slab stride in bytes) that step i writes: flat bf16 views."""
+        if self.in_place:
+            off = (self.layers[i] - self.layers[0]) * self.T0 * self.row // 2
+            return self.k_in.view(-1)[off:], self.v_in.view(-1)[off:], self.T0 * self.row
+        o = i % 2
+        return self.k_out[o], self.v_out[o], self.t_out[i] * self.row
+
+    def step_hidden_out(self, i):
+        return self.hidden_in if self.in_place else self.h_out[i % 2]
 
     def _schedule_steps(self):
         steps = []
         for i in range(len(self.layers)):
             o = i % 2
-            steps.append(dict(layer=self.layers[i], q=self.q[i], keep_count=self.counts[i], k_out=self.k_out[o],
-                              v_out=self.v_out[o], kv_out_layer_stride=self.t_out[i] * self.row,
-                              hidden_out=self.h_out[o], modality_out=self.mod_out[o], keep_idx=self.keep_idx[i],
+            k_out, v_out, stride = self.step_outputs(i)
+            steps.append(dict(layer=self.layers[i], q=self.q[i], keep_count=self.counts[i], k_out=k_out,
+                              v_out=v_out, kv_out_layer_stride=stride,
+                              hidden_out=self.step_hidden_out(i), modality_out=self.mod_out[o], keep_idx=self.keep_idx[i],
                               extra_planes=self._below_planes(i)))
         return steps
 
@@ -179,8 +199,8 @@ class ProgressivePrune:
     def select_first_step(self, stream=None):
         """Scoring and selection of step 0 on the device (slab 0 of k_in holds the scored keys):
         the first half of run_first_step_from_host."""
-        if self.slice_below:
-            raise ValueError("run_first_step_from_host: slice_below is not supported")
+        if self.slice_below or self.in_place:
+            raise ValueError("run_first_step_from_host: slice_below and in_place are not supported")
         seqs = self._step_seqs(0)
         apack_score(seqs, self.q[0], self.k_in.view(-1), self.row, self.scores, self.ws, stream=stream)
         apack_select(seqs, self.scores, self.counts[0], self.keep_idx[0], self.ws, select_mode=self.mode,
@@ -215,11 +235,11 @@ class ProgressivePrune:
             self.new_cu = [None] * len(self.layers)
         seqs, k, v, stride, h = self.step_args(i)
         o = i % 2
-        t_out = self.t_out[i]
+        k_out, v_out, out_stride = self.step_outputs(i)
         self.new_cu[i] = apack_prune_step(
             seqs, self.layers[i], self.L, self.q[i], k, v, stride, h, self.H, keep_count=self.counts[i],
-            select_mode=self.mode, k_out=self.k_out[o], v_out=self.v_out[o], kv_out_layer_stride=t_out * self.row,
-            hidden_out=self.h_out[o], modality_out=self.mod_out[o], keep_idx=self.keep_idx[i],
+            select_mode=self.mode, k_out=k_out, v_out=v_out, kv_out_layer_stride=out_stride,
+            hidden_out=self.step_hidden_out(i), modality_out=self.mod_out[o], keep_idx=self.keep_idx[i],
             scores=self.scores, ws=self.ws, stage_events=events, stream=stream)
         return self.new_cu[i]
 
@@ -253,14 +273,19 @@ class ProgressivePrune:
         return self.k_low[o][:n].view(shape), self.v_low[o][:n].view(shape)
 
     def output_kv(self, i):
-        """Views of step i's compacted K and V: [L - l_i, t_out_i, Hkv, D]."""
+        """Views of step i's compacted K and V: [L - l_i, t_out_i, Hkv, D] (in place: strided
+        views into k_in / v_in, valid until a later step compacts them again)."""
+        if self.in_place:
+            s = self.layers[i] - self.layers[0]
+            return self.k_in[s:, :self.t_out[i]], self.v_in[s:, :self.t_out[i]]
         o = i % 2
         n = (self.L - self.layers[i]) * self.t_out[i] * self.row // 2
         shape = (self.L - self.layers[i], self.t_out[i], self.hkv, APACK_HEAD_DIM)
         return self.k_out[o][:n].view(shape), self.v_out[o][:n].view(shape)
 
     def output_hidden(self, i):
-        return None if self.h_out[i % 2] is None else self.h_out[i % 2][:self.t_out[i]]
+        h = self.step_hidden_out(i)
+        return None if h is None else h[:self.t_out[i]]
 
     def mm_tokens_per_step(self):
         """|S| entering each step (the unit of the throughput metric)."""

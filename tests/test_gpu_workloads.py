@@ -214,6 +214,68 @@ def test_schedule_graph_replay_is_bit_identical(ap, name):
     graph.close()
 
 
+@pytest.mark.parametrize("name", ["7b_2min", "7b_ragged16", "7b_10min_paper"])
+def test_in_place_schedule_equals_ping_pong(ap, name):
+    """ProgressivePrune(in_place=True): every step compacts within k_in / v_in / hidden_in
+    (apack_compact in place); the last step's caches, hidden states, modality, offsets and
+    every step's kept indices equal those of the ping-pong schedule, through the schedule
+    call, per-step calls and a captured graph."""
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+
+    wl = workload(name)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod_d = torch.from_numpy(wl.modality()).cuda()
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_d,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
+
+    def make(in_place):
+        pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                              wl.prune_layers, counts, select_mode=mode, in_place=in_place)
+        fill_progressive_inputs(pp, wl)
+        return pp
+
+    def result(pp):
+        n = len(pp.layers)
+        k, v = pp.output_kv(n - 1)
+        return ([pp.keep_idx[i][:pp.t_out[i]].clone() for i in range(n)], [np.asarray(c).copy() for c in pp.new_cu],
+                k.contiguous().view(torch.int16).clone(), v.contiguous().view(torch.int16).clone(),
+                pp.output_hidden(n - 1).view(torch.int16).clone(), pp.mod_out[(n - 1) % 2][:pp.t_out[-1]].clone())
+
+    def check(a, b):
+        for x, y in zip(a[0], b[0]):
+            assert torch.equal(x, y)
+        for x, y in zip(a[1], b[1]):
+            np.testing.assert_array_equal(x, y)
+        for x, y in zip(a[2:], b[2:]):
+            assert torch.equal(x, y)
+
+    ref_pp = make(False)
+    ref_pp.run()
+    torch.cuda.synchronize()
+    ref = result(ref_pp)
+    del ref_pp
+    pp = make(True)
+    pp.run()
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+    check(ref, result(pp))
+    pp = make(True)
+    pp.run_steps()
+    torch.cuda.synchronize()
+    check(ref, result(pp))
+    pp = make(True)
+    graph = pp.capture()
+    graph.launch()
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+    check(ref, result(pp))
+    graph.close()
+
+
 @pytest.mark.parametrize("name", ["7b_2min", "7b_ragged16"])
 def test_first_step_from_host_caches_is_bit_identical(ap, name):
     """Step 0 with the K/V caches and hidden states in pinned host memory (only the scored
