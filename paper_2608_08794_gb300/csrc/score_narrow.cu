@@ -61,6 +61,7 @@ __global__ void __launch_bounds__(kThreads)
     score_narrow_logits_kernel(const __grid_constant__ NarrowPlan plan, const uint16_t *__restrict__ q,
                                const uint8_t *__restrict__ k, int64_t k_stride, const uint8_t *__restrict__ modality,
                                float *__restrict__ logits, float2 *__restrict__ part) {
+  pdl_wait_and_release();
   extern __shared__ __align__(16) float smem_f[];
   const int s = find_unit_seq(plan, blockIdx.x);
   const NSeq &sq = plan.seq[s];
@@ -143,6 +144,7 @@ __global__ void __launch_bounds__(kThreads)
 __global__ void __launch_bounds__(kThreads)
     score_narrow_merge_kernel(const __grid_constant__ NarrowPlan plan, const float2 *__restrict__ part,
                               float *__restrict__ lse2) {
+  pdl_wait_and_release();
   __shared__ float red[kWarps];
   __shared__ float mshared;
   const int64_t e = blockIdx.x;
@@ -188,6 +190,7 @@ __global__ void __launch_bounds__(kThreads)
     score_narrow_final_kernel(const __grid_constant__ NarrowPlan plan, const uint8_t *__restrict__ modality,
                               const float *__restrict__ logits, const float *__restrict__ lse2,
                               float *__restrict__ scores) {
+  pdl_wait_and_release();
   extern __shared__ __align__(16) float ls[];
   const int s = find_unit_seq(plan, blockIdx.x);
   const NSeq &sq = plan.seq[s];
@@ -238,8 +241,8 @@ cudaError_t launch_logits(int grid, size_t smem, cudaStream_t stream, const Narr
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  score_narrow_logits_kernel<RG><<<grid, kThreads, smem, stream>>>(P, q, k, k_stride, modality, logits, part);
-  return cudaGetLastError();
+  return launch_pdl(score_narrow_logits_kernel<RG>, dim3(grid), dim3(kThreads), smem, stream, P, q, k, k_stride,
+                    modality, logits, part);
 }
 
 }  // namespace
@@ -352,14 +355,16 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
     count_launches(1);
     if (check_cuda(e) != APACK_OK) return APACK_ECUDA;
     if (rows_all > 0) {
-      score_narrow_merge_kernel<<<static_cast<unsigned>(rows_all), kThreads, 0, stream>>>(P, part, lse2);
+      if (check_cuda(launch_pdl(score_narrow_merge_kernel, dim3(static_cast<unsigned>(rows_all)), dim3(kThreads), 0,
+                                stream, P, part, lse2)) != APACK_OK)
+        return APACK_ECUDA;
       count_launches(1);
-      if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
-    score_narrow_final_kernel<<<units, kThreads, static_cast<size_t>(max_rows) * sizeof(float), stream>>>(
-        P, seqs->modality, logits, lse2, scores);
+    if (check_cuda(launch_pdl(score_narrow_final_kernel, dim3(units), dim3(kThreads),
+                              static_cast<size_t>(max_rows) * sizeof(float), stream, P, seqs->modality, logits, lse2,
+                              scores)) != APACK_OK)
+      return APACK_ECUDA;
     count_launches(1);
-    if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
   }
   return APACK_OK;
 }

@@ -75,6 +75,7 @@ __global__ void __launch_bounds__(tc_threads<HKV>(), 1)
     score_narrow_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ NarrowPlan plan,
                            const uint16_t *__restrict__ q, const uint8_t *__restrict__ modality,
                            float *__restrict__ logits, float2 *__restrict__ part, DeviceError *err) {
+  pdl_wait_and_release();
   using Lay = TcLayout<HKV>;
   extern __shared__ __align__(1024) uint8_t smem[];
   if ((smem_u32(smem) & 1023u) != 0) {
@@ -311,8 +312,8 @@ cudaError_t launch_narrow_tc(int grid, cudaStream_t stream, const CUtensorMap &k
       if (e != cudaSuccess) return e;
       attr = true;
     }
-    score_narrow_tc_kernel<4><<<grid, tc_threads<4>(), TcLayout<4>::kBytes, stream>>>(kmap, P, q, modality,
-                                                                                      logits, part, err);
+    return launch_pdl(score_narrow_tc_kernel<4>, dim3(grid), dim3(tc_threads<4>()), TcLayout<4>::kBytes, stream,
+                      kmap, P, q, modality, logits, part, err);
   } else {
     static bool attr = false;
     if (!attr) {
@@ -322,10 +323,9 @@ cudaError_t launch_narrow_tc(int grid, cudaStream_t stream, const CUtensorMap &k
       if (e != cudaSuccess) return e;
       attr = true;
     }
-    score_narrow_tc_kernel<2><<<grid, tc_threads<2>(), TcLayout<2>::kBytes, stream>>>(kmap, P, q, modality,
-                                                                                      logits, part, err);
+    return launch_pdl(score_narrow_tc_kernel<2>, dim3(grid), dim3(tc_threads<2>()), TcLayout<2>::kBytes, stream,
+                      kmap, P, q, modality, logits, part, err);
   }
-  return cudaGetLastError();
 }
 
 }  // namespace apack
