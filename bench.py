@@ -405,12 +405,14 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
                          "note": "bf16 tokens read once + fp32 frame embeddings written once, over the whole call"}}
 
 
-def scoring_roofline(wl, pp, cuq, score_ms_per_step):
+def scoring_roofline(wl, pp, cuq, score_ms_per_step, sm_mhz=None):
     """Useful tensor work of the scoring stage: one Q K^T over the multimodal keys per
     step and sequence (2 n_q Hq |S| D flop, summed over the sequences of the batch).  The two-pass softmax computes Q K^T twice and every
     logit also needs one exp2 per pass (the SFU is the second ceiling), so this
-    fraction understates how busy the tensor pipe is."""
+    fraction understates how busy the tensor pipe is: `frac_executed` counts both
+    contractions, and `exp2_per_clk_per_sm` is the exp2 rate the stage sustained."""
     import numpy as np
+    import torch
     nq = np.diff(np.asarray(cuq, np.int64))                   # query rows per sequence
     # |S| per sequence entering each step: the original counts, then the previous step's kept counts
     s_seq = [np.asarray(pp.na0, np.int64) + np.asarray(pp.nv0, np.int64)]
@@ -419,11 +421,16 @@ def scoring_roofline(wl, pp, cuq, score_ms_per_step):
     ms = float(np.sum(score_ms_per_step))
     achieved = sum(flops) / (ms / 1e3) / 1e12
     peak, kind = measured_tensor_peak()
+    exp2 = 2 * sum(flops) / (2.0 * wl.head_dim)
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
     return {"bound": "tensor", "kernel": "score_rowstats_kernel + score_colsum_kernel (+ q_pack, merge, finalize)",
             "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
             "peak_source": kind, "useful_flops_per_iter": sum(flops),
-            "logits_per_iter": sum(flops) / (2.0 * wl.head_dim), "exp2_per_iter": 2 * sum(flops) / (2.0 * wl.head_dim),
-            "note": "useful flops = one Q K^T per step over the multimodal keys; the stage runs two passes"}
+            "executed_flops_per_iter": 2 * sum(flops), "frac_executed": 2 * achieved / peak,
+            "logits_per_iter": sum(flops) / (2.0 * wl.head_dim), "exp2_per_iter": exp2,
+            "exp2_per_clk_per_sm": (exp2 / (ms / 1e3) / sms / (sm_mhz * 1e6)) if sm_mhz else None,
+            "note": "useful flops = one Q K^T per step over the multimodal keys; the stage runs two passes "
+                    "(executed = both contractions) and one exp2 per logit in each"}
 
 
 def decode_measure(ap, wl, pp, steps, warmup, stream, dist):
@@ -813,6 +820,7 @@ def main():
         if prof is not None:   # ncu DRAM bytes of a captured launch, scaled to each launch by rows moved
             traffic = [int(prof["traffic_over_algorithmic"] * b) for b in comp_bytes]
         score_ms, select_ms = stage_ms[:, 0].sum(), stage_ms[:, 1].sum()
+        clock_summary = clocks.summary() if clocks else {}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": per_step_ms, "higher_is_better": True, "scaling": "weak",
@@ -830,7 +838,7 @@ def main():
                          "traffic": traffic, "peak_source": peak_kind,
                          "algorithmic_bytes_per_launch": comp_bytes,
                          "avg_launch_ms": [float(x) for x in comp_ms]},
-            "roofline_scoring": scoring_roofline(wl, pp, cuq, stage_ms[:, 0]),
+            "roofline_scoring": scoring_roofline(wl, pp, cuq, stage_ms[:, 0], clock_summary.get("sm_mhz")),
             "stages_ms_per_iter": {"score": float(score_ms), "select": float(select_ms),
                                    "compact": float(comp_ms.sum())},
             "launch": "the schedule captured once by apack_prune_schedule_graph and replayed every iteration "
@@ -847,7 +855,7 @@ def main():
                                 "two device buffer sets let the next iteration's upload, scoring and selection and "
                                 "the previous read-back run while the current gather holds the link",
                     "h2d_note": "h2d_bytes_per_step counts the copies and the kept rows read from host memory"},
-            "clocks": clocks.summary() if clocks else None,
+            "clocks": clock_summary or None,
             "context": schedule_context(wl, pp),
         }
         line["prellm_alignment"] = prellm

@@ -168,27 +168,15 @@ __device__ __forceinline__ void st_progress(uint16_t *p, uint32_t v) {
   asm volatile("st.relaxed.gpu.global.u16 [%0], %1;" ::"l"(p), "h"(static_cast<uint16_t>(v)) : "memory");
 }
 
-// First index j >= lo with a[j] >= x (n if none); a ascending and a[lo - 1] < x (or lo == 0).
-// The warp gallops (lane l probes lo + 2^l - 1), then probes 32 evenly spaced rows of the bracket
-// per round: two rounds when the answer is near lo, as it is for successive chunks of a CTA.
-__device__ __forceinline__ uint32_t warp_lower_bound(const int32_t *__restrict__ a, uint32_t n, uint32_t lo,
+// #{ r < n : a[r] < x } for a strictly increasing, given a bracket [lo, hi] that holds it
+// (a[lo - 1] < x or lo == 0; hi == n or a[hi] >= x).  Rounds of 32 evenly spaced probes narrow
+// wide brackets; a bracket of at most 256 rows is then counted in one round, 8 rows per lane
+// (independent loads of a few adjacent cache lines).
+constexpr uint32_t kCountRows = 8;
+
+__device__ __forceinline__ uint32_t warp_count_below(const int32_t *__restrict__ a, uint32_t lo, uint32_t hi,
                                                      int64_t x, int lane) {
-  if (lo >= n) return n;
-  uint32_t hi = n;
-  {
-    const uint64_t p = static_cast<uint64_t>(lo) + (1ull << lane) - 1;
-    const bool valid = p < n;
-    const uint32_t vm = __ballot_sync(0xffffffffu, valid);
-    const uint32_t b = __ballot_sync(0xffffffffu, valid && a[p] >= x);
-    if (b) {
-      const int f = __ffs(b) - 1;
-      hi = lo + (1u << f) - 1;                              // a[hi] >= x
-      if (f > 0) lo += 1u << (f - 1);                       // a[lo - 1] < x
-    } else {
-      lo += 1u << (31 - __clz(vm));                         // past the last probe inside [lo, n)
-    }
-  }
-  while (hi > lo) {                                         // a[lo - 1] < x <= a[hi] (or hi == n)
+  while (hi - lo > 32 * kCountRows) {
     const uint32_t span = hi - lo;
     const uint32_t step = (span + 31) / 32;
     const uint32_t p = lo + lane * step;
@@ -201,7 +189,11 @@ __device__ __forceinline__ uint32_t warp_lower_bound(const int32_t *__restrict__
       lo += ((span - 1) / step) * step + 1;                 // past the last probe inside [lo, hi)
     }
   }
-  return hi;
+  uint32_t cnt = 0;
+  const uint32_t p0 = lo + lane * kCountRows;
+#pragma unroll
+  for (uint32_t i = 0; i < kCountRows; ++i) cnt += (p0 + i < hi && a[p0 + i] < x) ? 1u : 0u;
+  return lo + __reduce_add_sync(0xffffffffu, cnt);
 }
 
 __global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constant__ TmaPlan plan,
@@ -224,8 +216,9 @@ __global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constan
     load_item(decode_item(plan, me + j * P), slots + j * kSlotBytes, &full[j], keep_idx, lane);
   bool ok = true;
   uint32_t waited = 0;                                        // positions whose loads were observed
-  uint32_t hint_row = 0;                                      // search hint: previous answer (same group)
+  uint32_t hint_row = 0;                                      // #{ keep_idx < hint_limit }, previous item
   int64_t hint_limit = 0;
+  const TmaGroup *hint_grp = nullptr;
   for (uint32_t j = 0; ok && j < n_mine; ++j) {
     const int slot = j % kInSlots;
     const uint32_t item = me + j * P;
@@ -252,9 +245,18 @@ __global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constan
     const TmaGroup &G = *it.grp;
     const uint32_t c = it.r0 / G.rows_per_slot;
     const int64_t limit = static_cast<int64_t>(it.r0) + it.nrows;
-    if (limit < hint_limit) hint_row = 0;                 // a new group: the search starts over
-    hint_row = warp_lower_bound(keep_idx, plan.n_out, hint_row, limit, lane);
-    hint_limit = limit;
+    {
+      // keep_idx holds distinct integers, so the count below limit grows by at most limit -
+      // hint_limit from the previous item of the group, and never exceeds limit
+      const int64_t n = plan.n_out;
+      const bool same = &G == hint_grp;
+      const uint32_t lo = same ? hint_row : 0;
+      const uint32_t hi = static_cast<uint32_t>(same ? min(n, static_cast<int64_t>(hint_row) + (limit - hint_limit))
+                                                     : min(n, limit));
+      hint_row = warp_count_below(keep_idx, lo, hi, limit, lane);
+      hint_limit = limit;
+      hint_grp = &G;
+    }
     uint32_t kmin = 1, kmax = 0;                          // no dependency unless some row reads below limit
     if (hint_row > 0) {
       const uint32_t c_hi = (hint_row - 1) / G.rows_per_slot;
@@ -262,31 +264,48 @@ __global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constan
       kmax = min(c, kmin + plan.dep_period - 1);
     }
     uint32_t owner[kInChecks / 32], need[kInChecks / 32];
+    {
+      // item - k * num_planes for k = kmin + lane + 32 u: one division, then steps of 32 planes
+      const uint32_t d = 32u * G.num_planes, dq = d / P, dr = d - dq * P;
+      const uint32_t other0 = item - (kmin + lane) * G.num_planes;   // only used while k <= kmax
+      uint32_t o = other0 % P, q = other0 / P;
 #pragma unroll
-    for (int u = 0; u < kInChecks / 32; ++u) {
-      const uint32_t k = kmin + lane + 32 * u;
-      owner[u] = me;                                      // no check: my own items are waited in order
-      need[u] = 0;
-      if (k <= kmax) {
-        const uint32_t other = item - k * G.num_planes;
-        owner[u] = other % P;
-        need[u] = other / P + 1;
+      for (int u = 0; u < kInChecks / 32; ++u) {
+        const uint32_t k = kmin + lane + 32 * u;
+        owner[u] = me;                                    // no check: my own items are waited in order
+        need[u] = 0;
+        if (k <= kmax) {
+          owner[u] = o;
+          need[u] = q + 1;
+        }
+        // the next u: other - d
+        const bool borrow = o < dr;
+        o = borrow ? o + P - dr : o - dr;
+        q = q - dq - (borrow ? 1u : 0u);
       }
     }
-    // each lane owns distinct owners (k differ by less than the period), so the cache needs no sync
+    // each lane owns distinct owners (k differ by less than the period), so the cache needs no sync.
+    // When any cached word is too old, every owner of the check is read again in the same round:
+    // the words read are far ahead of what later items need, so the cache then lasts until the
+    // needs have grown past them (a few rounds per launch instead of one per stale owner).
     bool mine_ok = true;
-    const uint64_t t0 = globaltimer_ns();
+    uint64_t t0 = 0;                                      // the clock is read once a round has failed
     for (;;) {
+      bool stale = false;
+#pragma unroll
+      for (int u = 0; u < kInChecks / 32; ++u) stale |= owner[u] != me && seen[owner[u]] < need[u];
+      if (!__any_sync(0xffffffffu, stale)) break;
       bool all = true;
 #pragma unroll
       for (int u = 0; u < kInChecks / 32; ++u) {
-        if (owner[u] != me && seen[owner[u]] < need[u]) {
+        if (owner[u] != me) {
           const uint32_t v = ld_progress(progress + owner[u]);
           seen[owner[u]] = v;
           all &= v >= need[u];
         }
       }
       if (__all_sync(0xffffffffu, all)) break;
+      if (t0 == 0) t0 = globaltimer_ns();
       if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > kWaitLimitNs)) {   // the warp gives up together
         mine_ok = false;
         break;

@@ -384,6 +384,31 @@ def test_compact_in_place_mixed_with_out_of_place_groups(ap):
     np.testing.assert_array_equal(bo.cpu().numpy(), b[keep])
 
 
+@pytest.mark.parametrize("density", [0.05, 0.43, 0.97])
+def test_compact_in_place_several_groups(ap, density):
+    """Three in-place groups in one launch (K/V-like 1024 B rows, hidden-like 7168 B rows, 16 B
+    metadata rows): every CTA's items run through group boundaries, where the dependency bounds
+    restart."""
+    rng = np.random.default_rng(int(density * 100))
+    T = 30011
+    n_keep = max(1, int(T * density))
+    keep = np.sort(rng.choice(T, n_keep, replace=False)).astype(np.int32)
+    shapes = [(6, 1024), (1, 7168), (1, 16)]
+    srcs = [rng.integers(0, 256, (pl, T, rb), dtype=np.uint8) for pl, rb in shapes]
+    bufs = [dev(s) for s in srcs]
+    ws = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    groups = [ap.make_plane(b, b, rb, pl, src_plane_stride=T * rb, dst_plane_stride=T * rb)
+              for b, (pl, rb) in zip(bufs, shapes)]
+    ap.apack_compact(dev(keep), n_keep, groups, ws=ws)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(ws) == ap.APACK_OK
+    for b, s in zip(bufs, srcs):
+        got = b.cpu().numpy()
+        for pl in range(s.shape[0]):
+            np.testing.assert_array_equal(got[pl, :n_keep], oracle.compact_rows(s[pl], keep))
+            np.testing.assert_array_equal(got[pl, n_keep:], s[pl, n_keep:])
+
+
 def test_compact_in_place_argument_checks(ap):
     T = 100
     keep = dev(np.arange(0, T, 2, dtype=np.int32))
