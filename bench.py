@@ -115,6 +115,19 @@ def host_cpu():
     return {"cpu_model": model or platform.processor() or platform.machine(), "nproc": os.cpu_count()}
 
 
+GATHER_SOURCES = ["compact.cu", "compact_plan.cuh"]     # the out-of-place gather and its item plan
+
+
+def source_sha256(kernel_src):
+    """sha256 of a kernel's source files (one name or a list, concatenated in order)."""
+    names = [kernel_src] if isinstance(kernel_src, str) else list(kernel_src)
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2608_08794_gb300", "csrc", n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
 def profiled_traffic(kernel_src, summary="gather_tma_traffic.json"):
     """DRAM bytes of a profiled launch from a committed ncu summary, if it was
     taken on the current kernel source (else None)."""
@@ -123,8 +136,7 @@ def profiled_traffic(kernel_src, summary="gather_tma_traffic.json"):
         return None
     with open(path) as f:
         d = json.load(f)
-    src = open(os.path.join(ROOT, "paper_2608_08794_gb300", "csrc", kernel_src), "rb").read()
-    if d.get("source_sha256") != hashlib.sha256(src).hexdigest():
+    if d.get("source_sha256") != source_sha256(kernel_src):
         return None
     return d
 
@@ -815,7 +827,7 @@ def main():
         peak, peak_kind = measured_peaks()
         comp_ms = stage_ms[:, 2]
         achieved = sum(comp_bytes) / (comp_ms.sum() / 1e3) / 1e9
-        prof = profiled_traffic("compact.cu")
+        prof = profiled_traffic(GATHER_SOURCES)
         traffic = None
         if prof is not None:   # ncu DRAM bytes of a captured launch, scaled to each launch by rows moved
             traffic = [int(prof["traffic_over_algorithmic"] * b) for b in comp_bytes]
