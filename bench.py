@@ -417,6 +417,39 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
                          "note": "bf16 tokens read once + fp32 frame embeddings written once, over the whole call"}}
 
 
+def link_rates(h_k, h_v, pp2, s_up, s_down, reps=3):
+    """The host link's rate on this machine, measured beside the e2e run: pinned host -> device
+    copies of up to 7 cache slabs alone, and the same copies while device -> host copies of as
+    many bytes run on another stream (the e2e pipeline keeps both directions busy)."""
+    import torch
+    lo = 1 if h_k.shape[0] > 1 else 0
+    n = min(lo + 7, h_k.shape[0])
+    src, dst = h_k[lo:n], pp2.k_in[lo:n]
+    back_src, back_dst = pp2.v_in[lo:n], h_v[lo:n]
+    nbytes = src.numel() * src.element_size()
+
+    def timed(both):
+        best = None
+        for _ in range(reps):
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            if both:
+                with torch.cuda.stream(s_down):
+                    back_dst.copy_(back_src, non_blocking=True)
+            with torch.cuda.stream(s_up):
+                a.record(s_up)
+                dst.copy_(src, non_blocking=True)
+                b.record(s_up)
+            torch.cuda.synchronize()
+            ms = a.elapsed_time(b)
+            best = ms if best is None else min(best, ms)
+        return nbytes / (best / 1e3) / 1e9
+
+    return {"h2d_gbs_alone": timed(False), "h2d_gbs_with_d2h": timed(True), "bytes": int(nbytes),
+            "how": "pinned host -> device copy of %d cache slabs, best of %d, alone and beside a device -> host "
+                   "copy of the same size" % (n - lo, reps)}
+
+
 def scoring_roofline(wl, pp, cuq, score_ms_per_step, sm_mhz=None):
     """Useful tensor work of the scoring stage: one Q K^T over the multimodal keys per
     step and sequence (2 n_q Hq |S| D flop, summed over the sequences of the batch).  The two-pass softmax computes Q K^T twice and every
@@ -813,6 +846,7 @@ def main():
         clocks.mark(False)
         clocks.stop()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dist, "cuda")
+    link = link_rates(h_k, h_v, pp2, s_up, s_down)
     del pp2, sets
 
     # the pre-LLM stage of the same clip, timed on its own after the prune steps
@@ -866,7 +900,9 @@ def main():
                                 "kept rows over the host link (its own stream), the later steps run on the device; "
                                 "two device buffer sets let the next iteration's upload, scoring and selection and "
                                 "the previous read-back run while the current gather holds the link",
-                    "h2d_note": "h2d_bytes_per_step counts the copies and the kept rows read from host memory"},
+                    "h2d_note": "h2d_bytes_per_step counts the copies and the kept rows read from host memory",
+                    "h2d_gbs": h2d / (e2e_ms / 1e3) / 1e9, "link": link,
+                    "frac_of_link": (h2d / (e2e_ms / 1e3) / 1e9) / link["h2d_gbs_alone"]},
             "clocks": clock_summary or None,
             "context": schedule_context(wl, pp),
         }
