@@ -741,11 +741,13 @@ def main():
 
     # end to end through the C ABI with host buffers: the caches of layers [l_0, L) and the hidden
     # states stay in pinned host memory.  Every iteration copies the scored layer's keys, the
-    # queries and the modality to the device, scores and selects there, gathers only the kept
-    # rows of every plane over the host link (apack_compact from a host source), runs the later
-    # steps on the device and reads the result back.  Two device buffer sets let iteration
-    # i+1's upload (copy stream) run while iteration i computes and while iteration i-1's result
-    # is read back (third stream): the link carries both directions.
+    # queries and the modality to the device and runs the schedule from the host caches
+    # (ProgressivePrune.host_step): each step scores and selects on the device and gathers over
+    # the host link, at the composed indices, only the layers that end at its level (and the keys
+    # the next step scores), so every layer's rows cross the link once.  The result (the last
+    # step's layers, the hidden states, the indices) is read back.  Two device buffer sets let
+    # iteration i+1's upload and first selection run while iteration i's gathers hold the link,
+    # and iteration i-1's result is read back on a third stream: the link carries both directions.
     e2e_steps = args.e2e_steps or max(3, min(args.steps, 20))
     pp2 = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
                            wl.prune_layers, counts, select_mode=mode)
@@ -760,8 +762,11 @@ def main():
         a.copy_(b)
     last = nsteps - 1
 
+    for p in sets:
+        p._final_buffers()
+
     def host_outputs(p):
-        ko, vo = p.output_kv(last)
+        ko, vo = p.final_kv(last)
         ho = p.output_hidden(last)
         return ([torch.empty(ko.shape, dtype=ko.dtype, pin_memory=True),
                  torch.empty(vo.shape, dtype=vo.dtype, pin_memory=True),
@@ -769,15 +774,17 @@ def main():
                 [torch.empty(int(t), dtype=torch.int32, pin_memory=True) for t in p.t_out])
 
     h_out = [host_outputs(p) for p in sets]
-    # bytes over the link per iteration: the copies (scored keys, modality, queries) and the kept
-    # rows the compaction reads from host memory
-    h2d = (h_k[0].numel() * h_k.element_size() + h_m.numel() + sum(x.numel() * x.element_size() for x in h_q) +
-           pp.t_out[0] * (2 * h_k.shape[0] * pp.row + pp.H * 2))
+    # bytes over the link per iteration: the copies (scored keys, modality, queries) and the rows
+    # the gathers read from host memory (step i: the V of its layers, their K but for its scored
+    # layer's after step 0, the next step's scored keys; step 0 also the hidden states)
+    h2d = h_k[0].numel() * h_k.element_size() + h_m.numel() + sum(x.numel() * x.element_size() for x in h_q)
+    for i in range(nsteps):
+        c = pp.fin_layers[i]
+        planes = 2 * c - (1 if i > 0 else 0) + (1 if i + 1 < nsteps else 0)
+        h2d += pp.t_out[i] * (planes * pp.row + (pp.H * 2 if i == 0 else 0))
     d2h = sum(x.numel() * x.element_size() for x in h_out[0])
     s_up, s_gather, s_down = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
     ev_up = [torch.cuda.Event() for _ in sets]
-    ev_sel = [torch.cuda.Event() for _ in sets]
-    ev_gath = [torch.cuda.Event() for _ in sets]
     ev_comp = [torch.cuda.Event() for _ in sets]
     ev_down = [torch.cuda.Event() for _ in sets]
     for e in ev_down:
@@ -795,24 +802,18 @@ def main():
                 a.copy_(qh, non_blocking=True)
             ev_up[b].record(s_up)
         stream.wait_event(ev_up[b])
-        p.select_first_step(stream=stream)
-        ev_sel[b].record(stream)
-        with torch.cuda.stream(s_gather):      # the link-bound gather runs beside the device work
-            s_gather.wait_event(ev_sel[b])
-            p.compact_first_step_from_host(h_k, h_v, h_h, stream=s_gather)
-            ev_gath[b].record(s_gather)
+        p.host_step(0, h_k, h_v, h_h, stream=stream, gather_stream=s_gather)
 
     def back(j):
         """The later steps and the read-back of iteration j."""
         b = j % 2
         p = sets[b]
-        stream.wait_event(ev_gath[b])
         for i in range(1, nsteps):
-            p.run_step(i, stream=stream)
+            p.host_step(i, h_k, h_v, h_h, stream=stream, gather_stream=s_gather)
         ev_comp[b].record(stream)
         with torch.cuda.stream(s_down):
             s_down.wait_event(ev_comp[b])
-            ko, vo = p.output_kv(last)
+            ko, vo = p.final_kv(last)
             o = h_out[b]
             o[0].copy_(ko, non_blocking=True); o[1].copy_(vo, non_blocking=True)
             o[2].copy_(p.output_hidden(last), non_blocking=True)
@@ -896,10 +897,13 @@ def main():
             "e2e": {"value": whole_job_value(mm_per_iter, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps,
                     "pipeline": "caches and hidden states in pinned host memory; per iteration the scored layer's "
-                                "keys, the queries and the modality are copied, the first compaction reads only the "
-                                "kept rows over the host link (its own stream), the later steps run on the device; "
-                                "two device buffer sets let the next iteration's upload, scoring and selection and "
-                                "the previous read-back run while the current gather holds the link",
+                                "keys, the queries and the modality are copied; every step scores and selects on the "
+                                "device and gathers over the host link (its own stream), at the composed indices, "
+                                "the layers that end at its level plus the keys the next step scores, so each "
+                                "layer's rows cross the link once; the result is every layer's final cache on the "
+                                "device, of which the last step's layers, the hidden states and the indices are read "
+                                "back; two device buffer sets let the next iteration's upload and first selection "
+                                "and the previous read-back run while the current gathers hold the link",
                     "h2d_note": "h2d_bytes_per_step counts the copies and the kept rows read from host memory",
                     "h2d_gbs": h2d / (e2e_ms / 1e3) / 1e9, "link": link,
                     "frac_of_link": (h2d / (e2e_ms / 1e3) / 1e9) / link["h2d_gbs_alone"]},

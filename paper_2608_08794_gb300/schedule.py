@@ -20,6 +20,15 @@ from . import (Seqs, apack_plane, apack_prune_step, apack_prune_schedule, apack_
                APACK_HEAD_DIM, APACK_SELECT_PER_MODALITY, APACK_SELECT_JOINT)
 
 
+def _wait(waiter, producer):
+    """Orders `waiter` after the work queued so far on `producer` (torch streams or None)."""
+    w = waiter if waiter is not None else torch.cuda.current_stream()
+    p = producer if producer is not None else torch.cuda.current_stream()
+    ev = torch.cuda.Event()
+    ev.record(p)
+    w.wait_event(ev)
+
+
 def _plane(src, dst, src_plane_stride, dst_plane_stride, row_bytes, num_planes):
     return apack_plane(src=src, dst=dst, src_plane_stride=src_plane_stride, dst_plane_stride=dst_plane_stride,
                        src_row_stride=row_bytes, dst_row_stride=row_bytes, row_bytes=row_bytes,
@@ -222,6 +231,99 @@ class ProgressivePrune:
         if len(self.new_cu) != len(self.layers):
             self.new_cu = [None] * len(self.layers)
         self.new_cu[0] = new_cu
+
+    def _final_buffers(self):
+        """Buffers of run_from_host, allocated on first use: every layer's cache at the level it
+        ends at (k_fin[i] / v_fin[i]: layers [l_i, l_(i+1)) at t_out_i rows), the scored keys of
+        each later step at the level that step reads (k_score[i]: layer l_i at t_out_(i-1) rows)
+        and the composed row indices into the step-0 input (comp[i], i >= 1)."""
+        if getattr(self, "k_fin", None) is not None:
+            return
+        n = len(self.layers)
+        ends = self.layers[1:] + [self.L]
+        self.fin_layers = [e - l for l, e in zip(self.layers, ends)]
+        self.k_fin = [torch.empty((c, max(1, t), self.hkv, APACK_HEAD_DIM), dtype=torch.bfloat16, device=self.dev)
+                      for c, t in zip(self.fin_layers, self.t_out)]
+        self.v_fin = [torch.empty_like(k) for k in self.k_fin]
+        self.k_score = [None] + [torch.empty((max(1, self.t_out[i - 1]), self.hkv, APACK_HEAD_DIM),
+                                             dtype=torch.bfloat16, device=self.dev) for i in range(1, n)]
+        self.comp = [None] + [torch.empty(max(1, t), dtype=torch.int32, device=self.dev) for t in self.t_out[1:]]
+
+    def run_from_host(self, k_host, v_host, hidden_host=None, stream=None, gather_stream=None):
+        """The whole schedule with the K/V caches of layers [l_0, L) and the hidden states in pinned
+        host memory (laid out like k_in / v_in / hidden_in; the caller copies the scored keys,
+        slab 0 of k_in, to the device).  Every layer's rows cross the host link once, at the level
+        that layer ends at: step i gathers, at the composed indices of steps 0..i, the K and V of
+        layers [l_i, l_(i+1)) and the keys that step i+1 scores (layer l_(i+1)).  Only the scored
+        keys of step i (already on the device) and the hidden states are compacted on the device.
+        Scoring and selection are those of run_step, so keep_idx, scores and the caches equal the
+        per-step schedule's bit for bit; the result is every layer's final cache (final_kv),
+        output_hidden(last) and keep_idx.  gather_stream: None, or a stream for the host-link
+        gathers (ordered against `stream` with events)."""
+        for i in range(len(self.layers)):
+            self.host_step(i, k_host, v_host, hidden_host, stream=stream, gather_stream=gather_stream)
+
+    def host_step(self, i, k_host, v_host, hidden_host=None, stream=None, gather_stream=None):
+        """Step i of run_from_host (steps run in order; step 0 needs the scored keys in slab 0 of
+        k_in).  After the last step, `stream` is ordered after every gather."""
+        if self.slice_below or self.in_place:
+            raise ValueError("run_from_host: slice_below and in_place are not supported")
+        self._final_buffers()
+        n, row, T0 = len(self.layers), self.row, self.T0
+        gs = gather_stream if gather_stream is not None else stream
+        kh, vh = k_host.data_ptr(), v_host.data_ptr()
+        if len(self.new_cu) != n:
+            self.new_cu = [None] * n
+        other = np.diff(self.cu0) - self.na0 - self.nv0
+        seqs = self._step_seqs(i)
+        t = self.t_out[i]
+        k_sc = self.k_in.view(-1) if i == 0 else self.k_score[i]
+        if i > 0 and gs is not stream:
+            _wait(stream, gs)                  # the scored keys came over the link
+        apack_score(seqs, self.q[i], k_sc, row, self.scores, self.ws, stream=stream)
+        apack_select(seqs, self.scores, self.counts[i], self.keep_idx[i], self.ws, select_mode=self.mode,
+                     modality_out=self.mod_out[i % 2], stream=stream)
+        if i > 0:                              # rows of the step-0 input that step i keeps
+            prev = self.keep_idx[0] if i == 1 else self.comp[i - 1]
+            apack_compact(self.keep_idx[i], t, [make_plane(prev, self.comp[i], 4, 1)], stream=stream)
+        comp = self.keep_idx[0] if i == 0 else self.comp[i]
+        # host-link gathers of this step, at the composed indices
+        l0, li = self.layers[0], self.layers[i]
+        c = self.fin_layers[i]
+        kf, vf = self.k_fin[i].data_ptr(), self.v_fin[i].data_ptr()
+        planes = [_plane(vh + (li - l0) * T0 * row, vf, T0 * row, t * row, row, c)]
+        k_first = 0 if i == 0 else 1           # layer l_i's keys of a later step come from the device
+        if c > k_first:
+            planes.append(_plane(kh + (li - l0 + k_first) * T0 * row, kf + k_first * t * row, T0 * row,
+                                 t * row, row, c - k_first))
+        if i + 1 < n:
+            planes.append(_plane(kh + (self.layers[i + 1] - l0) * T0 * row, self.k_score[i + 1].data_ptr(),
+                                 T0 * row, t * row, row, 1))
+        if i == 0 and hidden_host is not None and self.h_out[0] is not None:
+            planes.append(make_plane(hidden_host, self.h_out[0], self.H * 2, 1))
+        if gs is not stream:
+            _wait(gs, stream)
+        apack_compact(comp, t, planes, ws=self.ws, stream=gs)
+        if i > 0:                              # device-side: the scored keys and the hidden states
+            dev_planes = [_plane(self.k_score[i].data_ptr(), kf, 0, 0, row, 1)]
+            h_prev, h_new = self.h_out[(i - 1) % 2], self.h_out[i % 2]
+            if h_prev is not None and (i > 1 or hidden_host is not None):
+                if i == 1 and gs is not stream:
+                    _wait(stream, gs)          # the step-0 hidden rows came over the link
+                dev_planes.append(make_plane(h_prev, h_new, self.H * 2, 1))
+            apack_compact(self.keep_idx[i], t, dev_planes, ws=self.ws, stream=stream)
+        k = self.counts[i]
+        cu = np.zeros(self.B + 1, np.int32)
+        cu[1:] = np.cumsum(other + k[:, 0] + k[:, 1])
+        self.new_cu[i] = cu
+        if i + 1 == n and gs is not stream:
+            _wait(stream, gs)
+
+    def final_kv(self, i):
+        """run_from_host's caches of layers [l_i, l_(i+1)) (the last step: [l_i, L)) at their final
+        level: [n_layers, t_out_i, Hkv, D] K and V."""
+        t = self.t_out[i]
+        return self.k_fin[i][:, :t], self.v_fin[i][:, :t]
 
     def run_steps(self, events=None, stream=None):
         """Runs every step with one apack_prune_step call each; events[i] = 4 CUDA

@@ -314,6 +314,73 @@ def test_first_step_from_host_caches_is_bit_identical(ap, name):
     same(ref, snapshot(pp))
 
 
+@pytest.mark.parametrize("name,streams", [("3b_60s", 1), ("7b_2min", 2), ("7b_ragged16", 2),
+                                          ("7b_10min_paper", 2)])
+def test_schedule_from_host_caches_gathers_each_layer_at_its_final_level(ap, name, streams):
+    """run_from_host: caches in pinned host memory, every layer's rows gathered over the host
+    link once, at the level that layer ends at.  Each step's indices, offsets, modality and the
+    final hidden states equal the per-step device schedule's bit for bit, and every layer's final
+    cache equals its own step's device output and the original rows at the composed indices
+    (oracle compact_rows)."""
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+
+    wl = workload(name)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod_d = torch.from_numpy(wl.modality()).cuda()
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_d,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
+    pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                          wl.prune_layers, counts, select_mode=mode)
+    fill_progressive_inputs(pp, wl)
+    n = len(pp.layers)
+    ends = list(pp.layers[1:]) + [pp.L]
+    ref_kv, ref_m = [], []
+    for i in range(n):                           # the device schedule, one step at a time
+        pp.run_step(i)
+        k, v = pp.output_kv(i)
+        c = ends[i] - pp.layers[i]
+        ref_kv.append((k[:c].clone(), v[:c].clone()))
+        ref_m.append(pp.mod_out[i % 2][:pp.t_out[i]].clone())
+    torch.cuda.synchronize()
+    ref_keep = [pp.keep_idx[i][:pp.t_out[i]].clone() for i in range(n)]
+    ref_cu = [np.asarray(c).copy() for c in pp.new_cu]
+    ref_h = pp.output_hidden(n - 1).clone()
+    h_k = pp.k_in.cpu().pin_memory()
+    h_v = pp.v_in.cpu().pin_memory()
+    h_h = pp.hidden_in.cpu().pin_memory()
+    for buf in pp.k_out + pp.v_out + pp.h_out + pp.mod_out + pp.keep_idx:
+        buf.zero_()
+    pp.k_in[1:].zero_()                          # only the scored layer's keys stay on the device
+    pp.v_in.zero_()
+    pp.hidden_in.zero_()
+    side = torch.cuda.Stream() if streams == 2 else None
+    pp.run_from_host(h_k, h_v, h_h, gather_stream=side)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+    for i in range(n):
+        assert torch.equal(pp.keep_idx[i][:pp.t_out[i]], ref_keep[i]), i
+        np.testing.assert_array_equal(pp.new_cu[i], ref_cu[i])
+    assert torch.equal(pp.mod_out[(n - 1) % 2][:pp.t_out[n - 1]], ref_m[n - 1])
+    assert torch.equal(pp.output_hidden(n - 1).view(torch.int16), ref_h.view(torch.int16))
+    k_np, v_np = h_k.view(torch.int16).numpy(), h_v.view(torch.int16).numpy()
+    comp = np.arange(pp.T0)
+    for i in range(n):
+        comp = comp[pp.keep_idx[i][:pp.t_out[i]].cpu().numpy()]
+        k, v = pp.final_kv(i)
+        assert torch.equal(k.view(torch.int16), ref_kv[i][0].view(torch.int16)), i
+        assert torch.equal(v.view(torch.int16), ref_kv[i][1].view(torch.int16)), i
+        l0 = pp.layers[i] - pp.layers[0]
+        for j in (0, k.shape[0] - 1):            # first and last layer of the step's range
+            np.testing.assert_array_equal(k[j].view(torch.int16).cpu().numpy(),
+                                          oracle.compact_rows(k_np[l0 + j], comp))
+            np.testing.assert_array_equal(v[j].view(torch.int16).cpu().numpy(),
+                                          oracle.compact_rows(v_np[l0 + j], comp))
+
+
 @pytest.mark.parametrize("name", ["7b_2min", "7b_10min_paper"])
 def test_slicing_below_the_pruning_layers_keeps_every_layer_consistent(ap, name):
     """With slice_below, every step also compacts the caches of the layers below its
