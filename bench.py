@@ -783,6 +783,11 @@ def main():
         planes = 2 * c - (1 if i > 0 else 0) + (1 if i + 1 < nsteps else 0)
         h2d += pp.t_out[i] * (planes * pp.row + (pp.H * 2 if i == 0 else 0))
     d2h = sum(x.numel() * x.element_size() for x in h_out[0])
+    # the device work of the e2e pipeline runs on a stream of the highest priority, so that its
+    # kernels take SMs as soon as CTAs of the link-bound gather (default priority) retire
+    stream_dev = stream
+    stream = torch.cuda.Stream(priority=torch.cuda.Stream.priority_range()[1])
+    stream.wait_stream(stream_dev)
     s_up, s_gather, s_down = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
     ev_up = [torch.cuda.Event() for _ in sets]
     ev_comp = [torch.cuda.Event() for _ in sets]
@@ -848,6 +853,8 @@ def main():
         clocks.stop()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dist, "cuda")
     link = link_rates(h_k, h_v, pp2, s_up, s_down)
+    stream_dev.wait_stream(stream)
+    stream = stream_dev
     del pp2, sets
 
     # the pre-LLM stage of the same clip, timed on its own after the prune steps

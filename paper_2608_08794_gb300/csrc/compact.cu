@@ -69,8 +69,13 @@ __global__ void __launch_bounds__(32) gather_tma_kernel(const __grid_constant__ 
 // ------------------------------------------------------------------ host source
 // Source rows in pinned host memory (zero copy): only the kept rows cross the host link.
 // Consecutive threads take consecutive 16-byte pieces of a row (coalesced link reads); each
-// thread issues U loads before its U stores so that enough reads are in flight.
+// thread issues U loads before its U stores so that enough reads are in flight.  Every CTA moves
+// a fixed 64 KB and exits (no grid-stride loop): CTAs of kernels on other streams (scoring and
+// selection beside a link-bound gather) then get SMs as soon as gather CTAs retire, first when
+// their stream has the higher priority.
 constexpr int kHostUnroll = 4;
+constexpr int kHostRounds = 4;
+constexpr int64_t kHostPiecesPerCta = 256 * kHostUnroll * kHostRounds;   // 16-byte pieces
 
 __global__ void __launch_bounds__(256) gather_host_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst,
                                                           int64_t sps, int64_t dps, int64_t srs, int64_t drs,
@@ -78,13 +83,14 @@ __global__ void __launch_bounds__(256) gather_host_kernel(const uint8_t *__restr
                                                           const int32_t *__restrict__ keep_idx) {
   const int64_t vec_per_row = row_bytes / 16;
   const int64_t total = n_planes * n_out * vec_per_row;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t base = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; base < total;
-       base += stride * kHostUnroll) {
+  const int64_t cta0 = static_cast<int64_t>(blockIdx.x) * kHostPiecesPerCta + threadIdx.x;
+#pragma unroll 1
+  for (int r = 0; r < kHostRounds; ++r) {
+    const int64_t base = cta0 + r * (256 * kHostUnroll);
     uint4 v[kHostUnroll];
 #pragma unroll
     for (int u = 0; u < kHostUnroll; ++u) {
-      const int64_t e = base + u * stride;
+      const int64_t e = base + u * 256;
       if (e < total) {
         const int64_t row = e / vec_per_row, c = e - row * vec_per_row;
         const int64_t plane = row / n_out, j = row - plane * n_out;
@@ -93,7 +99,7 @@ __global__ void __launch_bounds__(256) gather_host_kernel(const uint8_t *__restr
     }
 #pragma unroll
     for (int u = 0; u < kHostUnroll; ++u) {
-      const int64_t e = base + u * stride;
+      const int64_t e = base + u * 256;
       if (e < total) {
         const int64_t row = e / vec_per_row, c = e - row * vec_per_row;
         const int64_t plane = row / n_out, j = row - plane * n_out;
@@ -189,6 +195,9 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
       // pinned host source: zero-copy gather (destination in device memory, never in place)
       if (p.src == p.dst || host_source(p.dst)) return APACK_EINVAL;
       if (n_host == kMaxGroups * 4) return APACK_EINVAL;
+      if (widest_unit(p) == 16 && static_cast<int64_t>(p.num_planes) * n_out * (p.row_bytes / 16) >
+                                      0x7FFFFFFFLL * kHostPiecesPerCta)
+        return APACK_EUNSUPPORTED;                  // beyond one launch's grid
       host_groups[n_host] = p;
       host_groups[n_host].src = hs;
       ++n_host;
@@ -236,9 +245,7 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
     const apack_plane &p = host_groups[k];
     if (widest_unit(p) == 16) {
       const int64_t n = static_cast<int64_t>(p.num_planes) * n_out * (p.row_bytes / 16);
-      int64_t blocks = (n + 256 * kHostUnroll - 1) / (256 * kHostUnroll);
-      const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
-      if (blocks > cap) blocks = cap;
+      const int64_t blocks = (n + kHostPiecesPerCta - 1) / kHostPiecesPerCta;   // checked when planned
       gather_host_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
           static_cast<const uint8_t *>(p.src), static_cast<uint8_t *>(p.dst), p.src_plane_stride, p.dst_plane_stride,
           p.src_row_stride, p.dst_row_stride, p.row_bytes, p.num_planes, n_out, keep_idx);
