@@ -115,7 +115,7 @@ def host_cpu():
     return {"cpu_model": model or platform.processor() or platform.machine(), "nproc": os.cpu_count()}
 
 
-GATHER_SOURCES = ["compact.cu", "compact_plan.cuh"]     # the out-of-place gather and its item plan
+GATHER_SOURCES = ["compact_tma.cu", "compact_plan.cuh"]   # the out-of-place gather and its item plan
 
 
 def source_sha256(kernel_src):

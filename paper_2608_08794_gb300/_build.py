@@ -75,7 +75,7 @@ def build_apack():
     csrc = os.path.join(HERE, "csrc")
     headers = [os.path.join(INCLUDE, "apack.h")] + [
         os.path.join(csrc, h) for h in os.listdir(csrc) if h.endswith((".cuh", ".h"))]
-    return _build_lib(csrc, ["apack.cu", "score.cu", "score_narrow.cu", "score_narrow_tc.cu", "select.cu", "compact.cu", "compact_inplace.cu", "score_static.cu", "prellm.cu", "decode.cu", "decode_tc.cu", "schedule.cu"], headers,
+    return _build_lib(csrc, ["apack.cu", "score.cu", "score_narrow.cu", "score_narrow_tc.cu", "select.cu", "compact.cu", "compact_tma.cu", "compact_inplace.cu", "score_static.cu", "prellm.cu", "decode.cu", "decode_tc.cu", "schedule.cu"], headers,
                       os.path.join(HERE, "_lib"), "libapack.so")
 
 

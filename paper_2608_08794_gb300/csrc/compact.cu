@@ -1,16 +1,14 @@
 // compact.cu -- KV-cache and hidden-state slicing of Sec. 3.2 (Algorithm 1, "slice their
 // KV-cache entries"): dst row j = src row keep_idx[j] for every plane.
 //
-// HBM-bound: every byte is read once and written once.
-//  - TMA kernel (rows of 16-byte multiples up to 32 KB, 16-byte aligned): one
-//    warp per CTA streams kept rows into a ring of 32 KB shared-memory slots
-//    with cp.async.bulk (one row per lane, completion on the slot's mbarrier)
-//    and writes each slot back with a single bulk store when the output rows
-//    are contiguous (one per row otherwise).  Several slots stay in flight per
-//    CTA, so a handful of threads keep the whole HBM pipe busy.
-//  - Rows that are not 16-byte multiples (or misaligned) take the narrow
-//    kernel, one thread per row.
-//  - In place (src == dst): compact_inplace.cu.
+// This file plans a call (validating every group before anything is launched) and holds the
+// small paths; the bulk paths live beside it:
+//  - rows of 16-byte multiples up to 32 KB, 16-byte aligned, out of place: the bulk-copy (TMA)
+//    gather of compact_tma.cu;
+//  - the same rows in place (src == dst): compact_inplace.cu;
+//  - a source in pinned host memory: the zero-copy gather below;
+//  - rows that are not 16-byte multiples (or misaligned): the narrow kernel below, one thread
+//    per row.
 #include "compact_plan.cuh"
 
 namespace apack {
@@ -18,53 +16,6 @@ namespace apack {
 using namespace gather;
 
 namespace {
-
-constexpr int kSlots = 3;                       // slots per CTA (two CTAs per SM)
-constexpr uint32_t kTmaSmem = kSlots * kSlotBytes;
-
-__global__ void __launch_bounds__(32) gather_tma_kernel(const __grid_constant__ TmaPlan plan,
-                                                        const int32_t *__restrict__ keep_idx, DeviceError *err) {
-  extern __shared__ __align__(1024) uint8_t slots[];
-  __shared__ __align__(8) uint64_t full[kSlots];
-  const int lane = threadIdx.x;
-  if (lane == 0) {
-    for (int i = 0; i < kSlots; ++i) mbar_init(&full[i], 1);
-    fence_mbar_init();
-  }
-  __syncwarp();
-  // this CTA's items: blockIdx.x, blockIdx.x + gridDim.x, ...
-  const uint32_t first = blockIdx.x, stride = gridDim.x;
-  const uint32_t n_mine = first < plan.total_items ? (plan.total_items - first + stride - 1) / stride : 0;
-  uint32_t issued = n_mine < kSlots ? n_mine : kSlots;   // positions whose loads were issued
-  for (uint32_t j = 0; j < issued; ++j)
-    load_item(decode_item(plan, first + j * stride), slots + j * kSlotBytes, &full[j], keep_idx, lane);
-  bool ok = true;
-  uint32_t j = 0;
-  for (; j < n_mine; ++j) {
-    const int slot = j % kSlots;
-    const Item it = decode_item(plan, first + j * stride);
-    if (!mbar_wait(&full[slot], (j / kSlots) & 1u, kWaitLimitNs)) {
-      if (lane == 0 && err) raise_device_error(err, APACK_ETIMEOUT, 41);
-      ok = false;
-      break;
-    }
-    fence_proxy_async_smem();
-    store_item(it, slots + slot * kSlotBytes, lane);
-    // refill the slot whose store was issued one item ago, once that store has read it
-    if (j >= 1 && j - 1 + kSlots < n_mine) {
-      bulk_wait_read<1>();
-      const uint32_t k = j - 1 + kSlots;
-      const int ks = k % kSlots;
-      load_item(decode_item(plan, first + k * stride), slots + ks * kSlotBytes, &full[ks], keep_idx, lane);
-      issued = k + 1;
-    }
-  }
-  if (!ok) {
-    // loads of items j .. issued - 1 may still be in flight: wait for them (bounded)
-    for (uint32_t k = j; k < issued; ++k) mbar_wait(&full[k % kSlots], (k / kSlots) & 1u, kWaitLimitNs / 4);
-  }
-  bulk_wait_all();
-}
 
 // ------------------------------------------------------------------ host source
 // Source rows in pinned host memory (zero copy): only the kept rows cross the host link.
@@ -269,19 +220,8 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
     if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
   }
   if (tp.ngroups > 0) {
-    static bool attr_done = false;
-    if (!attr_done) {
-      if (check_cuda(cudaFuncSetAttribute(gather_tma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          kTmaSmem)) != APACK_OK)
-        return APACK_ECUDA;
-      attr_done = true;
-    }
     tp.total_items = static_cast<uint32_t>(items);
-    uint64_t blocks = static_cast<uint64_t>(device_sm_count()) * 2;   // two CTAs of kSlots slots per SM
-    if (blocks > items) blocks = items;
-    gather_tma_kernel<<<static_cast<unsigned>(blocks), 32, kTmaSmem, stream>>>(tp, keep_idx, err);
-    count_launches(1);
-    if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+    if (launch_out_of_place(tp, keep_idx, err, stream) != APACK_OK) return APACK_ECUDA;
   }
   if (ip.ngroups > 0 && launch_inplace(ip, in_blocks, keep_idx, err, stream) != APACK_OK) return APACK_ECUDA;
   return APACK_OK;

@@ -83,6 +83,10 @@ __device__ __forceinline__ void store_item(const Item &it, const uint8_t *slot, 
   bulk_commit();
 }
 
+// Out of place (compact_tma.cu): tp.total_items set, at least one item.
+apack_status launch_out_of_place(const TmaPlan &tp, const int32_t *keep_idx, DeviceError *err,
+                                 cudaStream_t stream);
+
 // In place (compact_inplace.cu).  plan_inplace sizes the cooperative launch (APACK_EUNSUPPORTED
 // when the items exceed what 16-bit progress words count); launch_inplace zeroes the progress
 // words in the workspace (bytes 256..1023 past err) and launches.
