@@ -307,7 +307,7 @@ class ProgressivePrune:
         if i > 0:                              # device-side: the scored keys and the hidden states
             dev_planes = [_plane(self.k_score[i].data_ptr(), kf, 0, 0, row, 1)]
             h_prev, h_new = self.h_out[(i - 1) % 2], self.h_out[i % 2]
-            if h_prev is not None and (i > 1 or hidden_host is not None):
+            if h_prev is not None and hidden_host is not None:
                 if i == 1 and gs is not stream:
                     _wait(stream, gs)          # the step-0 hidden rows came over the link
                 dev_planes.append(make_plane(h_prev, h_new, self.H * 2, 1))
