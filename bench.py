@@ -417,6 +417,47 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
                          "note": "bf16 tokens read once + fp32 frame embeddings written once, over the whole call"}}
 
 
+def final_levels_measure(ap, pp, nsteps, mm_per_iter, steps, warmup, stream, dist):
+    """The same steps scheduled so that every layer's rows are written once, at the level that
+    layer ends at (ProgressivePrune.run_from_host with the device inputs as its source): step i
+    gathers layers [l_i, l_(i+1)) and the next step's scored keys from the step-0 input at the
+    composed indices.  Same scores, selections and final caches as the per-step schedule (checked
+    here against its last step's output); fewer bytes, because the per-step schedule compacts
+    layers [l_i, L) at every step.  Reported beside the headline, not as it."""
+    import torch
+    lo = pp.layers[0]
+    ref_k, ref_v = [x.clone() for x in pp.output_kv(nsteps - 1)]
+    ref_h = pp.output_hidden(nsteps - 1).clone()
+
+    def run():
+        pp.run_from_host(pp.k_in, pp.v_in, pp.hidden_in, stream=stream)
+
+    for _ in range(max(1, warmup)):
+        run()
+    torch.cuda.synchronize()
+    k, v = pp.final_kv(nsteps - 1)
+    same = (torch.equal(k.view(torch.int16), ref_k.view(torch.int16)) and
+            torch.equal(v.view(torch.int16), ref_v.view(torch.int16)) and
+            torch.equal(pp.output_hidden(nsteps - 1).view(torch.int16), ref_h.view(torch.int16)))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        run()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1) / steps, dist, "cuda")
+    moved = 0                         # read + write of every gathered row, 4 B index per kept row
+    for i in range(nsteps):
+        c, t = pp.fin_layers[i], pp.t_out[i]
+        planes = 2 * c + (1 if i + 1 < nsteps else 0)
+        moved += 2 * t * (planes * pp.row + pp.H * 2) + 4 * t
+    return {"value": mm_per_iter / (ms / 1e3), "unit": UNIT, "ms_per_step": ms, "steps": steps,
+            "bytes_moved_per_iter": int(moved), "equal_to_per_step_schedule": bool(same),
+            "how": "eager calls (no graph); every layer's K/V written once at its final level from the step-0 "
+                   "input, the scored keys and the hidden states compacted per step; the per-step schedule "
+                   "of the headline compacts layers [l_i, L) at every step"}
+
+
 def link_rates(h_k, h_v, pp2, s_up, s_down, reps=3):
     """The host link's rate on this machine, measured beside the e2e run: pinned host -> device
     copies of up to 7 cache slabs alone, and the same copies while device -> host copies of as
@@ -738,6 +779,7 @@ def main():
     g_launches = ap.apack_launch_count() - g_launch0
     graph_ms = max_over_ranks(g_start.elapsed_time(g_end) / args.steps, dist, "cuda")
     graph.close()
+    final_levels = final_levels_measure(ap, pp, nsteps, mm_per_iter, args.steps, args.warmup, stream, dist)
 
     # end to end through the C ABI with host buffers: the caches of layers [l_0, L) and the hidden
     # states stay in pinned host memory.  Every iteration copies the scored layer's keys, the
@@ -901,6 +943,8 @@ def main():
                       "ms_per_step": eager_ms, "gpu_launches": int(launches),
                       "how": "one apack_prune_schedule call per iteration with stage events; stages_ms_per_iter "
                              "and the compaction roofline come from this run"},
+            "schedule_final_levels": dict(final_levels, value=whole_job_value(mm_per_iter, world,
+                                                                              final_levels["ms_per_step"])),
             "e2e": {"value": whole_job_value(mm_per_iter, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps,
                     "pipeline": "caches and hidden states in pinned host memory; per iteration the scored layer's "

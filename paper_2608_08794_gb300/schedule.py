@@ -259,7 +259,9 @@ class ProgressivePrune:
         Scoring and selection are those of run_step, so keep_idx, scores and the caches equal the
         per-step schedule's bit for bit; the result is every layer's final cache (final_kv),
         output_hidden(last) and keep_idx.  gather_stream: None, or a stream for the host-link
-        gathers (ordered against `stream` with events)."""
+        gathers (ordered against `stream` with events).  The sources may also be device buffers
+        (k_in, v_in, hidden_in themselves): the same schedule then writes every layer once on the
+        device, where the per-step schedule compacts layers [l_i, L) at every step."""
         for i in range(len(self.layers)):
             self.host_step(i, k_host, v_host, hidden_host, stream=stream, gather_stream=gather_stream)
 

@@ -381,6 +381,47 @@ def test_schedule_from_host_caches_gathers_each_layer_at_its_final_level(ap, nam
                                           oracle.compact_rows(v_np[l0 + j], comp))
 
 
+@pytest.mark.parametrize("name", ["7b_2min", "7b_ragged16"])
+def test_final_level_schedule_from_device_inputs(ap, name):
+    """run_from_host with the device inputs as its source (every layer written once, at its final
+    level, by device gathers): the same indices as the per-step schedule, and every layer's final
+    cache equal to its own step's output, bit for bit."""
+    from paper_2608_08794_gb300.schedule import ProgressivePrune, schedule_keep_counts
+    from synth import workload
+    from synth.device import fill_progressive_inputs
+
+    wl = workload(name)
+    cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
+    na = np.array([s.n_audio for s in wl.seqs], np.int32)
+    nv = np.array([s.n_visual for s in wl.seqs], np.int32)
+    mod_d = torch.from_numpy(wl.modality()).cuda()
+    counts, mode = schedule_keep_counts(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, mod_d,
+                                        len(wl.prune_layers), wl.ratios, wl.joint_step_keep)
+    pp = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                          wl.prune_layers, counts, select_mode=mode)
+    fill_progressive_inputs(pp, wl)
+    n = len(pp.layers)
+    ends = list(pp.layers[1:]) + [pp.L]
+    ref = []
+    for i in range(n):
+        pp.run_step(i)
+        k, v = pp.output_kv(i)
+        c = ends[i] - pp.layers[i]
+        ref.append((pp.keep_idx[i][:pp.t_out[i]].clone(), k[:c].clone(), v[:c].clone()))
+    ref_h = pp.output_hidden(n - 1).clone()
+    for buf in pp.keep_idx + pp.h_out:
+        buf.zero_()
+    pp.run_from_host(pp.k_in, pp.v_in, pp.hidden_in)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(pp.ws) == ap.APACK_OK
+    for i in range(n):
+        k, v = pp.final_kv(i)
+        assert torch.equal(pp.keep_idx[i][:pp.t_out[i]], ref[i][0]), i
+        assert torch.equal(k.view(torch.int16), ref[i][1].view(torch.int16)), i
+        assert torch.equal(v.view(torch.int16), ref[i][2].view(torch.int16)), i
+    assert torch.equal(pp.output_hidden(n - 1).view(torch.int16), ref_h.view(torch.int16))
+
+
 @pytest.mark.parametrize("name", ["7b_2min", "7b_10min_paper"])
 def test_slicing_below_the_pruning_layers_keeps_every_layer_consistent(ap, name):
     """With slice_below, every step also compacts the caches of the layers below its
