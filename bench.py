@@ -446,15 +446,44 @@ def final_levels_measure(ap, pp, nsteps, mm_per_iter, steps, warmup, stream, dis
     e1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(e0.elapsed_time(e1) / steps, dist, "cuda")
+    # the same calls captured once as a CUDA graph (stream capture of the library calls) and replayed
+    graph_ms, graph_error = None, None
+    try:
+        graph = torch.cuda.CUDAGraph()
+        cap = torch.cuda.Stream()
+        cap.wait_stream(stream)
+        with torch.cuda.graph(graph, stream=cap, capture_error_mode="thread_local"):
+            pp.run_from_host(pp.k_in, pp.v_in, pp.hidden_in)
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            for _ in range(max(1, warmup)):
+                graph.replay()
+            torch.cuda.synchronize()
+            g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            g0.record(stream)
+            for _ in range(steps):
+                graph.replay()
+            g1.record(stream)
+            torch.cuda.synchronize()
+        graph_ms = max_over_ranks(g0.elapsed_time(g1) / steps, dist, "cuda")
+        k, v = pp.final_kv(nsteps - 1)
+        same = same and (torch.equal(k.view(torch.int16), ref_k.view(torch.int16)) and
+                         torch.equal(v.view(torch.int16), ref_v.view(torch.int16)))
+        del graph
+    except Exception as exc:  # report, do not hide: the eager number stands alone then
+        graph_error = str(exc)[-300:]
     moved = 0                         # read + write of every gathered row, 4 B index per kept row
     for i in range(nsteps):
         c, t = pp.fin_layers[i], pp.t_out[i]
         planes = 2 * c + (1 if i + 1 < nsteps else 0)
         moved += 2 * t * (planes * pp.row + pp.H * 2) + 4 * t
-    return {"value": mm_per_iter / (ms / 1e3), "unit": UNIT, "ms_per_step": ms, "steps": steps,
-            "bytes_moved_per_iter": int(moved), "equal_to_per_step_schedule": bool(same),
-            "how": "eager calls (no graph); every layer's K/V written once at its final level from the step-0 "
-                   "input, the scored keys and the hidden states compacted per step; the per-step schedule "
+    best = graph_ms if graph_ms is not None else ms
+    return {"value": mm_per_iter / (best / 1e3), "unit": UNIT, "ms_per_step": best, "steps": steps,
+            "eager_ms_per_step": ms, "graph_error": graph_error, "bytes_moved_per_iter": int(moved),
+            "equal_to_per_step_schedule": bool(same),
+            "how": "the library calls of ProgressivePrune.run_from_host captured once as a CUDA graph and replayed "
+                   "(eager_ms_per_step: direct calls); every layer's K/V written once at its final level from the "
+                   "step-0 input, the scored keys and the hidden states compacted per step; the per-step schedule "
                    "of the headline compacts layers [l_i, L) at every step"}
 
 
