@@ -242,16 +242,7 @@ apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num
   const int64_t n_out = new_cu_seqlens_h[seqs->num_seqs];
   if (n_layers > 1 && kv_out_layer_stride < n_out * row) return APACK_EINVAL;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  auto mark = [&](int i) {
-    if (stage_events_h && stage_events_h[i]) cudaEventRecord(static_cast<cudaEvent_t>(stage_events_h[i]), s);
-  };
-  mark(0);
-  st = run_score(seqs, q, k_cache, row, scores, ws, s);
-  if (st != APACK_OK) return st;
-  mark(1);
-  st = run_select(seqs, scores, counts.data(), select_mode, keep_idx, modality_out, nullptr, new_cu_seqlens, ws, s);
-  if (st != APACK_OK) return st;
-  mark(2);
+  // compaction groups: K/V of layers [layer, num_layers), hidden, extra planes
   std::vector<apack_plane> planes;
   planes.reserve(3 + static_cast<size_t>(num_extra));
   apack_plane kp{};
@@ -277,8 +268,21 @@ apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num
     planes.push_back(hp);
   }
   for (int i = 0; i < num_extra; ++i) planes.push_back(extra_planes_h[i]);
-  st = run_compact(keep_idx, n_out, planes.data(), static_cast<int32_t>(planes.size()),
-                   reinterpret_cast<DeviceError *>(static_cast<uint8_t *>(ws) + workspace_layout(seqs).err_off), s);
+  DeviceError *err = reinterpret_cast<DeviceError *>(static_cast<uint8_t *>(ws) + workspace_layout(seqs).err_off);
+  // every argument of the compaction is checked before the first launch of the step
+  st = run_compact(keep_idx, n_out, planes.data(), static_cast<int32_t>(planes.size()), err, s, true);
+  if (st != APACK_OK) return st;
+  auto mark = [&](int i) {
+    if (stage_events_h && stage_events_h[i]) cudaEventRecord(static_cast<cudaEvent_t>(stage_events_h[i]), s);
+  };
+  mark(0);
+  st = run_score(seqs, q, k_cache, row, scores, ws, s);
+  if (st != APACK_OK) return st;
+  mark(1);
+  st = run_select(seqs, scores, counts.data(), select_mode, keep_idx, modality_out, nullptr, new_cu_seqlens, ws, s);
+  if (st != APACK_OK) return st;
+  mark(2);
+  st = run_compact(keep_idx, n_out, planes.data(), static_cast<int32_t>(planes.size()), err, s);
   if (st != APACK_OK) return st;
   mark(3);
   return APACK_OK;

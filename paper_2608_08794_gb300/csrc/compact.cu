@@ -122,7 +122,7 @@ bool ranges_overlap(const apack_plane &p, int64_t n_rows_src, int64_t n_out) {
 }  // namespace
 
 apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes, int32_t num_groups,
-                         DeviceError *err, cudaStream_t stream) {
+                         DeviceError *err, cudaStream_t stream, bool check_only) {
   if (n_out < 0 || num_groups < 0 || (num_groups > 0 && !planes)) return APACK_EINVAL;
   if (n_out == 0 || num_groups == 0) return APACK_OK;
   if (!keep_idx || n_out > INT32_MAX) return APACK_EINVAL;
@@ -192,6 +192,7 @@ apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_pla
     const apack_status st = plan_inplace(ip, in_items, &in_blocks);
     if (st != APACK_OK) return st;
   }
+  if (check_only) return APACK_OK;
   for (int k = 0; k < n_host; ++k) {
     const apack_plane &p = host_groups[k];
     if (widest_unit(p) == 16) {

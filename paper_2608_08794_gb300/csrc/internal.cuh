@@ -100,8 +100,10 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
 apack_status run_select(const apack_seqs *seqs, const float *scores, const int32_t *keep_count_h, int32_t mode,
                         int32_t *keep_idx, uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu_seqlens,
                         void *ws, cudaStream_t stream);
+// check_only: validate and plan every group, launch nothing (callers that launch other
+// kernels first check their compaction this way before any launch).
 apack_status run_compact(const int32_t *keep_idx, int64_t n_out, const apack_plane *planes, int32_t num_groups,
-                         DeviceError *err, cudaStream_t stream);
+                         DeviceError *err, cudaStream_t stream, bool check_only = false);
 // 3-D TMA map over a K slab [tokens][hkv][128] bf16 (token_stride bytes between tokens):
 // boxes of 64 features x 1 head x box_tokens tokens, 128-byte swizzle.
 bool make_kv_tile_map(CUtensorMap *map, const void *k, int hkv, int64_t tokens, int64_t token_stride,

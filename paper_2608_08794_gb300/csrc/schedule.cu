@@ -20,6 +20,7 @@ struct StepPlan {
   apack_seqs seqs{};
   const void *k = nullptr, *v = nullptr, *hidden = nullptr;
   int64_t kv_layer_stride = 0;
+  std::vector<apack_plane> planes;     // the step's compaction groups
 };
 
 apack_plane plane(const void *src, void *dst, int64_t src_ps, int64_t dst_ps, int64_t row, int32_t n) {
@@ -57,6 +58,8 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
   const int64_t row = static_cast<int64_t>(seqs->num_kv_heads) * APACK_HEAD_DIM * 2;
 
   // plan every step on the host first: nothing is launched unless all steps are valid
+  DeviceError *err =
+      ws ? reinterpret_cast<DeviceError *>(static_cast<uint8_t *>(ws) + workspace_layout(seqs).err_off) : nullptr;
   std::vector<StepPlan> plan(static_cast<size_t>(num_steps));
   for (int i = 0; i < num_steps; ++i) {
     const apack_step &sp = steps_h[i];
@@ -109,6 +112,15 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
     // in place: both caches together, with the input's slab stride
     if ((sp.k_out == p.k) != (sp.v_out == p.v) || (sp.k_out == p.k && sp.kv_out_layer_stride != p.kv_layer_stride))
       return APACK_EINVAL;
+    // compaction: K/V of layers [l_i, L), hidden, extra planes, in one launch
+    if (sp.num_extra < 0 || (sp.num_extra > 0 && !sp.extra_planes_h)) return APACK_EINVAL;
+    p.planes.reserve(3 + static_cast<size_t>(sp.num_extra));
+    p.planes.push_back(plane(p.k, sp.k_out, p.kv_layer_stride, sp.kv_out_layer_stride, row, n_layers));
+    p.planes.push_back(plane(p.v, sp.v_out, p.kv_layer_stride, sp.kv_out_layer_stride, row, n_layers));
+    if (p.hidden) p.planes.push_back(plane(p.hidden, sp.hidden_out, 0, 0, hidden_dim * 2, 1));
+    for (int e = 0; e < sp.num_extra; ++e) p.planes.push_back(sp.extra_planes_h[e]);
+    st = run_compact(sp.keep_idx, n_out, p.planes.data(), static_cast<int32_t>(p.planes.size()), err, nullptr, true);
+    if (st != APACK_OK) return st;
   }
 
   cudaStream_t M = static_cast<cudaStream_t>(stream);
@@ -116,7 +128,6 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
     if (stage_events_h && stage_events_h[4 * step + k])
       cudaEventRecord(static_cast<cudaEvent_t>(stage_events_h[4 * step + k]), M);
   };
-  DeviceError *err = reinterpret_cast<DeviceError *>(static_cast<uint8_t *>(ws) + workspace_layout(seqs).err_off);
   for (int i = 0; i < num_steps; ++i) {
     const apack_step &sp = steps_h[i];
     const StepPlan &p = plan[i];
@@ -128,17 +139,8 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
                     sp.new_cu_seqlens, ws, M);
     if (st != APACK_OK) return st;
     mark(i, 2);
-    // compaction: K/V of layers [l_i, L), hidden, extra planes, in one launch
-    const int64_t n_out = sp.new_cu_seqlens_h[B];
-    const int32_t n_layers = num_layers - sp.layer;
-    const int64_t ps_in = p.kv_layer_stride, ps_out = sp.kv_out_layer_stride;
-    std::vector<apack_plane> planes;
-    planes.reserve(3 + static_cast<size_t>(sp.num_extra));
-    planes.push_back(plane(p.k, sp.k_out, ps_in, ps_out, row, n_layers));
-    planes.push_back(plane(p.v, sp.v_out, ps_in, ps_out, row, n_layers));
-    if (p.hidden) planes.push_back(plane(p.hidden, sp.hidden_out, 0, 0, hidden_dim * 2, 1));
-    for (int e = 0; e < sp.num_extra; ++e) planes.push_back(sp.extra_planes_h[e]);
-    st = run_compact(sp.keep_idx, n_out, planes.data(), static_cast<int32_t>(planes.size()), err, M);
+    st = run_compact(sp.keep_idx, sp.new_cu_seqlens_h[B], p.planes.data(), static_cast<int32_t>(p.planes.size()),
+                     err, M);
     if (st != APACK_OK) return st;
     mark(i, 3);
   }

@@ -35,6 +35,10 @@ extern "C" apack_status apack_score_static(const apack_seqs *seqs, const void *q
   int64_t T = 0, NQ = 0;
   apack_status st = validate_seqs(seqs, &T, &NQ);
   if (st != APACK_OK) return st;
+  // Pointer checks come before any device work, as in apack_score: q and k are
+  // read by TMA, so they must be device memory.
+  if (!q || !k || !scores) return APACK_EINVAL;
+  if (in_host_memory(k) || in_host_memory(q)) return APACK_EINVAL;
   // The whole scratch of the batch must fit the fixed array.
   if (workspace_layout(seqs).total > kStaticScratchBytes) return APACK_EWORKSPACE;
   int dev = -1;

@@ -99,6 +99,10 @@ def test_calls_reject_bad_arguments_before_the_device(ap):
     with pytest.raises(ap.ApackError) as e:
         ap.apack_score(s, ws_small, ws_small, 1024, ws_small, ws_small, stream=0)
     assert e.value.status == ap.APACK_EWORKSPACE
+    # the fixed-scratch scorer checks its pointers before it touches a device
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_score_static(s, None, ws_small, 1024, ws_small, stream=0)
+    assert e.value.status == ap.APACK_EINVAL
     with pytest.raises(ap.ApackError) as e:
         ap.apack_select(s, ws_small, np.array([[11, 0], [0, 0]]), ws_small, ws_small, stream=0)
     assert e.value.status in (ap.APACK_EINVAL, ap.APACK_EWORKSPACE)
@@ -122,3 +126,39 @@ def test_calls_reject_bad_arguments_before_the_device(ap):
         ap.apack_compact(t, 4, [ap.make_plane(t, t, 256, 2, 1024, 512)], ws=ws, stream=0)
     assert e.value.status == ap.APACK_EINVAL
     assert ap.status_string(ap.APACK_ETIMEOUT) == "device wait timed out"
+
+
+def test_step_and_schedule_check_their_compaction_before_any_launch(ap):
+    # A bad compaction group (a row wider than its stride) is refused while the
+    # call is planned: with no GPU, a call that reached its first launch would
+    # report a CUDA error instead of APACK_EINVAL.
+    import torch  # noqa: F401  (CPU tensors only: pointers are never dereferenced)
+    s = make_seqs(ap)
+    s.struct.modality = 0x1000
+    n = ap.apack_workspace_size(s)
+    ws = torch.zeros(n + 256, dtype=torch.uint8)
+    off = (-ws.data_ptr()) % 256
+    ws = ws[off:off + n]
+    T, row = 65, 4 * 128 * 2
+    kv = torch.zeros(2 * T * row, dtype=torch.uint8)
+    out = torch.zeros(2 * T * row, dtype=torch.uint8)
+    small = torch.zeros(4096, dtype=torch.int32)
+    bad = ap.make_plane(small, out, 64, src_row_stride=32, dst_row_stride=64)
+    counts = np.array([[5, 10], [2, 6]])
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_prune_step(s, 26, 28, small, kv, kv, T * row, None, 0, keep_count=counts, k_out=out, v_out=out,
+                            kv_out_layer_stride=T * row, extra_planes=[bad], modality_out=small, keep_idx=small,
+                            scores=small, ws=ws, stream=0)
+    assert e.value.status == ap.APACK_EINVAL
+    step = dict(layer=26, q=small, keep_count=counts, k_out=out, v_out=out, kv_out_layer_stride=T * row,
+                modality_out=small, keep_idx=small, extra_planes=[bad])
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_prune_schedule(s, 28, kv, kv, T * row, None, 0, [step], scores=small, ws=ws, stream=0)
+    assert e.value.status == ap.APACK_EINVAL
+    # the same calls with a valid group get past planning and fail only at the device
+    good = ap.make_plane(small, out, 64, src_row_stride=64, dst_row_stride=64)
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_prune_step(s, 26, 28, small, kv, kv, T * row, None, 0, keep_count=counts, k_out=out, v_out=out,
+                            kv_out_layer_stride=T * row, extra_planes=[good], modality_out=small, keep_idx=small,
+                            scores=small, ws=ws, stream=0)
+    assert e.value.status == ap.APACK_ECUDA

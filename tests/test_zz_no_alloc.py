@@ -83,3 +83,16 @@ def test_static_scratch_rejects_batches_over_its_limit(ap):
         ap.apack_score_static(seqs, q, k, stride, out)
     assert e.value.status == ap.APACK_EWORKSPACE
     assert not out.any()
+
+
+def test_static_scratch_refuses_host_keys_before_any_device_work(ap):
+    # the keys are read by TMA, so pinned host memory is refused as apack_score
+    # refuses it, and nothing is written
+    seqs, q, k, stride, T, _ = _inputs(ap, "tiny")
+    out = torch.zeros(T, dtype=torch.float32, device="cuda")
+    k_host = k.cpu().pin_memory()
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_score_static(seqs, q, k_host, stride, out)
+    assert e.value.status == ap.APACK_EINVAL
+    torch.cuda.synchronize()
+    assert not out.any()
