@@ -185,7 +185,10 @@ apack_status apack_compact(const int32_t *keep_idx, int64_t n_out, const apack_p
    returns (no device synchronisation needed).
    scores (device [T] fp32) receives the relevance scores.
    stage_events_h: NULL, or 4 cudaEvent_t recorded on `stream` before
-   scoring, before selection, before compaction and at the end. */
+   scoring, before selection, before compaction and at the end.
+   Every argument, the compaction groups included, is checked before the
+   first launch: a status other than APACK_OK and APACK_ECUDA means nothing
+   was queued on `stream`. */
 apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num_layers,
                               const void *q, const void *k_cache, const void *v_cache,
                               int64_t kv_layer_stride, const void *hidden, int64_t hidden_dim,
@@ -245,7 +248,8 @@ apack_status apack_frame_alignment(const void *visual, const void *audio, int32_
    modality_out, new_cu_seqlens_h, and the counts kept as the new audio/visual
    counts; (|S|, 0) in joint mode).  Layers are strictly ascending.  Each step
    needs its own keep_idx; outputs of step i+1 may reuse step i-1's buffers
-   (ping-pong).  All steps are checked on the host before the first launch;
+   (ping-pong).  All steps (queries and compaction groups included) are
+   checked on the host before the first launch;
    then everything runs in order on `stream` (bit-identical to one
    apack_prune_step per step).  stage_events_h: NULL or 4*num_steps events
    (entries may be NULL), recorded for step i before scoring [4i], after

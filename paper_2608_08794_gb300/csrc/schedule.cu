@@ -68,6 +68,8 @@ apack_status apack_prune_schedule(const apack_seqs *seqs, int32_t num_layers, co
     if (!sp.q || !sp.k_out || !sp.v_out || !sp.keep_idx || !sp.modality_out || !sp.new_cu_seqlens_h)
       return APACK_EINVAL;
     if (hidden && !sp.hidden_out) return APACK_EINVAL;
+    // the step's queries are read by TMA: 16-byte aligned device memory
+    if ((reinterpret_cast<uintptr_t>(sp.q) & 15) || in_host_memory(sp.q)) return APACK_EINVAL;
     if (i == 0) {
       p.cu.assign(seqs->cu_seqlens_h, seqs->cu_seqlens_h + B + 1);
       p.na.assign(seqs->n_audio_h, seqs->n_audio_h + B);
