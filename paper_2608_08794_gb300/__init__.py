@@ -305,7 +305,11 @@ def apack_prune_schedule(seqs, num_layers, k_cache, v_cache, kv_layer_stride, hi
     if capture:
         g = ctypes.c_void_p()
         _check(_lib.apack_prune_schedule_graph(*head, ctypes.byref(g)), "apack_prune_schedule_graph")
-        return new_cus, ScheduleGraph(g)
+        # the graph replays on these device buffers: keep them alive with it
+        buffers = [t for t in (k_cache, v_cache, hidden, scores, ws, seqs.modality) if t is not None]
+        for d in steps:
+            buffers += [v for v in d.values() if hasattr(v, "data_ptr")]
+        return new_cus, ScheduleGraph(g, buffers)
     stage = _event_handles(stage_events, 4 * n, "stage_events")
     _check(_lib.apack_prune_schedule(*head, stage, _stream(stream)), "apack_prune_schedule")
     return new_cus
@@ -313,10 +317,13 @@ def apack_prune_schedule(seqs, num_layers, k_cache, v_cache, kv_layer_stride, hi
 
 class ScheduleGraph:
     """An executable CUDA graph of one schedule (apack_prune_schedule_graph);
-    launch() replays it, the graph is freed with the object."""
+    launch() replays it, the graph is freed with the object.  The graph reads
+    and writes the device buffers it was captured on, so the object holds
+    references to them (inputs, outputs, scores, workspace) until it is closed."""
 
-    def __init__(self, handle):
+    def __init__(self, handle, buffers=()):
         self._h = handle
+        self._buffers = list(buffers)
 
     def launch(self, stream=None):
         _check(_lib.apack_graph_launch(self._h, _stream(stream)), "apack_graph_launch")
@@ -325,6 +332,7 @@ class ScheduleGraph:
         if self._h is not None and self._h.value:
             _check(_lib.apack_graph_destroy(self._h), "apack_graph_destroy")
         self._h = None
+        self._buffers = []
 
     def __del__(self):
         try:
