@@ -11,7 +11,7 @@ namespace apack {
 
 namespace {
 std::atomic<uint64_t> g_launches{0};
-int g_sm_count[64] = {0};
+std::atomic<int> g_sm_count[64];   // per device; 0 = not read yet
 }  // namespace
 
 void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
@@ -31,10 +31,13 @@ bool in_host_memory(const void *p) {
 int device_sm_count() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
-  if (dev < 64 && g_sm_count[dev] > 0) return g_sm_count[dev];
+  if (dev < 64) {
+    const int cached = g_sm_count[dev].load(std::memory_order_relaxed);
+    if (cached > 0) return cached;
+  }
   int n = 0;
   if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
-  if (dev < 64) g_sm_count[dev] = n;
+  if (dev < 64) g_sm_count[dev].store(n, std::memory_order_relaxed);
   return n;
 }
 

@@ -228,13 +228,11 @@ apack_status plan_inplace(TmaPlan &ip, uint64_t in_items, uint32_t *blocks_out) 
 
 apack_status launch_inplace(const TmaPlan &ip_in, uint32_t blocks, const int32_t *keep_idx, DeviceError *err,
                             cudaStream_t stream) {
-  static bool in_attr_done = false;
-  if (!in_attr_done) {
-    if (check_cuda(cudaFuncSetAttribute(gather_inplace_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        kInSmem)) != APACK_OK)
-      return APACK_ECUDA;
-    in_attr_done = true;
-  }
+  static std::atomic<uint64_t> in_attr_done{0};
+  if (once_per_device(in_attr_done, [] {
+        return cudaFuncSetAttribute(gather_inplace_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kInSmem);
+      }) != cudaSuccess)
+    return APACK_ECUDA;
   TmaPlan ip = ip_in;
   uint16_t *progress = reinterpret_cast<uint16_t *>(reinterpret_cast<uint8_t *>(err) + kProgressOff);
   if (check_cuda(cudaMemsetAsync(progress, 0, blocks * sizeof(uint16_t), stream)) != APACK_OK) return APACK_ECUDA;

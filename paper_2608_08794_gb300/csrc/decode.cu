@@ -398,13 +398,12 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
   float *opart = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + 256);
   float2 *mlpart = reinterpret_cast<float2 *>(static_cast<uint8_t *>(ws) + 256 +
                                               up256(static_cast<size_t>(chunks_all) * num_q_heads * 128 * sizeof(float)));
-  static bool attr_done = false;
-  if (!attr_done) {
-    if (check_cuda(cudaFuncSetAttribute(decode_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        static_cast<int>(kDecSmem))) != APACK_OK)
-      return APACK_ECUDA;
-    attr_done = true;
-  }
+  static std::atomic<uint64_t> attr_done{0};
+  if (once_per_device(attr_done, [] {
+        return cudaFuncSetAttribute(decode_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    static_cast<int>(kDecSmem));
+      }) != cudaSuccess)
+    return APACK_ECUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const uint16_t *q16 = static_cast<const uint16_t *>(q);
   const bool tc = decode_tc_applies(num_q_heads, num_kv_heads) && total > 0;

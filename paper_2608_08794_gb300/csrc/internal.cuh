@@ -3,6 +3,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstddef>
 #include <cstdint>
 
@@ -86,6 +87,20 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   cfg.attrs = at;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+// Kernel attributes (cudaFuncSetAttribute) belong to the current device: `set` runs once
+// per device, recorded in one bit of `done`.  Concurrent first calls on one device may
+// both run it, which is harmless (the same attribute is set twice).
+template <class F>
+cudaError_t once_per_device(std::atomic<uint64_t> &done, F &&set) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = (dev >= 0 && dev < 64) ? (uint64_t{1} << dev) : 0;
+  if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = set();
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_acq_rel);
+  return e;
 }
 bool in_host_memory(const void *p);   // pinned or registered host memory (cudaMemoryTypeHost)
 

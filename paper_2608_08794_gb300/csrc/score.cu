@@ -716,15 +716,16 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_
                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  if (!fn) {
+  // looked up once, by a thread-safe static initialiser (the entry point is the same on every device)
+  static const EncodeTiledFn fn = [] {
     void *p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
             cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(p);
-  }
+      return reinterpret_cast<EncodeTiledFn>(p);
+    return static_cast<EncodeTiledFn>(nullptr);
+  }();
   return fn;
 }
 
@@ -742,7 +743,7 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t mid, uint64_t rows, u
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-bool g_attr_done = false;
+std::atomic<uint64_t> g_attr_done{0};
 
 }  // namespace
 
@@ -775,18 +776,21 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
   uint8_t *qp = wsb + L.qp_off;
   float *gsum = reinterpret_cast<float *>(wsb + L.gsum_off);
 
-  if (!g_attr_done) {
-    if (check_cuda(cudaFuncSetAttribute(score_rowstats_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        kSmemBytes)) != APACK_OK ||
-        check_cuda(cudaFuncSetAttribute(score_rowstats_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        kSmemBytes)) != APACK_OK ||
-        check_cuda(cudaFuncSetAttribute(score_colsum_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        kSmemBytes)) != APACK_OK ||
-        check_cuda(cudaFuncSetAttribute(score_colsum_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        kSmemBytes)) != APACK_OK)
-      return APACK_ECUDA;
-    g_attr_done = true;
-  }
+  if (once_per_device(g_attr_done, [] {
+        cudaError_t e = cudaFuncSetAttribute(score_rowstats_kernel<false>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e == cudaSuccess)
+          e = cudaFuncSetAttribute(score_rowstats_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   kSmemBytes);
+        if (e == cudaSuccess)
+          e = cudaFuncSetAttribute(score_colsum_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   kSmemBytes);
+        if (e == cudaSuccess)
+          e = cudaFuncSetAttribute(score_colsum_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   kSmemBytes);
+        return e;
+      }) != cudaSuccess)
+    return APACK_ECUDA;
   CUtensorMap qmap1, kmap1, qmap2, kmap2;
   const uint64_t qp_rows = static_cast<uint64_t>(L.qp_rows > 0 ? L.qp_rows : 256);
   // pass 1: A = 256-row pairs of packed Q, B = 128-key blocks; pass 2: A = 256 keys, B = 128-row chunks

@@ -234,13 +234,12 @@ __global__ void __launch_bounds__(kThreads)
 template <int RG>
 cudaError_t launch_logits(int grid, size_t smem, cudaStream_t stream, const NarrowPlan &P, const uint16_t *q,
                           const uint8_t *k, int64_t k_stride, const uint8_t *modality, float *logits, float2 *part) {
-  static bool attr = false;
-  if (!attr) {
-    const cudaError_t e = cudaFuncSetAttribute(score_narrow_logits_kernel<RG>,
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  static std::atomic<uint64_t> attr{0};
+  const cudaError_t e = once_per_device(attr, [] {
+    return cudaFuncSetAttribute(score_narrow_logits_kernel<RG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                160 * 1024);
+  });
+  if (e != cudaSuccess) return e;
   return launch_pdl(score_narrow_logits_kernel<RG>, dim3(grid), dim3(kThreads), smem, stream, P, q, k, k_stride,
                     modality, logits, part);
 }

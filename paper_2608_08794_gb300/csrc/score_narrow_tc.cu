@@ -304,25 +304,21 @@ cudaError_t launch_narrow_tc(int grid, cudaStream_t stream, const CUtensorMap &k
                              const uint16_t *q, const uint8_t *modality, float *logits, float2 *part,
                              DeviceError *err) {
   if (P.hkv == 4) {
-    static bool attr = false;
-    if (!attr) {
-      const cudaError_t e = cudaFuncSetAttribute(score_narrow_tc_kernel<4>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 static_cast<int>(TcLayout<4>::kBytes));
-      if (e != cudaSuccess) return e;
-      attr = true;
-    }
+    static std::atomic<uint64_t> attr{0};
+    const cudaError_t e = once_per_device(attr, [] {
+      return cudaFuncSetAttribute(score_narrow_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(TcLayout<4>::kBytes));
+    });
+    if (e != cudaSuccess) return e;
     return launch_pdl(score_narrow_tc_kernel<4>, dim3(grid), dim3(tc_threads<4>()), TcLayout<4>::kBytes, stream,
                       kmap, P, q, modality, logits, part, err);
   } else {
-    static bool attr = false;
-    if (!attr) {
-      const cudaError_t e = cudaFuncSetAttribute(score_narrow_tc_kernel<2>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 static_cast<int>(TcLayout<2>::kBytes));
-      if (e != cudaSuccess) return e;
-      attr = true;
-    }
+    static std::atomic<uint64_t> attr{0};
+    const cudaError_t e = once_per_device(attr, [] {
+      return cudaFuncSetAttribute(score_narrow_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(TcLayout<2>::kBytes));
+    });
+    if (e != cudaSuccess) return e;
     return launch_pdl(score_narrow_tc_kernel<2>, dim3(grid), dim3(tc_threads<2>()), TcLayout<2>::kBytes, stream,
                       kmap, P, q, modality, logits, part, err);
   }

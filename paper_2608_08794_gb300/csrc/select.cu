@@ -366,8 +366,14 @@ cudaError_t launch_select(const SelectPlan &P, int ns, size_t smem, const float 
 constexpr int kWideFrom = 24576;
 
 int select_cluster_size(int max_len, int ns) {
-  static int ready = -1, large_ok = 0;
-  if (ready < 0) {
+  // per device (kernel attributes and residency are properties of the device):
+  // 0 = not probed yet, 1 = attributes refused, 2 = 8-CTA clusters, 3 = 16-CTA clusters too
+  static std::atomic<int> probed[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  int state = probed[dev].load(std::memory_order_acquire);
+  if (state == 0) {
+    int ready = 0, large_ok = 0;
     ready = cudaFuncSetAttribute(select_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(kCacheBytes)) == cudaSuccess;
     large_ok = ready &&
@@ -391,9 +397,11 @@ int select_cluster_size(int max_len, int ns) {
       large_ok = cudaOccupancyMaxActiveClusters(&nclusters, select_kernel<16>, &cfg) == cudaSuccess && nclusters > 0;
     }
     cudaGetLastError();
+    state = !ready ? 1 : (large_ok ? 3 : 2);
+    probed[dev].store(state, std::memory_order_release);
   }
-  if (!ready) return 0;
-  return (max_len > kWideFrom && large_ok && ns * 16 <= device_sm_count()) ? 16 : 8;
+  if (state == 1) return 0;
+  return (max_len > kWideFrom && state == 3 && ns * 16 <= device_sm_count()) ? 16 : 8;
 }
 
 apack_status run_select(const apack_seqs *seqs, const float *scores, const int32_t *keep_count_h, int32_t mode,
