@@ -203,7 +203,9 @@ apack_status apack_prune_step(const apack_seqs *seqs, int32_t layer, int32_t num
    an engine that owns every device allocation, and serving processes that fix
    their device memory at start-up.  The paper has no counterpart; it is a
    deployment variant of apack_score.
-   Same arguments and results as apack_score, without the workspace: the
+   Same arguments, checks and results as apack_score (q and k must be device
+   memory: host memory is refused with APACK_EINVAL before any device work),
+   without the workspace: the
    scratch is one 8 MiB array that the library keeps on every device it is
    loaded on, until the process exits.  Batches whose apack_workspace_size
    exceeds 8 MiB return APACK_EWORKSPACE (a single 7B-shaped sequence with

@@ -162,3 +162,21 @@ def test_step_and_schedule_check_their_compaction_before_any_launch(ap):
                             kv_out_layer_stride=T * row, extra_planes=[good], modality_out=small, keep_idx=small,
                             scores=small, ws=ws, stream=0)
     assert e.value.status == ap.APACK_ECUDA
+
+
+def test_schedule_graph_holds_its_buffers_until_closed(ap):
+    # a captured graph replays on the buffers it was captured on: the Python
+    # object keeps them referenced, and drops them when it is closed
+    import weakref
+
+    class Buf:
+        def data_ptr(self):
+            return 0
+
+    b = Buf()
+    ref = weakref.ref(b)
+    g = ap.ScheduleGraph(ctypes.c_void_p(None), [b])   # a null handle: close() calls nothing
+    del b
+    assert ref() is not None
+    g.close()
+    assert ref() is None
