@@ -64,13 +64,11 @@ __global__ void __launch_bounds__(32) gather_tma_kernel(const __grid_constant__ 
 
 apack_status launch_out_of_place(const TmaPlan &tp, const int32_t *keep_idx, DeviceError *err,
                                  cudaStream_t stream) {
-  static bool attr_done = false;
-  if (!attr_done) {
-    if (check_cuda(cudaFuncSetAttribute(gather_tma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        kTmaSmem)) != APACK_OK)
-      return APACK_ECUDA;
-    attr_done = true;
-  }
+  static std::atomic<uint64_t> attr_done{0};
+  if (once_per_device(attr_done, [] {
+        return cudaFuncSetAttribute(gather_tma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTmaSmem);
+      }) != cudaSuccess)
+    return APACK_ECUDA;
   uint64_t blocks = static_cast<uint64_t>(device_sm_count()) * 2;   // two CTAs of kSlots slots per SM
   if (blocks > tp.total_items) blocks = tp.total_items;
   gather_tma_kernel<<<static_cast<unsigned>(blocks), 32, kTmaSmem, stream>>>(tp, keep_idx, err);

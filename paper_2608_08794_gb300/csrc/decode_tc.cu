@@ -433,22 +433,20 @@ __global__ void __launch_bounds__(kDThreads, 1)
 cudaError_t launch_decode_tc(int grid, cudaStream_t stream, const CUtensorMap &kmap, const CUtensorMap &vmap,
                              const DecPlan &P, const uint16_t *q, float *opart, float2 *mlpart, DeviceError *err) {
   if (P.hkv == 4) {
-    static bool attr = false;
-    if (!attr) {
-      const cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 static_cast<int>(DLay<4>::kBytes));
-      if (e != cudaSuccess) return e;
-      attr = true;
-    }
+    static std::atomic<uint64_t> attr{0};
+    const cudaError_t e = once_per_device(attr, [] {
+      return cudaFuncSetAttribute(decode_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(DLay<4>::kBytes));
+    });
+    if (e != cudaSuccess) return e;
     decode_tc_kernel<4><<<grid, kDThreads, DLay<4>::kBytes, stream>>>(kmap, vmap, P, q, opart, mlpart, err);
   } else {
-    static bool attr = false;
-    if (!attr) {
-      const cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 static_cast<int>(DLay<2>::kBytes));
-      if (e != cudaSuccess) return e;
-      attr = true;
-    }
+    static std::atomic<uint64_t> attr{0};
+    const cudaError_t e = once_per_device(attr, [] {
+      return cudaFuncSetAttribute(decode_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(DLay<2>::kBytes));
+    });
+    if (e != cudaSuccess) return e;
     decode_tc_kernel<2><<<grid, kDThreads, DLay<2>::kBytes, stream>>>(kmap, vmap, P, q, opart, mlpart, err);
   }
   return cudaGetLastError();

@@ -27,10 +27,13 @@ def ap():
     return ap
 
 
-def _inputs(ap, name):
+def _inputs(ap, name, duration_s=None):
     from synth import workload
+    from synth.configs import scaled_copy
     from synth.inputs import query_rows, key_slab
     wl = workload(name)
+    if duration_s is not None:
+        wl = scaled_copy(wl, duration_s)
     layer = wl.prune_layers[0]
     q = query_rows(wl, layer)
     k = key_slab(wl, layer, q)
@@ -66,10 +69,15 @@ def _static(ap, seqs, q, k, stride, T):
 def test_static_scratch_matches_workspace_scores_on_consecutive_calls(ap):
     a = _inputs(ap, "7b_2min")
     b = _inputs(ap, "tiny")
+    # the paper's own setting (last query token only) on a 200-s sequence: the few-row
+    # scoring path, which lays the scratch array out differently (logits, per-CTA partials)
+    p = _inputs(ap, "7b_10min_paper", duration_s=200)
     ref_a = _with_workspace(ap, *a[:5])
     ref_b = _with_workspace(ap, *b[:5])
-    # two calls in a row on the same batch, then another batch, then the first again
-    for args, ref in ((a, ref_a), (a, ref_a), (b, ref_b), (a, ref_a)):
+    ref_p = _with_workspace(ap, *p[:5])
+    # two calls in a row on the same batch, then other batches, the two scoring paths
+    # interleaved, each reading an array the other layout wrote last
+    for args, ref in ((a, ref_a), (a, ref_a), (p, ref_p), (b, ref_b), (p, ref_p), (p, ref_p), (a, ref_a)):
         got = _static(ap, *args[:5])
         check_scores(got, ref)
         assert np.array_equal(got, ref)   # same kernels, same order: bit for bit
