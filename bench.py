@@ -10,15 +10,18 @@ per second (sum over steps of |S| / time).  The headline times the schedule
 captured once into a CUDA graph (apack_prune_schedule_graph) and replayed per
 step; the same JSON line carries the eager run (one apack_prune_schedule call
 per step, with per-stage events), the end-to-end run with host buffers, and
-the side measurements (pre-LLM alignment, decode attention).
+the side measurements (the paper's own 14-step last-query setting, pre-LLM
+alignment, decode attention).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
-Multi-GPU (torchrun): every rank runs its own copy of the workload (the step
-shards by independent sequences; there is no data-path collective), the
-barrier and max-over-ranks timing use torch.distributed, value = units of
-all ranks / time (weak scaling).  ``--impl reference`` times the CPU oracle
-on a bounded sample of the same workload (rank 0 only).
+Multi-GPU (torchrun): the step works on each sequence alone, so a batch of
+several sequences splits over the ranks by whole sequences (strong scaling;
+paper_2608_08794_gb300.shard), and a single sequence runs as one independent
+replica per rank (weak scaling).  There is no data-path collective; the
+barrier and max-over-ranks timing use torch.distributed, value = units of all
+ranks / time.  ``--impl reference`` times the CPU oracle on a bounded sample
+of the same workload (rank 0 only).
 """
 
 import argparse
@@ -50,6 +53,8 @@ def parse():
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=None)
+    p.add_argument("--replicas", action="store_true",
+                   help="with several GPUs, run the whole batch on every rank instead of splitting its sequences")
     p.add_argument("--no-paper-setting", action="store_true",
                    help="skip the side measurement of the paper's own 14-step setting")
     p.add_argument("--part", default="all", choices=["all", "decode", "compact"],
@@ -75,6 +80,16 @@ def max_over_ranks(x, dist, device):
 def whole_job_value(units_per_rank, world, ms_per_iter):
     """Units of all ranks per second, each rank running its own replica."""
     return world * units_per_rank / (ms_per_iter / 1e3)
+
+
+def sum_over_ranks(x, dist, device):
+    """The sum of x over all ranks (x itself without a process group)."""
+    if dist is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
 
 
 def measured_peaks():
@@ -274,12 +289,13 @@ def one():
         keep = out["keep_idx"]
         kk = out["planes"][0].transpose(1, 0, 2, 3); vv = out["planes"][1].transpose(1, 0, 2, 3); hh = out["planes"][2]
         comp, c, m = comp[keep], out["cu_seqlens"], out["modality"]
-    return mm
+    return mm, comp
 reps = {reps}
 times, mm = [], 0
 for r in range(reps):
-    t0 = time.perf_counter(); mm = one(); times.append(time.perf_counter() - t0)
-print(json.dumps(dict(times=times, mm=mm, tokens=wl.total_tokens, dur={dur})))
+    t0 = time.perf_counter(); mm, comp = one(); times.append(time.perf_counter() - t0)
+print(json.dumps(dict(times=times, mm=mm, tokens=wl.total_tokens, dur={dur}, kept=int(comp.size),
+                      kept_sum=int(comp.sum()))))
 """
 
 
@@ -374,16 +390,17 @@ if __name__ == "__main__":
                     j0 = layer - l0
                     copies = [(kind, j, comp) for kind in ("kk", "vv") for j in range(j0, L - l0)]
                     pool.map(_copy, copies + [("hid", 0, comp)])
-                return mm
+                return mm, comp
             one()                                         # warm-up: caches, page faults of the shared planes
             t0 = time.perf_counter()
-            mm = one()
+            mm, comp = one()
             t = time.perf_counter() - t0
     finally:
         for shm in shms:
             shm.close()
             shm.unlink()
-    print(json.dumps(dict(times=[t], mm=mm, tokens=T, dur={dur}, workers=workers)))
+    print(json.dumps(dict(times=[t], mm=mm, tokens=T, dur={dur}, workers=workers, kept=int(comp.size),
+                          kept_sum=int(comp.sum()))))
 """
 
 
@@ -978,6 +995,13 @@ def main():
         torch.cuda.synchronize()
 
     wl = workload(args.workload)
+    # a batch of several sequences splits over the ranks by whole sequences (no data-path exchange:
+    # each rank prunes and keeps its own sequences); a single sequence runs as one replica per rank
+    sharded = world > 1 and wl.num_seqs >= world and not args.replicas
+    if sharded:
+        from paper_2608_08794_gb300.shard import plan_by_sequence
+        from synth.configs import sequence_subset
+        wl = sequence_subset(wl, plan_by_sequence(wl.cu_seqlens(), world)[rank])
     cu0, cuq = wl.cu_seqlens(), wl.cu_qlens()
     na = np.array([s.n_audio for s in wl.seqs], np.int32)
     nv = np.array([s.n_visual for s in wl.seqs], np.int32)
@@ -988,6 +1012,8 @@ def main():
                           wl.prune_layers, counts, select_mode=mode)
     fill_progressive_inputs(pp, wl)
     mm_per_iter = sum(pp.mm_tokens_per_step())
+    # units of the whole job per iteration: every rank's own sequences (split), or world replicas
+    job_units = sum_over_ranks(mm_per_iter, dist, "cuda") if sharded else world * mm_per_iter
     nsteps = len(wl.prune_layers)
     stream = torch.cuda.current_stream()
 
@@ -1192,7 +1218,7 @@ def main():
     if rank == 0:
         eager_ms = ms / args.steps
         per_step_ms = graph_ms                     # the headline: the captured schedule, replayed
-        value = whole_job_value(mm_per_iter, world, per_step_ms)
+        value = job_units / (per_step_ms / 1e3)
         peak, peak_kind = measured_peaks()
         comp_ms = stage_ms[:, 2]
         achieved = sum(comp_bytes) / (comp_ms.sum() / 1e3) / 1e9
@@ -1204,7 +1230,7 @@ def main():
         clock_summary = clocks.summary() if clocks else {}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": per_step_ms, "higher_is_better": True, "scaling": "weak",
+            "warmup": args.warmup, "ms_per_step": per_step_ms, "higher_is_better": True, "scaling": "strong" if sharded else "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": args.workload, "tokens": wl.total_tokens, "mm_tokens": wl.total_mm,
                        "query_rows": int(cuq[-1]), "heads": f"{wl.num_q_heads}q/{wl.num_kv_heads}kv",
@@ -1212,7 +1238,9 @@ def main():
                        "tokens_after_steps": pp.t_out, "mm_tokens_per_iter": mm_per_iter,
                        "l2": "inputs larger than L2 (K/V of the compacted layers: %.1f GB)" %
                              (2 * pp.k_in.numel() * 2 / 1e9),
-                       "parallelism": f"{world} independent replicas" if world > 1 else "1 GPU"},
+                       "parallelism": (f"{world} ranks, the batch's sequences split by tokens (rank 0's share "
+                                       "shown above)" if sharded else
+                                       f"{world} independent replicas" if world > 1 else "1 GPU")},
             "gpu_launches": int(g_launches),
             "roofline": {"bound": "hbm", "kernel": "gather_tma_kernel (compaction)", "achieved": achieved,
                          "peak": peak, "unit": "GB/s", "frac": achieved / peak,
@@ -1224,13 +1252,12 @@ def main():
                                    "compact": float(comp_ms.sum())},
             "launch": "the schedule captured once by apack_prune_schedule_graph and replayed every iteration "
                       "(apack_graph_launch)",
-            "eager": {"value": whole_job_value(mm_per_iter, world, eager_ms), "unit": UNIT,
+            "eager": {"value": job_units / (eager_ms / 1e3), "unit": UNIT,
                       "ms_per_step": eager_ms, "gpu_launches": int(launches),
                       "how": "one apack_prune_schedule call per iteration with stage events; stages_ms_per_iter "
                              "and the compaction roofline come from this run"},
-            "schedule_final_levels": dict(final_levels, value=whole_job_value(mm_per_iter, world,
-                                                                              final_levels["ms_per_step"])),
-            "e2e": {"value": whole_job_value(mm_per_iter, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+            "schedule_final_levels": dict(final_levels, value=job_units / (final_levels["ms_per_step"] / 1e3)),
+            "e2e": {"value": job_units / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": e2e_steps,
                     "pipeline": "caches and hidden states in pinned host memory; per iteration the scored layer's "
                                 "keys, the queries and the modality are copied; every step scores and selects on the "

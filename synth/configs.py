@@ -214,3 +214,15 @@ def scaled_copy(wl: Workload, duration_s: int, n_q: int = None, name: str = None
                     num_q_heads=wl.num_q_heads, num_kv_heads=wl.num_kv_heads, head_dim=wl.head_dim,
                     hidden=wl.hidden, seqs=[s], prune_layers=list(wl.prune_layers),
                     ratios=[[r[0]] for r in wl.ratios], plants=[plants], joint_step_keep=wl.joint_step_keep)
+
+
+def sequence_subset(wl: Workload, seq_ids, name: str = None) -> Workload:
+    """The workload restricted to the sequences ``seq_ids`` (ascending), with their own
+    layouts, plants and keep ratios: one rank's share of a batch split by sequence."""
+    ids = [int(i) for i in seq_ids]
+    return Workload(name=name or f"{wl.name}[{','.join(map(str, ids))}]", seed=wl.seed, num_layers=wl.num_layers,
+                    num_q_heads=wl.num_q_heads, num_kv_heads=wl.num_kv_heads, head_dim=wl.head_dim,
+                    hidden=wl.hidden, seqs=[wl.seqs[i] for i in ids], prune_layers=list(wl.prune_layers),
+                    ratios=[[r[i] for i in ids] for r in wl.ratios],
+                    plants=[wl.plants[i] for i in ids] if wl.plants else [],
+                    joint_step_keep=wl.joint_step_keep)

@@ -186,3 +186,14 @@ def test_shard_maps_tokens_and_rejects_bad_ids():
         SequenceShard([2, 1], cu, cuq, [1, 0, 2, 2], [1, 0, 1, 2])
     with pytest.raises(ValueError):
         merge_keep([[1, 2], [2, 5]])
+
+
+def test_multicore_oracle_baseline_keeps_what_the_single_threaded_oracle_keeps():
+    """bench.py's multi-core CPU baseline splits the oracle's scoring over KV head groups and
+    query-row chunks and recombines the parts (the mean over heads and rows is linear): on a
+    20-s prefix of the 10-minute schedule it keeps exactly the tokens the plain oracle keeps."""
+    sys.path.insert(0, ROOT)
+    import bench
+    one = bench.run_oracle("7b_10min", 20, 1)
+    many = bench.run_oracle_pool("7b_10min", 20, 3)
+    assert (one["kept"], one["kept_sum"], one["mm"]) == (many["kept"], many["kept_sum"], many["mm"])
