@@ -91,7 +91,7 @@ WsLayout workspace_layout(const apack_seqs *s) {
   const size_t part_bytes = static_cast<size_t>(kMaxSplits) * NQ * s->num_q_heads * sizeof(float2);
   L.lse_off = up(L.part_off + part_bytes);
   L.lse_chunks = chunks;
-  L.qp_off = up(L.lse_off + static_cast<size_t>(chunks) * 128 * sizeof(float));
+  L.qp_off = up(L.lse_off + static_cast<size_t>(qp_rows) * sizeof(float));
   L.qp_rows = qp_rows;
   L.gsum_off = up(L.qp_off + static_cast<size_t>(qp_rows) * 256);
   L.total = up(L.gsum_off + static_cast<size_t>(s->num_kv_heads) * T * sizeof(float));

@@ -41,7 +41,7 @@ __device__ __forceinline__ void raise_device_error(DeviceError *e, int32_t code,
 struct WsLayout {
   size_t err_off;     // DeviceError
   size_t part_off;    // float2 [kMaxSplits][sum n_q][Hq]: per-split (max, sum) in log2 units
-  size_t lse_off;     // float [chunks][128]: negated log2 normalisers per 128-row query chunk, -inf padding
+  size_t lse_off;     // float [qp_rows]: negated log2 normaliser of every packed query row, -inf padding
   size_t qp_off;      // bf16 [qp_rows][128]: query rows repacked per KV head group, 256-row padded
   size_t gsum_off;    // float [Hkv][T]: per head group key sums of the column pass
   // few query rows per head group (narrow path, used instead of the four above):

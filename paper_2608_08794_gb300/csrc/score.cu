@@ -5,29 +5,39 @@
 // The softmax normaliser of every (query row, head) needs all keys of S before
 // any per-key average can be formed, so the scores take two passes over K:
 //
-//  pass 1 (row statistics): D[row][key] = Q . K_block^T with query rows in TMEM
-//     lanes; each epilogue thread owns one row and keeps an online (reference,
-//     sum of exp2) over its keys.  Keys are split across CTAs; each (split, row)
-//     writes a partial pair.
-//  merge: per row, the partials combine into a log2-domain normaliser
-//     lse2 = log2 sum_j 2^(x_j log2(e)/sqrt(D)), stored negated per 128-row chunk.
-//  pass 2 (column sums): D[key][row] = K . Q_chunk^T with keys in TMEM lanes;
-//     each thread owns one key and sums 2^(x c - lse2[row]) over the rows of one
-//     KV head group; a final pass adds the Hkv group sums in a fixed order and
+//  pass 1 (row statistics): D[row][key] = Q . K^T with query rows in TMEM lanes;
+//     each epilogue thread owns one row and keeps an online (reference, sum of
+//     exp2) over its keys.  The (row group, key block) space is cut into equal
+//     contiguous ranges, one per CTA pair; a pair writes one partial (m, sum) per
+//     row for each row group its range touches.
+//  merge: per packed query row, the partials combine into a log2-domain
+//     normaliser lse2 = log2 sum_j 2^(x_j log2(e)/sqrt(D)), stored negated.
+//  pass 2 (column sums): D[key][row] = K . Q^T with keys in TMEM lanes; each
+//     thread owns one key and sums 2^(x c - lse2[row]) over the rows of one KV
+//     head group; a final pass adds the Hkv group sums in a fixed order and
 //     scales by 1/(Hq n_q).  No atomics anywhere: scores are deterministic.
 //
 // Query rows are first repacked per KV head g into linear rows rho = token * G + j
 // (query head g*G + j), padded to a multiple of 256, so that tiles hold no holes.
 //
-// Both passes: A operand = two 128-row tiles (256 rows of Q in pass 1, 256 keys
-// in pass 2), B operand = a 128-row tile streamed through a 3-stage TMA ring;
-// each B tile feeds two M=128 x N=128 MMAs, one per A tile, into one of two
-// 256-column TMEM accumulators.  Warp 0 issues TMA, warp 1 owns TMEM and
-// issues tcgen05.mma, warps 2..17 are four epilogue warpgroups, warpgroup
-// (t, h) reading columns h*64.. of A tile t's accumulator; the two halves of
-// a row (pass 1) or key (pass 2) are combined once per work unit through
-// shared memory.  Operands sit in 128-byte swizzled shared memory.
-// Persistent CTAs, one per SM (the shared-memory footprint allows one).
+// Both passes run on CTA pairs (clusters of two CTAs on two SMs) with
+// tcgen05.mma.cta_group::2: one M=256 x N=256 x K=16 instruction per step, issued
+// by the even CTA, reads 128 rows of A and 128 rows of B from each CTA's shared
+// memory and leaves each CTA's 128 rows of D (256 fp32 columns) in its own TMEM.
+// Per SM that moves 64 B of operands from shared memory per clock at the full MMA
+// rate, against 128 B for an M=128 x N=128 instruction on one SM, which is what
+// bounded the single-CTA version.  Each CTA loads its halves of the operands with
+// TMA; the copies of both CTAs complete on the even CTA's barriers
+// (cp.async.bulk.tensor ... .cta_group::2), the MMA completions arrive on both CTAs'
+// barriers (tcgen05.commit ... .multicast::cluster).  The stationary operand A
+// (query rows in pass 1, keys in pass 2) is held for a run of streamed B tiles (key
+// blocks in pass 1, query chunks in pass 2), four B stages deep; two 256-column
+// accumulators alternate in TMEM.  Warp 0 issues TMA, warp 1 owns TMEM (and on the
+// even CTA issues the MMAs), warps 2..17 are four epilogue warpgroups; warpgroup w
+// reads columns 64w.. of the accumulator for the CTA's 128 lanes, 64 values per
+// thread and stage in one TMEM load.  In pass 1, warp 18 builds each key block's
+// masks once per CTA for all epilogue warps.  Operands sit in 128-byte swizzled
+// shared memory.  Persistent pairs, one CTA per SM.
 #include <cmath>
 #include <cstdio>
 
@@ -38,34 +48,39 @@ namespace apack {
 
 namespace {
 
-constexpr int kThreads = 576;          // warp 0: TMA, warp 1: MMA, warps 2..17: epilogue
-constexpr int kEpiWarps = 16;          // four warpgroups: (A tile t, column half h) each
-constexpr uint32_t kTmemCols = 512;    // 2 accumulators x 2 tiles x 128 fp32 columns
-constexpr int kAStages = 2, kBStages = 3;
-constexpr uint32_t kARows = 256, kBRows = 128;
-constexpr uint32_t kABytes = kARows * 256;     // 256 rows x 128 bf16
-constexpr uint32_t kBBytes = kBRows * 256;     // 128 rows x 128 bf16
-constexpr uint32_t kAHalf = kARows * 128;      // second 64-element K half of A
-constexpr uint32_t kBHalf = kBRows * 128;      // ... of B
-constexpr uint32_t kATile = 128 * 128;         // second 128-row tile within an A half
-constexpr uint32_t kIdesc = idesc_bf16_f32(128, 128);
-constexpr int kKeysPerBlock1 = kBRows;         // pass 1: keys per B tile
-constexpr int kKeysPerUnit2 = kARows;          // pass 2: keys per work unit (two tiles)
+constexpr int kEpiWG = 4;                         // epilogue warpgroups, one column range each
+constexpr int kEpiWarps = 4 * kEpiWG;
+constexpr int kCols = 256 / kEpiWG;               // accumulator columns per epilogue thread and stage
+static_assert(kCols == 64, "the epilogues read 64 columns per thread and stage");
+// warp 0: TMA, warp 1: TMEM (+ MMA on the even CTA), then the epilogue warps, then (pass 1) the
+// key-mask warp.  Nineteen warps take the same registers per thread as eighteen.
+constexpr int kMaskWarp = 2 + kEpiWarps;
+constexpr int kThreads = 32 * (kMaskWarp + 1);
+constexpr uint32_t kTmemCols = 512;    // 2 accumulators x 256 fp32 columns
+constexpr int kAStages = 2, kBStages = 4;
+constexpr uint32_t kRows = 128;                // rows of A and of B per CTA (M/2, N/2 of the pair)
+constexpr uint32_t kTileBytes = kRows * 256;   // 128 rows x 128 bf16
+constexpr uint32_t kHalf = kRows * 128;        // second 64-element K half of a tile
+constexpr uint32_t kIdesc = idesc_bf16_f32(256, 256);
+constexpr int kBlock = 256;                    // keys per key block (pass 1) / per key unit (pass 2)
+constexpr int kChunk = 256;                    // query rows per chunk (pass 2) / per row pair (pass 1)
+constexpr int kPairSlots = kMaxSplits;         // pair ranges per row group (one partial each)
 
 struct SeqPlan {
   int32_t t0, len;        // token range of the sequence in the packed batch
   int32_t q_off, n_q;     // query tokens in packed Q
   int32_t qp_base;        // first packed row of head group 0; group g starts at qp_base + g * rows_pad
   int32_t rows_pad;       // G * n_q rounded up to a multiple of 256
-  int32_t unit_begin;     // first work unit of this sequence in the launch
-  int32_t bps;            // pass 1: key blocks per split
-  int32_t n_split;        // pass 1: splits
-  int32_t chunk_base;     // index of this sequence's first normaliser chunk
+  int32_t nb;             // key blocks (256 keys) of the sequence
+  int32_t unit_begin;     // pass 2: first work unit of this sequence in the launch
+  int32_t flat0;          // pass 1: first flat (row group, key block) index of the sequence
 };
 
 struct ScorePlan {
   int32_t nseq;
-  int32_t total_units;
+  int32_t total_units;     // pass 2
+  int32_t pairs;           // pass 1: CTA pairs of the launch
+  int32_t flat_total;      // pass 1: (row group, key block) items of the launch (< 2^31, checked)
   int32_t hq, hkv, group;
   int32_t total_qrows;     // sum n_q over the whole batch
   int32_t total_tokens;    // T
@@ -77,38 +92,120 @@ struct ScorePlan {
 struct __align__(8) Bars {
   uint64_t a_full[kAStages], a_empty[kAStages], b_full[kBStages], b_empty[kBStages];
   uint64_t acc_full[2], acc_empty[2], drain;
-  uint64_t l_empty[kBStages];       // pass 2: normaliser slot released by the epilogue
-  uint64_t comb_full[2], comb_empty[2];   // pass 2, per key tile: column half 1 -> half 0 hand-off
+  uint64_t l_full[kBStages], l_empty[kBStages];   // pass 2: normaliser slot loaded / released (this CTA)
+  uint64_t comb_full[2], comb_empty[2];           // column ranges 1.. -> range 0 hand-off
+  uint64_t m_full[kBStages], m_empty[kBStages];   // pass 1: key masks of a block written / read
   uint32_t tmem_base;
   volatile int32_t abort;
 };
 
-// Shared memory: [A x2][B x3][-lse2 x3 (pass 2)][combine 2 x 128 float (pass 2)][Bars].
+// Shared memory: [A x2][B x4][-lse2 x4 (pass 2)][combine 2 x (kEpiWG - 1) x 128 float2]
+// [key masks 4 x 8 words (pass 1)][Bars].
 // The dynamic shared window is declared 1024-byte aligned (the 128-byte swizzle
 // atoms of the operand tiles need it); the kernels verify it before any use.
 constexpr uint32_t kOffA = 0;
-constexpr uint32_t kOffB = kAStages * kABytes;
-constexpr uint32_t kOffL = kOffB + kBStages * kBBytes;
-constexpr uint32_t kOffC = kOffL + kBStages * kBRows * sizeof(float);
-constexpr uint32_t kOffBars = kOffC + 2 * 128 * sizeof(float);
-constexpr uint32_t kSmemBytes = kOffBars + 256;
+constexpr uint32_t kOffB = kAStages * kTileBytes;
+constexpr uint32_t kOffL = kOffB + kBStages * kTileBytes;
+constexpr uint32_t kOffC = kOffL + kBStages * kChunk * sizeof(float);
+constexpr uint32_t kOffM = kOffC + 2 * (kEpiWG - 1) * kRows * sizeof(float2);
+constexpr uint32_t kOffBars = kOffM + kBStages * (kBlock / 32) * sizeof(uint32_t);
+constexpr uint32_t kSmemBytes = kOffBars + 512;
+static_assert(sizeof(Bars) <= 512, "barrier block");
 static_assert(kSmemBytes <= 232448, "shared memory budget");
-
-__device__ __forceinline__ int find_seq(const ScorePlan &p, int u) {
-  int s = 0;
-  while (s + 1 < p.nseq && p.seq[s + 1].unit_begin <= u) ++s;
-  return s;
-}
 
 __device__ __forceinline__ bool is_mm(uint8_t m) { return m == APACK_MOD_AUDIO || m == APACK_MOD_VISUAL; }
 
-__host__ __device__ __forceinline__ int n_pairs(const SeqPlan &sp) { return sp.rows_pad / 256; }
-__host__ __device__ __forceinline__ int n_chunks(const SeqPlan &sp, int G) { return (G * sp.n_q + 127) / 128; }
-__host__ __device__ __forceinline__ int n_keypairs(const SeqPlan &sp) { return (sp.len + 255) / 256; }
+__host__ __device__ __forceinline__ int n_pairs(const SeqPlan &sp) { return sp.rows_pad / kChunk; }
+__host__ __device__ __forceinline__ int64_t pass1_items(const SeqPlan &sp, int hkv) {
+  return static_cast<int64_t>(sp.nb) * hkv * n_pairs(sp);
+}
 
-// A wait that also gives up when another role has aborted.
-__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, Bars *bars, DeviceError *err,
-                                              int where) {
+// Pass 1: pair p of P owns the flat items [start(p), start(p + 1)), start(p) = p W / P,
+// and the pair holding item x is ((x + 1) P - 1) / W (64-bit products of 32-bit indices).
+__host__ __device__ __forceinline__ int32_t range_start(int64_t p, int64_t P, int64_t W) {
+  return static_cast<int32_t>(p * W / P);
+}
+__host__ __device__ __forceinline__ int32_t pair_of(int64_t x, int64_t P, int64_t W) {
+  return static_cast<int32_t>(((x + 1) * P - 1) / W);
+}
+
+// ---------------------------------------------------------------- cluster-pair helpers
+// Barrier waits and arrivals keep the default (CTA-scope) semantics: what crosses the pair
+// through them is ordered by the asynchronous proxies themselves (TMA byte counts, MMA
+// commits) and by the tcgen05 fences around TMEM reads, not by generic memory accesses.
+// (Cluster-scope acquire and release here made every wait and arrival a memory barrier:
+// measured 1.5x slower, with memory-barrier stalls the largest stall reason.)
+
+// Remote (or local) arrive on a barrier given by its shared::cluster address.
+__device__ __forceinline__ void arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+__device__ __forceinline__ void st_cluster_u32(uint32_t cluster_addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
+}
+
+// 3-D tiled load into this CTA's shared memory, completion counted on a barrier of
+// either CTA of the pair (given as a shared::cluster address).
+__device__ __forceinline__ void tma_load_3d_pair(void *dst, const CUtensorMap *map, uint32_t bar_cluster, int32_t c0,
+                                                 int32_t c1, int32_t c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, "
+      "%5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(kIdesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on the barrier at this offset in both CTAs once the issued MMAs complete.
+__device__ __forceinline__ void commit_pair(uint64_t *bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          smem_u32(bar)),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+
+// Arrive on this CTA's own barrier once the issued MMAs complete.
+__device__ __forceinline__ void commit_pair_self(uint64_t *bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t *dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+struct PairCtx {
+  uint32_t rank;          // 0: the even CTA (issues the MMAs), 1: its peer
+  uint32_t lead_bars;     // shared::cluster address of the even CTA's Bars
+  uint32_t peer_abort;    // shared::cluster address of the other CTA's abort flag
+};
+
+template <typename T>
+__device__ __forceinline__ uint32_t lead_addr(const PairCtx &pc, const Bars *bars, const T *member) {
+  return pc.lead_bars + static_cast<uint32_t>(reinterpret_cast<const uint8_t *>(member) -
+                                              reinterpret_cast<const uint8_t *>(bars));
+}
+
+// A wait that also gives up when a role of either CTA has aborted; a timeout aborts both.
+__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, Bars *bars, const PairCtx &pc,
+                                              DeviceError *err, int where) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (;;) {
@@ -117,6 +214,7 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, Ba
     if (bars->abort) return false;
     if (globaltimer_ns() - t0 > kWaitLimitNs) {
       bars->abort = 1;
+      st_cluster_u32(pc.peer_abort, 1u);
       raise_device_error(err, APACK_ETIMEOUT, where);
       return false;
     }
@@ -126,8 +224,10 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, Ba
 // True when the dynamic shared window has the 1024-byte alignment the operand tiles need.
 __device__ __forceinline__ bool smem_aligned(const uint8_t *smem) { return (smem_u32(smem) & 1023u) == 0; }
 
-__device__ void init_common(uint8_t *smem, Bars *bars, int warp) {
-  // Zero the operand buffers so that MMA rows no TMA box writes stay finite.
+__device__ PairCtx init_pair(uint8_t *smem, Bars *bars, int warp) {
+  PairCtx pc;
+  pc.rank = cluster_ctarank();
+  // Zero the operand buffers once (every tile is then fully written by its TMA boxes).
   for (uint32_t i = threadIdx.x; i < kOffL / 16; i += blockDim.x)
     reinterpret_cast<uint4 *>(smem)[i] = make_uint4(0, 0, 0, 0);
   if (threadIdx.x == 0) {
@@ -138,145 +238,171 @@ __device__ void init_common(uint8_t *smem, Bars *bars, int warp) {
     for (int i = 0; i < kBStages; ++i) {
       mbar_init(&bars->b_full[i], 1);
       mbar_init(&bars->b_empty[i], 1);
+      mbar_init(&bars->l_full[i], 1);
       mbar_init(&bars->l_empty[i], kEpiWarps);
+      mbar_init(&bars->m_full[i], 1);
+      mbar_init(&bars->m_empty[i], kEpiWarps);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->acc_full[i], 1);
-      mbar_init(&bars->acc_empty[i], kEpiWarps);
-      mbar_init(&bars->comb_full[i], 128);
-      mbar_init(&bars->comb_empty[i], 128);
+      mbar_init(&bars->acc_empty[i], 2 * kEpiWarps);   // the epilogue warps of both CTAs
+      mbar_init(&bars->comb_full[i], (kEpiWG - 1) * 4);
+      mbar_init(&bars->comb_empty[i], 4);
     }
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
     fence_mbar_init();
   }
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  pc.lead_bars = map_shared_rank(bars, 0);
+  pc.peer_abort = map_shared_rank(const_cast<const int32_t *>(&bars->abort), pc.rank ^ 1u);
+  cluster_sync();                      // both CTAs' barriers exist before any remote arrive or copy
   if (warp == 1) {
-    tmem_alloc(&bars->tmem_base, kTmemCols);
+    tmem_alloc_pair(&bars->tmem_base, kTmemCols);
     tc_fence_before();
   }
   __syncthreads();
   tc_fence_after();
+  return pc;
 }
 
-// Teardown: after an abort the MMA thread makes sure no MMA is in flight; then TMEM is freed.
-__device__ void finish_common(Bars *bars, int warp, bool mma_thread) {
+// Teardown: after an abort the MMA thread makes sure no MMA is in flight; both CTAs
+// then meet (every TMEM read and every MMA of the pair is done) and free TMEM.
+__device__ void finish_pair(Bars *bars, const PairCtx &pc, int warp, bool mma_thread) {
   if (mma_thread && bars->abort) {
-    tc_commit(&bars->drain);
+    commit_pair_self(&bars->drain);
     mbar_wait(&bars->drain, 0, kWaitLimitNs / 4);
+  }
+  if (threadIdx.x == 0 && bars->abort) {
+    // copies of this CTA complete on the even CTA's barriers, which this CTA cannot watch:
+    // give any still in flight time to land before the pair meets (bounded)
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < 200000ull) {
+    }
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(bars->tmem_base, kTmemCols);
+  if (warp == 1) tmem_dealloc_pair(bars->tmem_base, kTmemCols);
 }
 
-// Waits (bounded, ignoring the abort flag) for TMA loads that were issued
-// but never consumed, so that no copy lands in shared memory after exit.
+// Waits (bounded, ignoring the abort flag) for TMA loads that were issued but never
+// consumed, so that no copy lands in shared memory after exit (the even CTA's barriers).
 __device__ void drain_loads(uint64_t *full, const bool *pending, const uint32_t *parity, int n) {
   for (int i = 0; i < n; ++i)
     if (pending[i]) mbar_wait(&full[i], parity[i], kWaitLimitNs / 4);
 }
 
-// Issues the two MMAs of one B tile (one per A tile) into accumulator `ci`.
-__device__ __forceinline__ void issue_mma_pair(uint32_t tmem, int ci, uint32_t a_base, uint32_t b_base, int ntiles) {
-  for (int t = 0; t < ntiles; ++t) {
+// kCols consecutive TMEM columns of this warp's 32 lanes -> registers, loaded and waited for
+// in one statement (the registers are defined only once the data is there).
+__device__ __forceinline__ void tmem_load_cols(uint32_t taddr, uint32_t (&r)[64]) { tmem_ld64_wait(taddr, r); }
+
+// The eight K=16 steps of one 256 x 256 x 128 product into accumulator `ci`.
+__device__ __forceinline__ void issue_mma(uint32_t tmem, int ci, uint32_t a_base, uint32_t b_base) {
 #pragma unroll
-    for (int kk = 0; kk < 8; ++kk) {
-      const uint32_t ao = (kk >> 2) * kAHalf + t * kATile + (kk & 3) * 32;
-      const uint32_t bo = (kk >> 2) * kBHalf + (kk & 3) * 32;
-      tc_mma_bf16(tmem + ci * 256 + t * 128, smem_desc_sw128(a_base + ao), smem_desc_sw128(b_base + bo), kIdesc,
-                  kk > 0 ? 1u : 0u);
-    }
+  for (int kk = 0; kk < 8; ++kk) {
+    const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
+    mma_pair(tmem + ci * 256, smem_desc_sw128(a_base + off), smem_desc_sw128(b_base + off), kk > 0 ? 1u : 0u);
   }
 }
 
 // ------------------------------------------------------------------ pass 1
-struct Unit1 {
-  int s, g, qp, b0, b1, split, ntiles;
+// A run: the part of a pair's flat range that lies in one row group (sequence s, KV head
+// group g, 256-row pair qp): key blocks [b0, b1) of that row group.
+struct Run {
+  int s, g, qp, b0, b1;
+  int x1;          // flat index after the run
+  int slot;        // partial slot: pair - first pair of the row group
 };
 
-__device__ __forceinline__ Unit1 decode_unit1(const ScorePlan &p, int u) {
-  Unit1 w;
-  w.s = find_seq(p, u);
-  const SeqPlan &sp = p.seq[w.s];
-  const int local = u - sp.unit_begin;
-  const int np = n_pairs(sp);
-  w.qp = local % np;
-  const int pg = local / np;
-  w.g = pg % p.hkv;
-  w.split = pg / p.hkv;
-  const int nb = (sp.len + kKeysPerBlock1 - 1) / kKeysPerBlock1;
-  w.b0 = w.split * sp.bps;
-  w.b1 = min(nb, w.b0 + sp.bps);
-  w.ntiles = p.group * sp.n_q - w.qp * 256 > 128 ? 2 : 1;
-  return w;
+__device__ __forceinline__ int seq_of_flat(const ScorePlan &p, int x) {
+  int s = 0;
+  while (s + 1 < p.nseq && p.seq[s + 1].flat0 <= x) ++s;
+  return s;
 }
 
-// Online (reference, sum) update with 32 logits in log2 units: the reference
-// is only raised when a value exceeds it by 2^64 (sum overflow check), which
-// keeps the max computation off the common path.  Four independent partial
-// sums keep the add chain short.
-template <int OFF>
-__device__ __forceinline__ void online_chunk(const uint32_t (&r)[64], uint32_t mask, float c2, float &m,
+__device__ __forceinline__ Run next_run(const ScorePlan &p, int x, int x_end, int pair) {
+  Run r;
+  r.s = seq_of_flat(p, x);
+  const SeqPlan &sp = p.seq[r.s];
+  const int local = x - sp.flat0;
+  const int grp = local / sp.nb;                      // row group index within the sequence
+  const int np = n_pairs(sp);
+  r.g = grp / np;
+  r.qp = grp - r.g * np;
+  r.b0 = local - grp * sp.nb;
+  const int grp_end = sp.flat0 + (grp + 1) * sp.nb;
+  r.x1 = x_end < grp_end ? x_end : grp_end;
+  r.b1 = r.b0 + (r.x1 - x);
+  r.slot = pair - pair_of(sp.flat0 + grp * sp.nb, p.pairs, p.flat_total);
+  return r;
+}
+
+// Online (reference, sum) update with a thread's 64 logits of a block, in log2 units.  Keys
+// that do not count are first replaced by -inf (exp2 gives 0), so that one code path serves
+// every mask.  The reference is the first counted block's maximum and is only raised when a
+// block's sum exceeds 2^64 (or overflows): the maximum stays off the common path.  Four
+// independent partial sums keep the add chains short.
+__device__ __forceinline__ void online_block(uint32_t (&r)[64], uint32_t mask0, uint32_t mask1, float c2, float &m,
                                              float &sum) {
-  if (mask == 0u) return;
-  if (m == -INFINITY) {
-    float mx = -INFINITY;
+  if ((mask0 & mask1) != 0xffffffffu) {
+    if ((mask0 | mask1) == 0u) return;
+    const uint32_t ninf = __float_as_uint(-INFINITY);
 #pragma unroll
-    for (int i = 0; i < 32; ++i)
-      if ((mask >> i) & 1u) mx = fmaxf(mx, __uint_as_float(r[OFF + i]));
+    for (int i = 0; i < 32; ++i) {
+      r[i] = ((mask0 >> i) & 1u) ? r[i] : ninf;
+      r[32 + i] = ((mask1 >> i) & 1u) ? r[32 + i] : ninf;
+    }
+  }
+  if (m == -INFINITY) {
+    float mx = __uint_as_float(r[0]);
+#pragma unroll
+    for (int i = 1; i < 64; ++i) mx = fmaxf(mx, __uint_as_float(r[i]));
     m = mx * c2;
   }
   float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
   const float2 cc = make_float2(c2, c2), nm = make_float2(-m, -m);
-  if (mask == 0xffffffffu) {
 #pragma unroll
-    for (int i = 0; i < 32; i += 2) {
-      const float2 y = ffma2(make_float2(__uint_as_float(r[OFF + i]), __uint_as_float(r[OFF + i + 1])), cc, nm);
-      a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(y.x), ex2_approx(y.y)));
-    }
-  } else {
-#pragma unroll
-    for (int i = 0; i < 32; i += 2) {
-      const float2 y = ffma2(make_float2(__uint_as_float(r[OFF + i]), __uint_as_float(r[OFF + i + 1])), cc, nm);
-      a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(((mask >> i) & 1u) ? ex2_approx(y.x) : 0.f,
-                                                           ((mask >> (i + 1)) & 1u) ? ex2_approx(y.y) : 0.f));
-    }
+  for (int i = 0; i < 64; i += 2) {
+    const float2 y = ffma2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), cc, nm);
+    a[(i >> 1) & 3] = fadd2(a[(i >> 1) & 3], make_float2(ex2_approx(y.x), ex2_approx(y.y)));
   }
   const float2 s01 = fadd2(a[0], a[1]), s23 = fadd2(a[2], a[3]);
   const float2 s4 = fadd2(s01, s23);
   float t = s4.x + s4.y;
   if (!(t <= 1.8446744e19f)) {   // a value exceeded the reference by more than 2^64 (or inf): rescale
-    float mx = -INFINITY;
+    float mx = __uint_as_float(r[0]);
 #pragma unroll
-    for (int i = 0; i < 32; ++i)
-      if ((mask >> i) & 1u) mx = fmaxf(mx, __uint_as_float(r[OFF + i]));
+    for (int i = 1; i < 64; ++i) mx = fmaxf(mx, __uint_as_float(r[i]));
     mx *= c2;
     sum *= ex2_approx(m - mx);
     m = mx;
     t = 0.f;
 #pragma unroll
-    for (int i = 0; i < 32; ++i)
-      if ((mask >> i) & 1u) t += ex2_approx(fmaf(__uint_as_float(r[OFF + i]), c2, -m));
+    for (int i = 0; i < 64; ++i) t += ex2_approx(fmaf(__uint_as_float(r[i]), c2, -m));
   }
   sum += t;
 }
 
 template <bool CAUSAL>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     score_rowstats_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                           const __grid_constant__ ScorePlan plan, const uint8_t *__restrict__ modality,
                           float2 *__restrict__ part, DeviceError *err) {
   extern __shared__ __align__(1024) uint8_t smem[];
-  if (!smem_aligned(smem)) {
+  if (!smem_aligned(smem)) {   // the same in both CTAs of the pair: both leave here
     if (threadIdx.x == 0) raise_device_error(err, APACK_EDEVICE, 10);
     return;
   }
   Bars *bars = reinterpret_cast<Bars *>(smem + kOffBars);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  init_common(smem, bars, warp);
+  const PairCtx pc = init_pair(smem, bars, warp);
   const int G = plan.group;
+  const int pair = blockIdx.x >> 1;
+  const int x_begin = range_start(pair, plan.pairs, plan.flat_total);
+  const int x_end = range_start(pair + 1, plan.pairs, plan.flat_total);
+  const int row_half = static_cast<int>(pc.rank) * kRows;   // this CTA's rows of the 256-row pair
 
   if (warp == 0) {
     if (lane == 0) {
@@ -287,136 +413,202 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool pend[kBStages] = {}, apend[kAStages] = {};
       uint32_t pend_par[kBStages] = {}, apend_par[kAStages] = {};
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < plan.total_units; u += gridDim.x) {
-        const Unit1 w = decode_unit1(plan, u);
+      for (int x = x_begin; ok && x < x_end;) {
+        const Run w = next_run(plan, x, x_end, pair);
         const SeqPlan &sp = plan.seq[w.s];
-        if (!wait_or_abort(&bars->a_empty[ai], aph ^ 1, bars, err, 11)) { ok = false; break; }
-        uint8_t *A = smem + kOffA + ai * kABytes;
-        mbar_arrive_expect_tx(&bars->a_full[ai], kABytes);
-        const int arow = sp.qp_base + w.g * sp.rows_pad + w.qp * 256;
-        tma_load_3d(A, &qmap, &bars->a_full[ai], 0, 0, arow);
-        tma_load_3d(A + kAHalf, &qmap, &bars->a_full[ai], 64, 0, arow);
+        x = w.x1;
+        if (!wait_or_abort(&bars->a_empty[ai], aph ^ 1, bars, pc, err, 11)) { ok = false; break; }
+        uint8_t *A = smem + kOffA + ai * kTileBytes;
+        if (pc.rank == 0) mbar_arrive_expect_tx(&bars->a_full[ai], 2 * kTileBytes);
+        const uint32_t afull = lead_addr(pc, bars, &bars->a_full[ai]);
+        const int arow = sp.qp_base + w.g * sp.rows_pad + w.qp * kChunk + row_half;
+        tma_load_3d_pair(A, &qmap, afull, 0, 0, arow);
+        tma_load_3d_pair(A + kHalf, &qmap, afull, 64, 0, arow);
         apend[ai] = true;
         apend_par[ai] = aph;
         for (int b = w.b0; b < w.b1; ++b) {
-          if (!wait_or_abort(&bars->b_empty[bi], bph ^ 1, bars, err, 12)) { ok = false; break; }
-          uint8_t *B = smem + kOffB + bi * kBBytes;
-          mbar_arrive_expect_tx(&bars->b_full[bi], kBBytes);
-          const int key0 = sp.t0 + b * kKeysPerBlock1;
-          tma_load_3d(B, &kmap, &bars->b_full[bi], 0, w.g, key0);
-          tma_load_3d(B + kBHalf, &kmap, &bars->b_full[bi], 64, w.g, key0);
+          if (!wait_or_abort(&bars->b_empty[bi], bph ^ 1, bars, pc, err, 12)) { ok = false; break; }
+          uint8_t *B = smem + kOffB + bi * kTileBytes;
+          if (pc.rank == 0) mbar_arrive_expect_tx(&bars->b_full[bi], 2 * kTileBytes);
+          const uint32_t bfull = lead_addr(pc, bars, &bars->b_full[bi]);
+          const int key0 = sp.t0 + b * kBlock + row_half;
+          tma_load_3d_pair(B, &kmap, bfull, 0, w.g, key0);
+          tma_load_3d_pair(B + kHalf, &kmap, bfull, 64, w.g, key0);
           pend[bi] = true;
           pend_par[bi] = bph;
           if (++bi == kBStages) { bi = 0; bph ^= 1; }
         }
         if (++ai == kAStages) { ai = 0; aph ^= 1; }
       }
-      if (!ok) {
+      if (!ok && pc.rank == 0) {
         drain_loads(bars->b_full, pend, pend_par, kBStages);
         drain_loads(bars->a_full, apend, apend_par, kAStages);
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && pc.rank == 0) {
       int ai = 0, bi = 0, ci = 0;
       uint32_t aph = 0, bph = 0, cph = 0;
       const uint32_t tmem = bars->tmem_base;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < plan.total_units; u += gridDim.x) {
-        const Unit1 w = decode_unit1(plan, u);
-        if (!wait_or_abort(&bars->a_full[ai], aph, bars, err, 13)) { ok = false; break; }
-        const uint32_t a_base = smem_u32(smem + kOffA + ai * kABytes);
+      for (int x = x_begin; ok && x < x_end;) {
+        const Run w = next_run(plan, x, x_end, pair);
+        x = w.x1;
+        if (!wait_or_abort(&bars->a_full[ai], aph, bars, pc, err, 13)) { ok = false; break; }
+        const uint32_t a_base = smem_u32(smem + kOffA + ai * kTileBytes);
         for (int b = w.b0; b < w.b1; ++b) {
-          if (!wait_or_abort(&bars->b_full[bi], bph, bars, err, 14)) { ok = false; break; }
-          if (!wait_or_abort(&bars->acc_empty[ci], cph ^ 1, bars, err, 15)) { ok = false; break; }
+          if (!wait_or_abort(&bars->b_full[bi], bph, bars, pc, err, 14)) { ok = false; break; }
+          if (!wait_or_abort(&bars->acc_empty[ci], cph ^ 1, bars, pc, err, 15)) { ok = false; break; }
           tc_fence_after();
-          issue_mma_pair(tmem, ci, a_base, smem_u32(smem + kOffB + bi * kBBytes), w.ntiles);
-          tc_commit(&bars->b_empty[bi]);
-          tc_commit(&bars->acc_full[ci]);
+          issue_mma(tmem, ci, a_base, smem_u32(smem + kOffB + bi * kTileBytes));
+          commit_pair(&bars->b_empty[bi]);
+          commit_pair(&bars->acc_full[ci]);
           if (++bi == kBStages) { bi = 0; bph ^= 1; }
           if (++ci == 2) { ci = 0; cph ^= 1; }
         }
         if (!ok) break;
-        tc_commit(&bars->a_empty[ai]);
+        commit_pair(&bars->a_empty[ai]);
         if (++ai == kAStages) { ai = 0; aph ^= 1; }
       }
     }
-  } else {
-    // Epilogue: warpgroup q = (t, h) reads columns h*64.. of A tile t (query
-    // rows t*128 ..); warp w reads TMEM lanes 32*(w%4)..
-    const int q = (warp - 2) >> 2;
-    const int t = q & 1, h = q >> 1;
-    const int quad = warp & 3;
-    const int row = t * 128 + quad * 32 + lane;         // row of the 256-row query pair
-    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-    const float c2 = plan.scale2;
-    int ci = 0;
-    uint32_t cph = 0;
-    bool ok = true;
-    for (int u = blockIdx.x; ok && u < plan.total_units; u += gridDim.x) {
-      const Unit1 w = decode_unit1(plan, u);
-      const SeqPlan &sp = plan.seq[w.s];
-      const int t_end = sp.t0 + sp.len;
-      const bool active = t < w.ntiles;
-      float m = -INFINITY, sum = 0.f;
-      // modality of this lane's 2 keys of a block, prefetched one block ahead
-      uint8_t mod_next[2];
+  } else if (warp == kMaskWarp) {
+    // Key masks: for every block, bit k of word c says whether key c*32 + k of the block counts
+    // (in the sequence and, outside the causal domain, in S); written once per CTA for all
+    // epilogue warps.  The modality bytes are loaded two blocks ahead of the block being masked.
+    uint32_t *masks = reinterpret_cast<uint32_t *>(smem + kOffM);
+    constexpr int kW = kBlock / 32;
+    // key range of flat item x: first key of its block and end of its sequence
+    auto block_keys = [&](int x, int &key_base, int &t_end) {
+      const SeqPlan &sp = plan.seq[seq_of_flat(plan, x)];
+      key_base = sp.t0 + ((x - sp.flat0) % sp.nb) * kBlock;
+      t_end = sp.t0 + sp.len;
+    };
+    auto load = [&](int x, uint8_t (&mod)[kW]) {
+      if (x >= x_end) return;
+      int kb, te;
+      block_keys(x, kb, te);
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        const int key = sp.t0 + w.b0 * kKeysPerBlock1 + h * 64 + c * 32 + lane;
-        mod_next[c] = (active && key < t_end) ? modality[key] : 0;
+      for (int c = 0; c < kW; ++c) {
+        const int key = kb + c * 32 + lane;
+        mod[c] = key < te ? modality[key] : 0;
       }
+    };
+    uint8_t m0[kW], m1[kW], m2[kW];
+    load(x_begin, m0);
+    load(x_begin + 1, m1);
+    int mi = 0;
+    uint32_t mph = 0;
+    for (int x = x_begin; x < x_end; ++x) {
+      load(x + 2, m2);
+      int kb, te;
+      block_keys(x, kb, te);
+      if (!wait_or_abort(&bars->m_empty[mi], mph ^ 1, bars, pc, err, 19)) break;
+      uint32_t word = 0;
+#pragma unroll
+      for (int c = 0; c < kW; ++c) {
+        const int key = kb + c * 32 + lane;
+        const uint32_t mk = __ballot_sync(0xffffffffu, key < te && (CAUSAL || is_mm(m0[c])));
+        if (lane == c) word = mk;
+      }
+      if (lane < kW) masks[mi * kW + lane] = word;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->m_full[mi]);
+      if (++mi == kBStages) { mi = 0; mph ^= 1; }
+#pragma unroll
+      for (int c = 0; c < kW; ++c) {
+        m0[c] = m1[c];
+        m1[c] = m2[c];
+      }
+    }
+  } else {
+    // Epilogue: warpgroup q reads columns q*kCols.. (keys of the block) for the CTA's 128 rows;
+    // warp w reads TMEM lanes 32*(w%4)..
+    const int q = (warp - 2) >> 2;
+    const int quad = warp & 3;
+    const int row = row_half + quad * 32 + lane;            // row of the 256-row pair
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    const uint32_t acc_empty0 = lead_addr(pc, bars, &bars->acc_empty[0]);
+    const float c2 = plan.scale2;
+    float2 *comb = reinterpret_cast<float2 *>(smem + kOffC);   // [2 parities][kEpiWG - 1 ranges][128 rows]
+    const uint32_t *masks = reinterpret_cast<const uint32_t *>(smem + kOffM);
+    int ci = 0, mi = 0;
+    uint32_t cph = 0, xph = 0, mph = 0;
+    bool ok = true;
+    for (int x = x_begin; ok && x < x_end;) {
+      const Run w = next_run(plan, x, x_end, pair);
+      const SeqPlan &sp = plan.seq[w.s];
+      x = w.x1;
+      float m = -INFINITY, sum = 0.f;
       // causal rows: this lane's row (token r of the query span) sees keys up to len - n_q + r
-      const int see = sp.len - sp.n_q + (w.qp * 256 + row) / G;
+      const int see = sp.len - sp.n_q + (w.qp * kChunk + row) / G;
       for (int b = w.b0; b < w.b1; ++b) {
-        uint32_t mask[2], rmask[2];   // keys of the chunk (warp-uniform); and those this lane's row sees
-        const int key_base = sp.t0 + b * kKeysPerBlock1 + h * 64;
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          const int key = key_base + c * 32 + lane;
-          mask[c] = __ballot_sync(0xffffffffu, key < t_end && (CAUSAL || is_mm(mod_next[c])));
-          rmask[c] = mask[c];
-          if (CAUSAL) {        // keys at local index <= see
-            const int lim = see - (key_base - sp.t0 + c * 32);
-            rmask[c] &= lim >= 31 ? 0xffffffffu : (lim < 0 ? 0u : (2u << lim) - 1u);
-          }
+        // the keys of this thread's two 32-key chunks that count; and those this lane's row sees
+        if (!wait_or_abort(&bars->m_full[mi], mph, bars, pc, err, 20)) { ok = false; break; }
+        const uint2 mk = *reinterpret_cast<const uint2 *>(masks + mi * (kBlock / 32) + q * 2);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->m_empty[mi]);
+        if (++mi == kBStages) { mi = 0; mph ^= 1; }
+        uint32_t rmask0 = mk.x, rmask1 = mk.y;
+        if (CAUSAL) {        // keys at local index <= see
+          const int lim0 = see - (b * kBlock + q * kCols), lim1 = lim0 - 32;
+          rmask0 &= lim0 >= 31 ? 0xffffffffu : (lim0 < 0 ? 0u : (2u << lim0) - 1u);
+          rmask1 &= lim1 >= 31 ? 0xffffffffu : (lim1 < 0 ? 0u : (2u << lim1) - 1u);
         }
-        if (active && b + 1 < w.b1) {
-#pragma unroll
-          for (int c = 0; c < 2; ++c) {
-            const int key = key_base + kKeysPerBlock1 + c * 32 + lane;
-            mod_next[c] = key < t_end ? modality[key] : 0;
-          }
-        }
-        if (!wait_or_abort(&bars->acc_full[ci], cph, bars, err, 16)) { ok = false; break; }
+        if (!wait_or_abort(&bars->acc_full[ci], cph, bars, pc, err, 16)) { ok = false; break; }
         tc_fence_after();
-        if (active && (mask[0] | mask[1])) {
-          const uint32_t tcol = bars->tmem_base + lane_off + ci * 256 + t * 128 + h * 64;
-          uint32_t rr[64];
-          tmem_ld64_wait(tcol, rr);
+        if (mk.x | mk.y) {
+          const uint32_t tcol = bars->tmem_base + lane_off + ci * 256 + q * kCols;
+          uint32_t rr[kCols];
+          tmem_load_cols(tcol, rr);
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->acc_empty[ci]);   // registers hold the data: release early
-          online_chunk<0>(rr, rmask[0], c2, m, sum);
-          online_chunk<32>(rr, rmask[1], c2, m, sum);
+          if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);   // registers hold the data: release early
+          online_block(rr, rmask0, rmask1, c2, m, sum);
         } else {
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->acc_empty[ci]);
+          if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);
         }
         if (++ci == 2) { ci = 0; cph ^= 1; }
       }
       if (!ok) break;
-      // each column half is its own split partial; the merge combines them in a fixed order
-      const int rho = w.qp * 256 + row;                  // linear row of the head group
-      if (active && rho < G * sp.n_q) {
-        const int r = rho / G, j = rho - r * G;
-        part[(static_cast<size_t>(2 * w.split + h) * plan.total_qrows + sp.q_off + r) * plan.hq + w.g * G + j] =
-            make_float2(m, sum);
+      // the column ranges of each row combine in a fixed order (range 0 writes the pair's
+      // partial of the row group; the merge combines the pairs' partials in pair order)
+      float2 *cb = comb + (xph & 1) * (kEpiWG - 1) * kRows;
+      const int trow = quad * 32 + lane;
+      if (q > 0) {
+        if (!wait_or_abort(&bars->comb_empty[xph & 1], ((xph >> 1) & 1) ^ 1, bars, pc, err, 17)) break;
+        cb[(q - 1) * kRows + trow] = make_float2(m, sum);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->comb_full[xph & 1]);
+      } else {
+        if (!wait_or_abort(&bars->comb_full[xph & 1], (xph >> 1) & 1, bars, pc, err, 18)) break;
+        float2 v[kEpiWG];
+        v[0] = make_float2(m, sum);
+#pragma unroll
+        for (int i = 1; i < kEpiWG; ++i) v[i] = cb[(i - 1) * kRows + trow];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->comb_empty[xph & 1]);
+        float mm = v[0].x;
+#pragma unroll
+        for (int i = 1; i < kEpiWG; ++i) mm = fmaxf(mm, v[i].x);
+        float tot = 0.f;
+        if (mm != -INFINITY) {
+#pragma unroll
+          for (int i = 0; i < kEpiWG; ++i)
+            if (v[i].x != -INFINITY) tot += v[i].y * exp2f(v[i].x - mm);
+        }
+        const int rho = w.qp * kChunk + row;                  // linear row of the head group
+        if (rho < G * sp.n_q) {
+          const int r = rho / G, j = rho - r * G;
+          part[(static_cast<size_t>(w.slot) * plan.total_qrows + sp.q_off + r) * plan.hq + w.g * G + j] =
+              make_float2(mm, tot);
+        }
       }
+      ++xph;
     }
   }
-  finish_common(bars, warp, warp == 1 && lane == 0);
+  finish_pair(bars, pc, warp, warp == 1 && lane == 0 && pc.rank == 0);
 }
 
 // ------------------------------------------------------------------ repack
@@ -443,28 +635,30 @@ __global__ void q_pack_kernel(const __grid_constant__ ScorePlan plan, const uint
 }
 
 // ------------------------------------------------------------------ merge
-// One thread per normaliser entry (sequence, KV head, 128-row chunk, column);
-// writes -lse2 (padding columns -inf, so that they add exp2(-inf) = 0).
+// One thread per packed query row (sequence, KV head group, rho); writes -lse2 at the
+// row's packed index (padding rows -inf, so that they add exp2(-inf) = 0).
 __global__ void lse_merge_kernel(const __grid_constant__ ScorePlan plan, const float2 *__restrict__ part,
-                                 float *__restrict__ nlse2, int64_t n_entries, int64_t entry_base) {
+                                 float *__restrict__ nlse2, int64_t row_begin, int64_t n_rows) {
   const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (e >= n_entries) return;
-  const int64_t chunk = entry_base / kBRows + e / kBRows;
-  const int col = static_cast<int>(e % kBRows);
+  if (e >= n_rows) return;
+  const int64_t prow = row_begin + e;
   int s = 0;
-  while (s + 1 < plan.nseq && plan.seq[s + 1].chunk_base <= chunk) ++s;
+  while (s + 1 < plan.nseq && plan.seq[s + 1].qp_base <= prow) ++s;
   const SeqPlan &sp = plan.seq[s];
   const int G = plan.group;
-  const int nch = n_chunks(sp, G);
-  const int local = static_cast<int>(chunk - sp.chunk_base);
-  const int g = local / nch, c = local - g * nch;
-  const int rho = c * kBRows + col;
+  const int local = static_cast<int>(prow - sp.qp_base);
+  const int g = local / sp.rows_pad, rho = local - g * sp.rows_pad;
   float out = -INFINITY;
   if (rho < G * sp.n_q) {
     const int r = rho / G, j = rho - r * G;
     const int qrow = sp.q_off + r;
     const int h = g * G + j;
-    const int np = 2 * sp.n_split;   // two column halves per split
+    // the pair ranges that touched this row group, one partial each
+    const int grp = g * n_pairs(sp) + rho / kChunk;
+    const int x0 = sp.flat0 + grp * sp.nb;
+    const int np = sp.nb > 0 ? static_cast<int>(pair_of(x0 + sp.nb - 1, plan.pairs, plan.flat_total) -
+                                                pair_of(x0, plan.pairs, plan.flat_total) + 1)
+                             : 0;
     float mm = -INFINITY;
     for (int p = 0; p < np; ++p)
       mm = fmaxf(mm, part[(static_cast<size_t>(p) * plan.total_qrows + qrow) * plan.hq + h].x);
@@ -479,28 +673,28 @@ __global__ void lse_merge_kernel(const __grid_constant__ ScorePlan plan, const f
       out = -(mm + log2f(tot));
     }
   }
-  nlse2[chunk * kBRows + col] = out;
+  nlse2[prow] = out;
 }
 
 // ------------------------------------------------------------------ pass 2
 struct Unit2 {
-  int s, kp, g, ntiles;
+  int s, kp, g;
 };
 
 __device__ __forceinline__ Unit2 decode_unit2(const ScorePlan &p, int u) {
   Unit2 w;
-  w.s = find_seq(p, u);
-  const int local = u - p.seq[w.s].unit_begin;
+  int s = 0;
+  while (s + 1 < p.nseq && p.seq[s + 1].unit_begin <= u) ++s;
+  w.s = s;
+  const int local = u - p.seq[s].unit_begin;
   w.g = local % p.hkv;
   w.kp = local / p.hkv;
-  const int keys = min(kKeysPerUnit2, p.seq[w.s].len - w.kp * kKeysPerUnit2);
-  w.ntiles = keys > 128 ? 2 : 1;
   return w;
 }
 
 // a[0..3] += 2^(x c2 + nl[col]) over 32 columns (four independent partial sums).
 template <int OFF>
-__device__ __forceinline__ void colsum_chunk(const uint32_t (&r)[64], const float *nl, float c2, float2 (&a)[4]) {
+__device__ __forceinline__ void colsum_chunk(const uint32_t (&r)[kCols], const float *nl, float c2, float2 (&a)[4]) {
   const float2 cc = make_float2(c2, c2);
 #pragma unroll
   for (int i = 0; i < 32; i += 4) {
@@ -517,31 +711,32 @@ __device__ __forceinline__ void colsum_chunk(const uint32_t (&r)[64], const floa
 // The same over the columns OFF + i >= first only (causal rows that cannot see the key drop out;
 // taken only by keys inside the query span).
 template <int OFF>
-__device__ __forceinline__ void colsum_chunk_from(const uint32_t (&r)[64], const float *nl, float c2, int first,
+__device__ __forceinline__ void colsum_chunk_from(const uint32_t (&r)[kCols], const float *nl, float c2, int first,
                                                   float2 (&a)[4]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i)
     if (OFF + i >= first) a[i & 3].x += ex2_approx(fmaf(__uint_as_float(r[OFF + i]), c2, nl[i]));
 }
 
-// Work unit = (256-key pair, KV head group g); writes the group's sum for each
-// key to gsum[g][key]; the final kernel adds the groups.
+// Work unit = (256 keys, KV head group g): 128 keys per CTA of the pair; writes the group's
+// sum for each key to gsum[g][key]; the final kernel adds the groups.
 template <bool CAUSAL>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     score_colsum_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                         const __grid_constant__ ScorePlan plan, const float *__restrict__ nlse2,
                         float *__restrict__ gsum, DeviceError *err) {
   extern __shared__ __align__(1024) uint8_t smem[];
-  if (!smem_aligned(smem)) {
+  if (!smem_aligned(smem)) {   // the same in both CTAs of the pair: both leave here
     if (threadIdx.x == 0) raise_device_error(err, APACK_EDEVICE, 10);
     return;
   }
   Bars *bars = reinterpret_cast<Bars *>(smem + kOffBars);
-  float *lse_s = reinterpret_cast<float *>(smem + kOffL);   // [3][128], indexed by B stage
+  float *lse_s = reinterpret_cast<float *>(smem + kOffL);   // [4][256], indexed by B stage
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  init_common(smem, bars, warp);
+  const PairCtx pc = init_pair(smem, bars, warp);
   const int G = plan.group;
-  constexpr uint32_t b_tx = kBBytes + kBRows * sizeof(float);
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const int row_half = static_cast<int>(pc.rank) * kRows;   // this CTA's keys of a unit, rows of a chunk
 
   if (warp == 0) {
     if (lane == 0) {
@@ -552,30 +747,32 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool pend[kBStages] = {}, apend[kAStages] = {};
       uint32_t pend_par[kBStages] = {}, apend_par[kAStages] = {};
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < plan.total_units; u += gridDim.x) {
+      for (int u = pair; ok && u < plan.total_units; u += npairs) {
         const Unit2 w = decode_unit2(plan, u);
         const SeqPlan &sp = plan.seq[w.s];
-        const int nch = n_chunks(sp, G);
+        const int nch = sp.rows_pad / kChunk;
         if (nch == 0) continue;
-        if (!wait_or_abort(&bars->a_empty[ai], aph ^ 1, bars, err, 21)) { ok = false; break; }
-        uint8_t *A = smem + kOffA + ai * kABytes;
-        mbar_arrive_expect_tx(&bars->a_full[ai], kABytes);
-        const int key0 = sp.t0 + w.kp * kKeysPerUnit2;
-        tma_load_3d(A, &kmap, &bars->a_full[ai], 0, w.g, key0);
-        tma_load_3d(A + kAHalf, &kmap, &bars->a_full[ai], 64, w.g, key0);
+        if (!wait_or_abort(&bars->a_empty[ai], aph ^ 1, bars, pc, err, 21)) { ok = false; break; }
+        uint8_t *A = smem + kOffA + ai * kTileBytes;
+        if (pc.rank == 0) mbar_arrive_expect_tx(&bars->a_full[ai], 2 * kTileBytes);
+        const uint32_t afull = lead_addr(pc, bars, &bars->a_full[ai]);
+        const int key0 = sp.t0 + w.kp * kBlock + row_half;
+        tma_load_3d_pair(A, &kmap, afull, 0, w.g, key0);
+        tma_load_3d_pair(A + kHalf, &kmap, afull, 64, w.g, key0);
         apend[ai] = true;
         apend_par[ai] = aph;
         for (int c = 0; c < nch; ++c) {
-          if (!wait_or_abort(&bars->b_empty[bi], bph ^ 1, bars, err, 22)) { ok = false; break; }
-          // normaliser slot bi is free once the epilogue of the chunk that used it is done
-          if (!wait_or_abort(&bars->l_empty[bi], bph ^ 1, bars, err, 29)) { ok = false; break; }
-          uint8_t *B = smem + kOffB + bi * kBBytes;
-          mbar_arrive_expect_tx(&bars->b_full[bi], b_tx);
-          const int brow = sp.qp_base + w.g * sp.rows_pad + c * kBRows;
-          tma_load_3d(B, &qmap, &bars->b_full[bi], 0, 0, brow);
-          tma_load_3d(B + kBHalf, &qmap, &bars->b_full[bi], 64, 0, brow);
-          bulk_load(lse_s + bi * kBRows, nlse2 + (static_cast<int64_t>(sp.chunk_base) + w.g * nch + c) * kBRows,
-                    kBRows * sizeof(float), &bars->b_full[bi]);
+          if (!wait_or_abort(&bars->b_empty[bi], bph ^ 1, bars, pc, err, 22)) { ok = false; break; }
+          // normaliser slot bi is free once this CTA's epilogue of the chunk that used it is done
+          if (!wait_or_abort(&bars->l_empty[bi], bph ^ 1, bars, pc, err, 29)) { ok = false; break; }
+          const int64_t row0 = static_cast<int64_t>(sp.qp_base) + w.g * sp.rows_pad + c * kChunk;
+          mbar_arrive_expect_tx(&bars->l_full[bi], kChunk * sizeof(float));
+          bulk_load(lse_s + bi * kChunk, nlse2 + row0, kChunk * sizeof(float), &bars->l_full[bi]);
+          uint8_t *B = smem + kOffB + bi * kTileBytes;
+          if (pc.rank == 0) mbar_arrive_expect_tx(&bars->b_full[bi], 2 * kTileBytes);
+          const uint32_t bfull = lead_addr(pc, bars, &bars->b_full[bi]);
+          tma_load_3d_pair(B, &qmap, bfull, 0, 0, static_cast<int32_t>(row0) + row_half);
+          tma_load_3d_pair(B + kHalf, &qmap, bfull, 64, 0, static_cast<int32_t>(row0) + row_half);
           pend[bi] = true;
           pend_par[bi] = bph;
           if (++bi == kBStages) { bi = 0; bph ^= 1; }
@@ -583,111 +780,110 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (++ai == kAStages) { ai = 0; aph ^= 1; }
       }
       if (!ok) {
-        drain_loads(bars->b_full, pend, pend_par, kBStages);
-        drain_loads(bars->a_full, apend, apend_par, kAStages);
+        // this CTA's normaliser copies complete on its own barriers
+        drain_loads(bars->l_full, pend, pend_par, kBStages);
+        if (pc.rank == 0) {
+          drain_loads(bars->b_full, pend, pend_par, kBStages);
+          drain_loads(bars->a_full, apend, apend_par, kAStages);
+        }
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && pc.rank == 0) {
       int ai = 0, bi = 0, ci = 0;
       uint32_t aph = 0, bph = 0, cph = 0;
       const uint32_t tmem = bars->tmem_base;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < plan.total_units; u += gridDim.x) {
+      for (int u = pair; ok && u < plan.total_units; u += npairs) {
         const Unit2 w = decode_unit2(plan, u);
-        const int nch = n_chunks(plan.seq[w.s], G);
+        const int nch = plan.seq[w.s].rows_pad / kChunk;
         if (nch == 0) continue;
-        if (!wait_or_abort(&bars->a_full[ai], aph, bars, err, 23)) { ok = false; break; }
-        const uint32_t a_base = smem_u32(smem + kOffA + ai * kABytes);
+        if (!wait_or_abort(&bars->a_full[ai], aph, bars, pc, err, 23)) { ok = false; break; }
+        const uint32_t a_base = smem_u32(smem + kOffA + ai * kTileBytes);
         for (int c = 0; c < nch; ++c) {
-          if (!wait_or_abort(&bars->b_full[bi], bph, bars, err, 24)) { ok = false; break; }
-          if (!wait_or_abort(&bars->acc_empty[ci], cph ^ 1, bars, err, 25)) { ok = false; break; }
+          if (!wait_or_abort(&bars->b_full[bi], bph, bars, pc, err, 24)) { ok = false; break; }
+          if (!wait_or_abort(&bars->acc_empty[ci], cph ^ 1, bars, pc, err, 25)) { ok = false; break; }
           tc_fence_after();
-          issue_mma_pair(tmem, ci, a_base, smem_u32(smem + kOffB + bi * kBBytes), w.ntiles);
-          tc_commit(&bars->b_empty[bi]);
-          tc_commit(&bars->acc_full[ci]);
+          issue_mma(tmem, ci, a_base, smem_u32(smem + kOffB + bi * kTileBytes));
+          commit_pair(&bars->b_empty[bi]);
+          commit_pair(&bars->acc_full[ci]);
           if (++bi == kBStages) { bi = 0; bph ^= 1; }
           if (++ci == 2) { ci = 0; cph ^= 1; }
         }
         if (!ok) break;
-        tc_commit(&bars->a_empty[ai]);
+        commit_pair(&bars->a_empty[ai]);
         if (++ai == kAStages) { ai = 0; aph ^= 1; }
       }
     }
-  } else {
-    // Epilogue: warpgroup q = (t, h) reads columns h*64.. of key tile t; one key per thread.
+  } else if (warp < kMaskWarp) {
+    // Epilogue: warpgroup q reads columns q*kCols.. (rows of the chunk); one key per thread.
     const int q = (warp - 2) >> 2;
-    const int t = q & 1, h = q >> 1;
     const int quad = warp & 3;
     const int tkey = quad * 32 + lane;
-    const int klane = t * 128 + tkey;
+    const int klane = row_half + tkey;                  // key of the 256-key unit
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    const uint32_t acc_empty0 = lead_addr(pc, bars, &bars->acc_empty[0]);
     const float c2 = plan.scale2;
-    float *comb = reinterpret_cast<float *>(smem + kOffC) + t * 128;
+    float *comb = reinterpret_cast<float *>(smem + kOffC);   // [2 parities][kEpiWG - 1 ranges][128 keys]
     int ci = 0, li = 0;
-    uint32_t cph = 0, xph = 0;
+    uint32_t cph = 0, lph = 0, xph = 0;
     bool ok = true;
-    for (int u = blockIdx.x; ok && u < plan.total_units; u += gridDim.x) {
+    for (int u = pair; ok && u < plan.total_units; u += npairs) {
       const Unit2 w = decode_unit2(plan, u);
       const SeqPlan &sp = plan.seq[w.s];
-      const int nch = n_chunks(sp, G);
+      const int nch = sp.rows_pad / kChunk;
       if (nch == 0) continue;
-      const bool active = t < w.ntiles;
       float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
       // causal rows: only packed rows rho >= rho_min (tokens r >= key - (len - n_q)) see this key
-      const int rho_min = CAUSAL ? max(0, w.kp * kKeysPerUnit2 + klane - (sp.len - sp.n_q)) * G : 0;
+      const int rho_min = CAUSAL ? max(0, w.kp * kBlock + klane - (sp.len - sp.n_q)) * G : 0;
       for (int c = 0; c < nch; ++c) {
-        if (!wait_or_abort(&bars->acc_full[ci], cph, bars, err, 26)) { ok = false; break; }
+        if (!wait_or_abort(&bars->l_full[li], lph, bars, pc, err, 30)) { ok = false; break; }
+        if (!wait_or_abort(&bars->acc_full[ci], cph, bars, pc, err, 26)) { ok = false; break; }
         tc_fence_after();
-        if (active) {
-          const float *nl = lse_s + li * kBRows + h * 64;
-          const uint32_t tcol = bars->tmem_base + lane_off + ci * 256 + t * 128 + h * 64;
-          uint32_t rr[64];
-          tmem_ld64_wait(tcol, rr);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->acc_empty[ci]);   // registers hold the data: release early
-          const int first = rho_min - (c * kBRows + h * 64);
-          if (!CAUSAL || first <= 0) {
-            colsum_chunk<0>(rr, nl, c2, a);
-            colsum_chunk<32>(rr, nl + 32, c2, a);
-          } else if (first < 64) {
-            colsum_chunk_from<0>(rr, nl, c2, first, a);
-            colsum_chunk_from<32>(rr, nl + 32, c2, first, a);
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->l_empty[li]);
-        } else {
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) {
-            mbar_arrive(&bars->acc_empty[ci]);
-            mbar_arrive(&bars->l_empty[li]);
-          }
+        const float *nl = lse_s + li * kChunk + q * kCols;
+        const uint32_t tcol = bars->tmem_base + lane_off + ci * 256 + q * kCols;
+        uint32_t rr[kCols];
+        tmem_load_cols(tcol, rr);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);   // registers hold the data: release early
+        const int first = rho_min - (c * kChunk + q * kCols);
+        if (!CAUSAL || first <= 0) {
+          colsum_chunk<0>(rr, nl, c2, a);
+          colsum_chunk<32>(rr, nl + 32, c2, a);
+        } else if (first < kCols) {
+          colsum_chunk_from<0>(rr, nl, c2, first, a);
+          colsum_chunk_from<32>(rr, nl + 32, c2, first, a);
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->l_empty[li]);
         if (++ci == 2) { ci = 0; cph ^= 1; }
-        if (++li == kBStages) li = 0;
+        if (++li == kBStages) { li = 0; lph ^= 1; }
       }
       if (!ok) break;
-      if (!active) continue;
       const float2 s01 = fadd2(a[0], a[1]), s23 = fadd2(a[2], a[3]);
       const float2 s4 = fadd2(s01, s23);
       const float mine = s4.x + s4.y;
-      if (h == 1) {
-        if (!wait_or_abort(&bars->comb_empty[t], xph ^ 1, bars, err, 27)) break;
-        comb[tkey] = mine;
-        mbar_arrive(&bars->comb_full[t]);
+      float *cb = comb + (xph & 1) * (kEpiWG - 1) * kRows;
+      if (q > 0) {
+        if (!wait_or_abort(&bars->comb_empty[xph & 1], ((xph >> 1) & 1) ^ 1, bars, pc, err, 27)) break;
+        cb[(q - 1) * kRows + tkey] = mine;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->comb_full[xph & 1]);
       } else {
-        if (!wait_or_abort(&bars->comb_full[t], xph, bars, err, 28)) break;
-        const float other = comb[tkey];
-        mbar_arrive(&bars->comb_empty[t]);
-        const int key = sp.t0 + w.kp * kKeysPerUnit2 + klane;
-        if (key < sp.t0 + sp.len) gsum[static_cast<int64_t>(w.g) * plan.total_tokens + key] = mine + other;
+        if (!wait_or_abort(&bars->comb_full[xph & 1], (xph >> 1) & 1, bars, pc, err, 28)) break;
+        float tot = mine;
+#pragma unroll
+        for (int i = 1; i < kEpiWG; ++i) tot += cb[(i - 1) * kRows + tkey];   // fixed order
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->comb_empty[xph & 1]);
+        const int key = sp.t0 + w.kp * kBlock + klane;
+        if (key < sp.t0 + sp.len) gsum[static_cast<int64_t>(w.g) * plan.total_tokens + key] = tot;
       }
-      xph ^= 1;
+      ++xph;
     }
   }
-  finish_common(bars, warp, warp == 1 && lane == 0);
+  finish_pair(bars, pc, warp, warp == 1 && lane == 0 && pc.rank == 0);
 }
 
 // ------------------------------------------------------------------ final
@@ -744,6 +940,31 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t mid, uint64_t rows, u
 }
 
 std::atomic<uint64_t> g_attr_done{0};
+std::atomic<int> g_max_pairs[64];   // per device: CTA pairs that can be resident at once (0 = not probed)
+
+// CTA pairs of the scoring kernels that fit the device at once (one CTA per SM).
+int max_resident_pairs() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 1;
+  if (dev < 64) {
+    const int cached = g_max_pairs[dev].load(std::memory_order_relaxed);
+    if (cached > 0) return cached;
+  }
+  int n = 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * (device_sm_count() / 2), 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  // the kernels declare their cluster shape (__cluster_dims__), so the configuration leaves it out
+  if (cudaOccupancyMaxActiveClusters(&n, score_colsum_kernel<false>, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = device_sm_count() / 2;
+  }
+  if (n > device_sm_count() / 2) n = device_sm_count() / 2;
+  if (n < 1) n = 1;
+  if (dev < 64) g_max_pairs[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
 
 }  // namespace
 
@@ -766,7 +987,7 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
   const int hq = seqs->num_q_heads, hkv = seqs->num_kv_heads, G = hq / hkv;
   if (hkv > 256) return APACK_EUNSUPPORTED;
   if (T == 0) return APACK_OK;
-  // few query rows per head group (e.g. the last query token only): K-read-bound CUDA-core path
+  // few query rows per head group (e.g. the last query token only): K-read-bound path
   if (narrow_score_applies(seqs)) return run_score_narrow(seqs, q, k, k_token_stride, scores, ws, stream);
   const WsLayout L = workspace_layout(seqs);
   uint8_t *wsb = static_cast<uint8_t *>(ws);
@@ -791,17 +1012,14 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
         return e;
       }) != cudaSuccess)
     return APACK_ECUDA;
-  CUtensorMap qmap1, kmap1, qmap2, kmap2;
+  CUtensorMap qmap, kmap;
   const uint64_t qp_rows = static_cast<uint64_t>(L.qp_rows > 0 ? L.qp_rows : 256);
-  // pass 1: A = 256-row pairs of packed Q, B = 128-key blocks; pass 2: A = 256 keys, B = 128-row chunks
-  if (!make_map(&qmap1, qp, 1, qp_rows, 256, 256, 1, 256) ||
-      !make_map(&kmap1, k, hkv, T, 256, k_token_stride, 1, kKeysPerBlock1) ||
-      !make_map(&qmap2, qp, 1, qp_rows, 256, 256, 1, kBRows) ||
-      !make_map(&kmap2, k, hkv, T, 256, k_token_stride, 1, kKeysPerUnit2))
+  // every operand tile is 128 rows (of packed Q or of one KV head's keys) per CTA
+  if (!make_map(&qmap, qp, 1, qp_rows, 256, 256, 1, kRows) || !make_map(&kmap, k, hkv, T, 256, k_token_stride, 1, kRows))
     return APACK_ECUDA;
 
-  const int sms = device_sm_count();
-  int64_t chunk_base = 0, qp_base = 0;
+  const int max_pairs = max_resident_pairs();
+  int64_t qp_base = 0;
   for (int s0 = 0; s0 < B; s0 += kSeqsPerLaunch) {
     const int ns = (B - s0 < kSeqsPerLaunch) ? (B - s0) : kSeqsPerLaunch;
     ScorePlan P{};
@@ -813,7 +1031,8 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
     P.total_tokens = static_cast<int32_t>(T);
     P.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(APACK_HEAD_DIM)));
     P.causal = seqs->softmax_domain == APACK_SOFTMAX_CAUSAL_ROW;
-    int64_t chunks = 0, qrows = 0, work = 0;
+    int64_t qrows = 0, flat = 0, nb_max = 0;
+    int units2 = 0;
     for (int i = 0; i < ns; ++i) {
       const int b = s0 + i;
       SeqPlan &sp = P.seq[i];
@@ -821,28 +1040,28 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
       sp.len = seqs->cu_seqlens_h[b + 1] - sp.t0;
       sp.q_off = seqs->cu_qlens_h[b];
       sp.n_q = seqs->cu_qlens_h[b + 1] - sp.q_off;
-      sp.rows_pad = ((G * sp.n_q + 255) / 256) * 256;
+      sp.rows_pad = ((G * sp.n_q + kChunk - 1) / kChunk) * kChunk;
       sp.qp_base = static_cast<int32_t>(qp_base + qrows);
       qrows += static_cast<int64_t>(hkv) * sp.rows_pad;
-      sp.chunk_base = static_cast<int32_t>(chunk_base + chunks);
-      chunks += static_cast<int64_t>(hkv) * n_chunks(sp, G);
-      work += static_cast<int64_t>((sp.len + kKeysPerBlock1 - 1) / kKeysPerBlock1) * hkv * n_pairs(sp);
+      sp.nb = sp.n_q > 0 ? (sp.len + kBlock - 1) / kBlock : 0;
+      sp.flat0 = static_cast<int32_t>(flat);
+      flat += pass1_items(sp, hkv);
+      if (sp.nb > nb_max) nb_max = sp.nb;
+      sp.unit_begin = units2;
+      if (sp.rows_pad > 0) units2 += ((sp.len + kBlock - 1) / kBlock) * hkv;
     }
-    // Pass 1 units: (split, head group, query pair); splits sized for a few units per SM.
-    const int64_t target_units = 4LL * sms;
-    int64_t bps_all = (work + target_units - 1) / target_units;
-    if (bps_all < 4) bps_all = 4;
-    int units1 = 0, units2 = 0;
-    for (int i = 0; i < ns; ++i) {
-      SeqPlan &sp = P.seq[i];
-      const int nb = (sp.len + kKeysPerBlock1 - 1) / kKeysPerBlock1;
-      int bps = static_cast<int>(bps_all);
-      if ((nb + bps - 1) / bps > kMaxSplits / 2) bps = (nb + kMaxSplits / 2 - 1) / (kMaxSplits / 2);
-      sp.bps = bps > 0 ? bps : 1;
-      sp.n_split = (sp.n_q > 0 && nb > 0) ? (nb + sp.bps - 1) / sp.bps : 0;
-      sp.unit_begin = units1;
-      units1 += sp.n_split * hkv * n_pairs(sp);
+    // Pass 1: equal ranges of the flat (row group, key block) items per pair; a range must stay at
+    // least ceil(nb_max / (kPairSlots - 1)) items long so that a row group meets at most kPairSlots
+    // pairs (its partial slots).
+    if (flat >= (int64_t{1} << 31) - 1) return APACK_EUNSUPPORTED;   // flat indices are 32-bit on the device
+    P.flat_total = static_cast<int32_t>(flat);
+    int64_t pairs1 = max_pairs;
+    if (flat > 0) {
+      const int64_t min_len = (nb_max + kPairSlots - 2) / (kPairSlots - 1);
+      if (pairs1 > flat / min_len) pairs1 = flat / min_len;
+      if (pairs1 < 1) pairs1 = 1;
     }
+    P.pairs = static_cast<int32_t>(pairs1);
     // repack the query rows of this launch's sequences
     if (qrows > 0) {
       const int64_t n_vec = qrows * 16;
@@ -851,35 +1070,30 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
-    P.total_units = units1;
-    if (units1 > 0) {
-      const int grid = units1 < sms ? units1 : sms;
+    if (flat > 0) {
+      const unsigned grid = static_cast<unsigned>(2 * pairs1);
       if (P.causal)
-        score_rowstats_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap1, kmap1, P, seqs->modality, part, err);
+        score_rowstats_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, seqs->modality, part, err);
       else
-        score_rowstats_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap1, kmap1, P, seqs->modality, part, err);
+        score_rowstats_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, seqs->modality, part, err);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
-    if (chunks > 0) {
-      const int64_t n_entries = chunks * kBRows;
-      lse_merge_kernel<<<static_cast<unsigned>((n_entries + 255) / 256), 256, 0, stream>>>(P, part, nlse2, n_entries,
-                                                                                          chunk_base * kBRows);
+    if (qrows > 0) {
+      lse_merge_kernel<<<static_cast<unsigned>((qrows + 255) / 256), 256, 0, stream>>>(P, part, nlse2, qp_base,
+                                                                                       qrows);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
-    // Pass 2 units: (256-key pair, head group).
-    for (int i = 0; i < ns; ++i) {
-      P.seq[i].unit_begin = units2;
-      units2 += n_keypairs(P.seq[i]) * hkv;
-    }
+    // Pass 2 units: (256 keys, head group), dealt round-robin to the pairs.
     P.total_units = units2;
     if (units2 > 0) {
-      const int grid = units2 < sms ? units2 : sms;
+      const int pairs2 = units2 < max_pairs ? units2 : max_pairs;
+      const unsigned grid = static_cast<unsigned>(2 * pairs2);
       if (P.causal)
-        score_colsum_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap2, kmap2, P, nlse2, gsum, err);
+        score_colsum_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, nlse2, gsum, err);
       else
-        score_colsum_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap2, kmap2, P, nlse2, gsum, err);
+        score_colsum_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, nlse2, gsum, err);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
@@ -891,7 +1105,6 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
-    chunk_base += chunks;
     qp_base += qrows;
   }
   return APACK_OK;
