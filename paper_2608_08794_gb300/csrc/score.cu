@@ -11,7 +11,8 @@
 //     contiguous ranges, one per CTA pair; a pair writes one partial (m, sum) per
 //     row for each row group its range touches.
 //  merge: per packed query row, the partials combine into a log2-domain
-//     normaliser lse2 = log2 sum_j 2^(x_j log2(e)/sqrt(D)), stored negated.
+//     normaliser lse2 = log2 sum_j 2^(x_j log2(e)/sqrt(D)), stored negated (a row whose
+//     logits overflowed its run's reference is recomputed there exactly).
 //  pass 2 (column sums): D[key][row] = K . Q^T with keys in TMEM lanes; each
 //     thread owns one key and sums 2^(x c - lse2[row]) over the rows of one KV
 //     head group; a final pass adds the Hkv group sums in a fixed order and
@@ -341,11 +342,15 @@ __device__ __forceinline__ Run next_run(const ScorePlan &p, int x, int x_end, in
 
 // Online (reference, sum) update with a thread's 64 logits of a block, in log2 units.  Keys
 // that do not count are first replaced by -inf (exp2 gives 0), so that one code path serves
-// every mask.  The reference is the first counted block's maximum and is only raised when a
-// block's sum exceeds 2^64 (or overflows): the maximum stays off the common path.  Four
-// independent partial sums keep the add chains short.
+// every mask.  The reference is the first counted block's maximum and stays fixed for the
+// run: no block's sums feed back into the next block's arithmetic.  A block whose sum leaves
+// the safe range (a logit more than about 2^99 above the reference, or an overflow) only sets
+// `bad`; such a row's normaliser is recomputed exactly by the merge kernel.  Four independent
+// partial sums keep the add chains short.
+constexpr float kSumLimit = 6.338253e29f;   // 2^99
+
 __device__ __forceinline__ void online_block(uint32_t (&r)[64], uint32_t mask0, uint32_t mask1, float c2, float &m,
-                                             float &sum) {
+                                             float &sum, bool &bad) {
   if ((mask0 & mask1) != 0xffffffffu) {
     if ((mask0 | mask1) == 0u) return;
     const uint32_t ninf = __float_as_uint(-INFINITY);
@@ -370,18 +375,8 @@ __device__ __forceinline__ void online_block(uint32_t (&r)[64], uint32_t mask0, 
   }
   const float2 s01 = fadd2(a[0], a[1]), s23 = fadd2(a[2], a[3]);
   const float2 s4 = fadd2(s01, s23);
-  float t = s4.x + s4.y;
-  if (!(t <= 1.8446744e19f)) {   // a value exceeded the reference by more than 2^64 (or inf): rescale
-    float mx = __uint_as_float(r[0]);
-#pragma unroll
-    for (int i = 1; i < 64; ++i) mx = fmaxf(mx, __uint_as_float(r[i]));
-    mx *= c2;
-    sum *= ex2_approx(m - mx);
-    m = mx;
-    t = 0.f;
-#pragma unroll
-    for (int i = 0; i < 64; ++i) t += ex2_approx(fmaf(__uint_as_float(r[i]), c2, -m));
-  }
+  const float t = s4.x + s4.y;
+  bad |= !(t <= kSumLimit);
   sum += t;
 }
 
@@ -539,6 +534,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const SeqPlan &sp = plan.seq[w.s];
       x = w.x1;
       float m = -INFINITY, sum = 0.f;
+      bool bad = false;
       // causal rows: this lane's row (token r of the query span) sees keys up to len - n_q + r
       const int see = sp.len - sp.n_q + (w.qp * kChunk + row) / G;
       for (int b = w.b0; b < w.b1; ++b) {
@@ -563,7 +559,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);   // registers hold the data: release early
-          online_block(rr, rmask0, rmask1, c2, m, sum);
+          online_block(rr, rmask0, rmask1, c2, m, sum, bad);
         } else {
           tc_fence_before();
           __syncwarp();
@@ -573,7 +569,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       if (!ok) break;
       // the column ranges of each row combine in a fixed order (range 0 writes the pair's
-      // partial of the row group; the merge combines the pairs' partials in pair order)
+      // partial of the row group; the merge combines the pairs' partials in pair order).  A
+      // sum out of range travels as a negative sum: the merge then recomputes the row.
+      if (bad) sum = -1.f;
       float2 *cb = comb + (xph & 1) * (kEpiWG - 1) * kRows;
       const int trow = quad * 32 + lane;
       if (q > 0) {
@@ -590,14 +588,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->comb_empty[xph & 1]);
         float mm = v[0].x;
+        bool flagged = v[0].y < 0.f;
 #pragma unroll
-        for (int i = 1; i < kEpiWG; ++i) mm = fmaxf(mm, v[i].x);
+        for (int i = 1; i < kEpiWG; ++i) {
+          mm = fmaxf(mm, v[i].x);
+          flagged |= v[i].y < 0.f;
+        }
         float tot = 0.f;
         if (mm != -INFINITY) {
 #pragma unroll
           for (int i = 0; i < kEpiWG; ++i)
             if (v[i].x != -INFINITY) tot += v[i].y * exp2f(v[i].x - mm);
         }
+        if (flagged) tot = -1.f;
         const int rho = w.qp * kChunk + row;                  // linear row of the head group
         if (rho < G * sp.n_q) {
           const int r = rho / G, j = rho - r * G;
@@ -635,11 +638,23 @@ __global__ void q_pack_kernel(const __grid_constant__ ScorePlan plan, const uint
 }
 
 // ------------------------------------------------------------------ merge
-// One thread per packed query row (sequence, KV head group, rho); writes -lse2 at the
-// row's packed index (padding rows -inf, so that they add exp2(-inf) = 0).
+// One warp per packed query row (sequence, KV head group, rho); writes -lse2 at the row's
+// packed index (padding rows -inf, so that they add exp2(-inf) = 0).  Lane p takes the partial
+// of pair range p (at most 32), and a fixed shuffle tree combines them: deterministic.
+//
+// A row with a partial marked out of range (negative sum: a logit far above its run's
+// reference) is recomputed exactly here instead: the warp's lanes take every 32nd key of
+// the sequence, dot it with the row's query vector in fp32 from the bf16 values, keep an
+// online (max, sum of exp2) with exact rescaling, and combine in a fixed order.  Slow, and
+// only taken for inputs whose logits span more than about 99 binary orders of magnitude.
+template <bool CAUSAL>
 __global__ void lse_merge_kernel(const __grid_constant__ ScorePlan plan, const float2 *__restrict__ part,
-                                 float *__restrict__ nlse2, int64_t row_begin, int64_t n_rows) {
-  const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+                                 const uint16_t *__restrict__ qp, const uint8_t *__restrict__ k,
+                                 int64_t k_stride, const uint8_t *__restrict__ modality, float *__restrict__ nlse2,
+                                 int64_t row_begin, int64_t n_rows) {
+  __shared__ float qsh[8][128];                           // the query row of each warp (fallback only)
+  const int64_t e = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   if (e >= n_rows) return;
   const int64_t prow = row_begin + e;
   int s = 0;
@@ -648,32 +663,60 @@ __global__ void lse_merge_kernel(const __grid_constant__ ScorePlan plan, const f
   const int G = plan.group;
   const int local = static_cast<int>(prow - sp.qp_base);
   const int g = local / sp.rows_pad, rho = local - g * sp.rows_pad;
-  float out = -INFINITY;
-  if (rho < G * sp.n_q) {
-    const int r = rho / G, j = rho - r * G;
-    const int qrow = sp.q_off + r;
-    const int h = g * G + j;
-    // the pair ranges that touched this row group, one partial each
-    const int grp = g * n_pairs(sp) + rho / kChunk;
-    const int x0 = sp.flat0 + grp * sp.nb;
-    const int np = sp.nb > 0 ? static_cast<int>(pair_of(x0 + sp.nb - 1, plan.pairs, plan.flat_total) -
-                                                pair_of(x0, plan.pairs, plan.flat_total) + 1)
-                             : 0;
-    float mm = -INFINITY;
-    for (int p = 0; p < np; ++p)
-      mm = fmaxf(mm, part[(static_cast<size_t>(p) * plan.total_qrows + qrow) * plan.hq + h].x);
-    if (mm == -INFINITY) {
-      out = INFINITY;   // no key at all (S empty): no score is written for this sequence
-    } else {
-      float tot = 0.f;
-      for (int p = 0; p < np; ++p) {
-        const float2 v = part[(static_cast<size_t>(p) * plan.total_qrows + qrow) * plan.hq + h];
-        if (v.x != -INFINITY) tot += v.y * exp2f(v.x - mm);
-      }
-      out = -(mm + log2f(tot));
-    }
+  if (rho >= G * sp.n_q) {
+    if (lane == 0) nlse2[prow] = -INFINITY;
+    return;
   }
-  nlse2[prow] = out;
+  const int r = rho / G, j = rho - r * G;
+  const int qrow = sp.q_off + r;
+  const int h = g * G + j;
+  // the pair ranges that touched this row group, one partial each
+  const int grp = g * n_pairs(sp) + rho / kChunk;
+  const int x0 = sp.flat0 + grp * sp.nb;
+  const int np = sp.nb > 0 ? pair_of(x0 + sp.nb - 1, plan.pairs, plan.flat_total) -
+                                 pair_of(x0, plan.pairs, plan.flat_total) + 1
+                           : 0;
+  float2 v = make_float2(-INFINITY, 0.f);
+  if (lane < np) v = part[(static_cast<size_t>(lane) * plan.total_qrows + qrow) * plan.hq + h];
+  float out;
+  if (__ballot_sync(0xffffffffu, v.y < 0.f) == 0u) {
+    float mm = v.x;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, o));
+    float tot = (v.x != -INFINITY) ? v.y * exp2f(v.x - mm) : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+    out = mm == -INFINITY ? INFINITY : -(mm + log2f(tot));   // no key at all (S empty): nothing is scored
+  } else {
+    float *qv = qsh[wib];
+    const uint16_t *qr = qp + prow * 128;
+    for (int d = lane; d < 128; d += 32) qv[d] = __uint_as_float(static_cast<uint32_t>(qr[d]) << 16);
+    __syncwarp();
+    const int see = sp.len - sp.n_q + r;                  // causal rows: keys up to the row's position
+    float m = -INFINITY, sum = 0.f;
+    for (int key = sp.t0 + lane; key < sp.t0 + sp.len; key += 32) {
+      if (CAUSAL ? key - sp.t0 > see : !is_mm(modality[key])) continue;
+      const uint16_t *kr = reinterpret_cast<const uint16_t *>(k + key * k_stride) + g * 128;
+      float dot = 0.f;
+#pragma unroll 16
+      for (int d = 0; d < 128; ++d) dot = fmaf(qv[d], __uint_as_float(static_cast<uint32_t>(kr[d]) << 16), dot);
+      const float y = dot * plan.scale2;
+      if (y > m) {
+        sum = (m == -INFINITY ? 0.f : sum * exp2f(m - y)) + 1.f;
+        m = y;
+      } else {
+        sum += exp2f(y - m);
+      }
+    }
+    float mm = m;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, o));
+    float tot = (m != -INFINITY) ? sum * exp2f(m - mm) : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+    out = mm == -INFINITY ? INFINITY : -(mm + log2f(tot));
+  }
+  if (lane == 0) nlse2[prow] = out;
 }
 
 // ------------------------------------------------------------------ pass 2
@@ -1080,8 +1123,15 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
     if (qrows > 0) {
-      lse_merge_kernel<<<static_cast<unsigned>((qrows + 255) / 256), 256, 0, stream>>>(P, part, nlse2, qp_base,
-                                                                                       qrows);
+      const unsigned blocks = static_cast<unsigned>((qrows * 32 + 255) / 256);   // one warp per packed row
+      const uint16_t *qp16 = reinterpret_cast<const uint16_t *>(qp);
+      const uint8_t *k8 = static_cast<const uint8_t *>(k);
+      if (P.causal)
+        lse_merge_kernel<true><<<blocks, 256, 0, stream>>>(P, part, qp16, k8, k_token_stride, seqs->modality, nlse2,
+                                                           qp_base, qrows);
+      else
+        lse_merge_kernel<false><<<blocks, 256, 0, stream>>>(P, part, qp16, k8, k_token_stride, seqs->modality, nlse2,
+                                                            qp_base, qrows);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }

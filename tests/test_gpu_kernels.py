@@ -187,6 +187,28 @@ def test_scores_large_logits_and_sequence_without_S(ap):
     assert np.all(got[900:] == 0)
 
 
+@pytest.mark.parametrize("domain", [0, 1])
+def test_scores_with_a_logit_far_above_its_run_reference(ap, domain):
+    """A late key aligned with one query row gives that row a logit about 190 binary orders of
+    magnitude above the maximum of the first key block: the row's online sum would overflow
+    its run's fixed reference, so the pass-1 partial is marked and the merge recomputes the
+    row's normaliser exactly.  Scores must still match the oracle on every token of S."""
+    rng = np.random.default_rng(99 + domain)
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, [2000], [5], 28, 4, scale_k=0.05)
+    h, r = 9, 2                                    # query head 9 (KV head 1), query row 2
+    qv = oracle.bf16_to_f64(q[r, h])
+    kv = bf16(12.0 * qv)
+    for key in (1500, 1777):
+        mod[key] = 2
+        k[key, h // 7] = kv
+    na = [int((mod == 1).sum())]
+    nv = [int((mod == 2).sum())]
+    got = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, 28, 4, softmax_domain=domain)
+    ref = oracle.relevance_scores(q, k, cu, cuq, mod, 28, 4, softmax_domain=domain)
+    check_scores(got, ref)
+    assert ref[1500] > 1e-3 and ref[1777] > 1e-3
+
+
 def test_scores_identical_keys_are_uniform(ap):
     mod = np.array([0] * 16 + [1, 2, 2, 2] * 300 + [0] * 8, np.uint8)
     T = mod.size
