@@ -59,9 +59,10 @@ enum { APACK_SELECT_PER_MODALITY = 0, APACK_SELECT_JOINT = 1 };
    multimodal tokens S of the sequence only.
    CAUSAL_ROW: the denominator is the decoder's own attention row, every token
    the query row attends to causally (system, text, audio, visual and the
-   query tokens up to and including its own position); the query rows are the
-   last n_q tokens of the sequence, row r at position len - n_q + r, and a token
-   of S that a row cannot see contributes 0 for that row. */
+   query tokens up to and including its own position); query row r sits at
+   position q_start + r of its sequence (apack_seqs.q_start_h; by default the
+   query rows are the last n_q tokens, q_start = len - n_q), and a token of S
+   that a row cannot see contributes 0 for that row. */
 enum { APACK_SOFTMAX_MM = 0, APACK_SOFTMAX_CAUSAL_ROW = 1 };
 
 /* Maximum sizes of this build. */
@@ -83,6 +84,11 @@ typedef struct apack_seqs {
   int32_t head_dim;             /* D; must be APACK_HEAD_DIM */
   int32_t softmax_domain;       /* APACK_SOFTMAX_MM (0, zero-initialised default) or
                                    APACK_SOFTMAX_CAUSAL_ROW (needs n_q <= len per sequence) */
+  const int32_t *q_start_h;     /* [B] or NULL: position of each sequence's first query row
+                                   within the sequence (the query span of Sec. 3.2's problem
+                                   statement), 0 <= q_start, q_start + n_q <= len; NULL means
+                                   the span ends the sequence.  Read in the CAUSAL_ROW domain
+                                   only (in the MM domain no query token is in S). */
 } apack_seqs;
 
 /* One group of per-token planes to compact (e.g. the K cache of layers l..L-1).
@@ -122,8 +128,9 @@ apack_status apack_keep_counts(const apack_seqs *seqs, const float *keep_ratio_h
                                       / sum_{j in S} exp(q_{r,h}.k_{j,g(h)} / sqrt(D))
    for i in S of the sequence, and I_i = 0 for tokens outside S.  With
    seqs->softmax_domain = APACK_SOFTMAX_CAUSAL_ROW the sum in the denominator
-   runs over every token j <= p_r (p_r = len - n_q + r, the row's position)
-   and row r adds to I_i only when i <= p_r.
+   runs over every token j <= p_r (p_r = q_start + r, the row's position within
+   its sequence; q_start = len - n_q without seqs->q_start_h) and row r adds to
+   I_i only when i <= p_r.
    q: bf16 [sum n_q][Hq][D], contiguous (the query rows at the pruning layer).
    k: bf16 keys of the pruning layer, token t at k + t*k_token_stride, laid
       out [Hkv][D] within the row; k_token_stride a multiple of 16 bytes.
@@ -136,16 +143,19 @@ apack_status apack_score(const apack_seqs *seqs, const void *q, const void *k, i
 /* Top-k selection of Eq. inner per segment (see APACK_SELECT_*): keeps the
    keep_count_h[b][m] highest scores of each segment, equal scores going to the
    lower token index, plus every token outside S.
+   keep_count_h: host [B][2] counts (JOINT: [b][0] over |S|), or NULL: the
+   counts come from keep_ratio_h (host [B][2], the keep ratios 1-P of Eq. inner)
+   by the rule of apack_keep_counts.
    Outputs: keep_idx [T_out] (kept token indices in ascending order, i.e. the
    original order; T_out = new_cu_seqlens_h[B] of apack_keep_counts),
    modality_out [T_out] (nullable; the compacted modality mask),
    dst_of_src [T] (nullable; output row of each token or -1),
    new_cu_seqlens [B+1] (nullable; device copy of the new offsets).
    scores must be finite and >= 0 (as apack_score produces). */
-apack_status apack_select(const apack_seqs *seqs, const float *scores, const int32_t *keep_count_h,
-                          int32_t select_mode, int32_t *keep_idx, uint8_t *modality_out,
-                          int32_t *dst_of_src, int32_t *new_cu_seqlens, void *ws, size_t ws_bytes,
-                          void *stream);
+apack_status apack_select(const apack_seqs *seqs, const float *scores, const float *keep_ratio_h,
+                          const int32_t *keep_count_h, int32_t select_mode, int32_t *keep_idx,
+                          uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu_seqlens, void *ws,
+                          size_t ws_bytes, void *stream);
 
 /* KV-cache and hidden-state slicing (Sec. 3.2, last sentence; Algorithm 1,
    "slice their KV-cache entries"): for every plane of every group,

@@ -31,8 +31,8 @@ A second softmax domain reads "the full key row" as the decoder's own
 attention row: the denominator of Eq. (inner_score) then runs over the
 causal attention row of the query token, i.e. every token at or before the
 query row's position (system, text, audio, visual and query tokens), with the
-query rows taken as the last n_q tokens of the sequence; a token of S after a
-row's position gets nothing from that row.
+query rows at a given position of the sequence (by default its last n_q
+tokens); a token of S after a row's position gets nothing from that row.
 
 The arithmetic is fp64 from exactly widened bf16 inputs; numpy's matmul,
 exp and stable argsort are the only library steps.
@@ -53,7 +53,7 @@ def bf16_to_f64(bits):
 
 
 def relevance_scores(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads,
-                     row_chunk=512, softmax_domain=SOFTMAX_MM):
+                     row_chunk=512, softmax_domain=SOFTMAX_MM, q_start=None):
     """Eq. (inner_score), averaged over query heads and query rows.
 
     q_bits: uint16 [sum n_q, Hq, D] (bf16) query rows, packed per sequence by cu_qlens.
@@ -61,10 +61,13 @@ def relevance_scores(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads
     modality: uint8 [T]; 1 = audio, 2 = visual form S, anything else is outside S.
     softmax_domain: SOFTMAX_MM (the denominator over S, as Eq. inner_score prints it) or
     SOFTMAX_CAUSAL_ROW (over the causal attention row; see the module docstring).
+    q_start: per sequence, the position of its first query row (causal domain only);
+    None puts the query rows at the end of each sequence.
     Returns float64 [T]; 0 outside S.
     """
     if softmax_domain == SOFTMAX_CAUSAL_ROW:
-        return _relevance_causal(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads)
+        return _relevance_causal(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads,
+                                 q_start)
     q_bits = np.asarray(q_bits)
     k_bits = np.asarray(k_bits)
     T = k_bits.shape[0]
@@ -94,11 +97,12 @@ def relevance_scores(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads
     return scores
 
 
-def _relevance_causal(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads):
+def _relevance_causal(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_heads, num_kv_heads, q_start=None):
     """Eq. (inner_score) with the causal-row denominator: query row r of a
-    sequence of length L with n_q query rows is token p_r = L - n_q + r; its
-    softmax runs over the tokens 0..p_r of the sequence, and the score of a token
-    i of S averages that row's probability of i (0 when i > p_r) over heads and rows."""
+    sequence of length L with n_q query rows is token p_r = q_start + r (q_start =
+    L - n_q when not given); its softmax runs over the tokens 0..p_r of the
+    sequence, and the score of a token i of S averages that row's probability of
+    i (0 when i > p_r) over heads and rows."""
     q_bits = np.asarray(q_bits)
     k_bits = np.asarray(k_bits)
     T = k_bits.shape[0]
@@ -116,7 +120,7 @@ def _relevance_causal(q_bits, k_bits, cu_seqlens, cu_qlens, modality, num_q_head
         for h in range(num_q_heads):
             keys = bf16_to_f64(k_bits[t0:t1, h // group, :])     # [L, D], every token
             for r in range(n_q):
-                p = L - n_q + r                                   # position of query row r
+                p = (L - n_q if q_start is None else int(q_start[s])) + r   # position of query row r
                 qv = bf16_to_f64(q_bits[r0 + r, h, :])
                 x = (keys[:p + 1] @ qv) / math.sqrt(D)            # the row's visible logits
                 e = np.exp(x - x.max())

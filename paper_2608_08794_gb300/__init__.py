@@ -49,7 +49,8 @@ class apack_seqs(ctypes.Structure):
                 ("num_q_heads", ctypes.c_int32),
                 ("num_kv_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32),
-                ("softmax_domain", ctypes.c_int32)]
+                ("softmax_domain", ctypes.c_int32),
+                ("q_start_h", ctypes.POINTER(ctypes.c_int32))]
 
 
 class apack_plane(ctypes.Structure):
@@ -77,7 +78,7 @@ def _load():
     lib.apack_workspace_size.argtypes = [P(apack_seqs), P(SZ)]
     lib.apack_keep_counts.argtypes = [P(apack_seqs), P(ctypes.c_float), I32, PI32, PI32]
     lib.apack_score.argtypes = [P(apack_seqs), VP, VP, I64, VP, VP, SZ, VP]
-    lib.apack_select.argtypes = [P(apack_seqs), VP, PI32, I32, VP, VP, VP, VP, VP, SZ, VP]
+    lib.apack_select.argtypes = [P(apack_seqs), VP, P(ctypes.c_float), PI32, I32, VP, VP, VP, VP, VP, SZ, VP]
     lib.apack_compact.argtypes = [VP, I64, P(apack_plane), I32, VP, VP]
     lib.apack_prune_step.argtypes = [P(apack_seqs), I32, I32, VP, VP, VP, I64, VP, I64, P(ctypes.c_float), PI32,
                                      I32, VP, VP, I64, VP, P(apack_plane), I32, VP, VP, PI32, VP, VP, VP, SZ,
@@ -141,11 +142,12 @@ class Seqs:
     Keeps the host arrays alive for as long as the ``apack_seqs`` struct is used."""
 
     def __init__(self, cu_seqlens, cu_qlens, n_audio, n_visual, modality, num_q_heads, num_kv_heads,
-                 head_dim=APACK_HEAD_DIM, softmax_domain=0):
+                 head_dim=APACK_HEAD_DIM, softmax_domain=0, q_start=None):
         self.cu_seqlens = _i32(cu_seqlens)
         self.cu_qlens = _i32(cu_qlens)
         self.n_audio = _i32(n_audio)
         self.n_visual = _i32(n_visual)
+        self.q_start = None if q_start is None else _i32(q_start)
         self.modality = modality
         I32P = ctypes.POINTER(ctypes.c_int32)
         self.struct = apack_seqs(
@@ -156,7 +158,8 @@ class Seqs:
             n_visual_h=self.n_visual.ctypes.data_as(I32P),
             modality=None if modality is None else modality.data_ptr(),
             num_q_heads=num_q_heads, num_kv_heads=num_kv_heads, head_dim=head_dim,
-            softmax_domain=int(softmax_domain))
+            softmax_domain=int(softmax_domain),
+            q_start_h=None if self.q_start is None else self.q_start.ctypes.data_as(I32P))
         self.softmax_domain = int(softmax_domain)
 
     @property
@@ -194,9 +197,13 @@ def apack_score(seqs, q, k, k_token_stride, scores, ws, stream=None):
 
 
 def apack_select(seqs, scores, keep_count, keep_idx, ws, select_mode=APACK_SELECT_PER_MODALITY,
-                 modality_out=None, dst_of_src=None, new_cu_seqlens=None, stream=None):
-    kc = _i32(keep_count).reshape(-1)
-    _check(_lib.apack_select(seqs.ref(), _ptr(scores), kc.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
+                 modality_out=None, dst_of_src=None, new_cu_seqlens=None, stream=None, keep_ratio=None):
+    """keep_count: [B, 2] counts, or None with keep_ratio [B, 2] (ratios 1-P of Eq. inner)."""
+    kc = None if keep_count is None else _i32(keep_count).reshape(-1)
+    kr = None if keep_ratio is None else np.ascontiguousarray(np.asarray(keep_ratio, np.float32).reshape(-1))
+    _check(_lib.apack_select(seqs.ref(), _ptr(scores),
+                             None if kr is None else kr.ctypes.data_as(ctypes.POINTER(ctypes.c_float)),
+                             None if kc is None else kc.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
                              select_mode, _ptr(keep_idx), _ptr(modality_out), _ptr(dst_of_src),
                              _ptr(new_cu_seqlens), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)),
            "apack_select")

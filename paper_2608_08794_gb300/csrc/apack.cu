@@ -53,6 +53,9 @@ apack_status validate_seqs(const apack_seqs *s, int64_t *total_tokens, int64_t *
     const int64_t nq = static_cast<int64_t>(s->cu_qlens_h[b + 1]) - s->cu_qlens_h[b];
     if (len < 0 || nq < 0) return APACK_EINVAL;
     if (s->softmax_domain == APACK_SOFTMAX_CAUSAL_ROW && nq > len) return APACK_EINVAL;   // rows are tokens
+    if (s->softmax_domain == APACK_SOFTMAX_CAUSAL_ROW && s->q_start_h &&
+        (s->q_start_h[b] < 0 || static_cast<int64_t>(s->q_start_h[b]) + nq > len))
+      return APACK_EINVAL;
     if (s->n_audio_h[b] < 0 || s->n_visual_h[b] < 0 ||
         static_cast<int64_t>(s->n_audio_h[b]) + s->n_visual_h[b] > len)
       return APACK_EINVAL;
@@ -62,6 +65,12 @@ apack_status validate_seqs(const apack_seqs *s, int64_t *total_tokens, int64_t *
   *total_tokens = T;
   *total_qrows = s->cu_qlens_h[s->num_seqs];
   return APACK_OK;
+}
+
+int32_t query_position(const apack_seqs *s, int b) {
+  const int32_t len = s->cu_seqlens_h[b + 1] - s->cu_seqlens_h[b];
+  const int32_t nq = s->cu_qlens_h[b + 1] - s->cu_qlens_h[b];
+  return s->q_start_h ? s->q_start_h[b] : len - nq;
 }
 
 WsLayout workspace_layout(const apack_seqs *s) {
@@ -198,14 +207,19 @@ apack_status apack_score(const apack_seqs *seqs, const void *q, const void *k, i
   return run_score(seqs, q, k, k_token_stride, scores, ws, static_cast<cudaStream_t>(stream));
 }
 
-apack_status apack_select(const apack_seqs *seqs, const float *scores, const int32_t *keep_count_h,
-                          int32_t select_mode, int32_t *keep_idx, uint8_t *modality_out, int32_t *dst_of_src,
-                          int32_t *new_cu_seqlens, void *ws, size_t ws_bytes, void *stream) {
+apack_status apack_select(const apack_seqs *seqs, const float *scores, const float *keep_ratio_h,
+                          const int32_t *keep_count_h, int32_t select_mode, int32_t *keep_idx,
+                          uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu_seqlens, void *ws,
+                          size_t ws_bytes, void *stream) {
   int64_t T = 0, NQ = 0;
-  const apack_status st = validate_seqs(seqs, &T, &NQ);
+  apack_status st = validate_seqs(seqs, &T, &NQ);
   if (st != APACK_OK) return st;
   if (!ws_ok(seqs, ws, ws_bytes)) return ws ? APACK_EWORKSPACE : APACK_EINVAL;
-  return run_select(seqs, scores, keep_count_h, select_mode, keep_idx, modality_out, dst_of_src, new_cu_seqlens, ws,
+  // counts from the ratios when none are given (the rule of apack_keep_counts), checked either way
+  std::vector<int32_t> counts(2 * static_cast<size_t>(seqs->num_seqs));
+  st = counts_and_offsets(seqs, keep_ratio_h, keep_count_h, select_mode, counts.data(), nullptr);
+  if (st != APACK_OK) return st;
+  return run_select(seqs, scores, counts.data(), select_mode, keep_idx, modality_out, dst_of_src, new_cu_seqlens, ws,
                     static_cast<cudaStream_t>(stream));
 }
 

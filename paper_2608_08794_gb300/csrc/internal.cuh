@@ -105,6 +105,9 @@ cudaError_t once_per_device(std::atomic<uint64_t> &done, F &&set) {
 bool in_host_memory(const void *p);   // pinned or registered host memory (cudaMemoryTypeHost)
 
 apack_status validate_seqs(const apack_seqs *seqs, int64_t *total_tokens, int64_t *total_qrows);
+// Position of sequence b's first query row within the sequence (the causal-row domain's
+// rows are tokens q .. q + n_q - 1): q_start_h[b], or len - n_q without q_start_h.
+int32_t query_position(const apack_seqs *seqs, int b);
 
 apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int64_t k_token_stride,
                        float *scores, void *ws, cudaStream_t stream);

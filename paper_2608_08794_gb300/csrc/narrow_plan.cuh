@@ -14,6 +14,7 @@ struct NSeq {
   int32_t unit8_begin;                 // first chunk (CTA) of this sequence in the rows8 logits kernel
   int32_t nparts;                      // CTA partials of the logits kernel in use
   int32_t rows;                        // logit rows R = Hq * n_q
+  int32_t q_pos;                       // causal rows: position of query row 0 within the sequence
   int64_t lstride;                     // logit row stride: len rounded up to kLogitPad
   int64_t logit_base;                  // float offset of this sequence's logits [R][lstride]
   int64_t part_base;                   // float2 offset of its CTA partials [nparts][R]
@@ -26,7 +27,7 @@ struct NarrowPlan {
   int32_t total_units8;
   int32_t chunk;                       // keys per CTA of the rows8 kernel (a multiple of the kernel's tile)
   int32_t hq, hkv, group;
-  int32_t causal;                      // APACK_SOFTMAX_CAUSAL_ROW: row r of n_q sees keys <= len - n_q + r
+  int32_t causal;                      // APACK_SOFTMAX_CAUSAL_ROW: row r of n_q sees keys <= q_pos + r
   float scale2;
   NSeq seq[kSeqsPerLaunch];
 };

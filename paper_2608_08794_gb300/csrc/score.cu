@@ -73,6 +73,7 @@ struct SeqPlan {
   int32_t qp_base;        // first packed row of head group 0; group g starts at qp_base + g * rows_pad
   int32_t rows_pad;       // G * n_q rounded up to a multiple of 256
   int32_t nb;             // key blocks (256 keys) of the sequence
+  int32_t q_pos;          // causal rows: position of query row 0 within the sequence
   int32_t unit_begin;     // pass 2: first work unit of this sequence in the launch
   int32_t flat0;          // pass 1: first flat (row group, key block) index of the sequence
 };
@@ -535,8 +536,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       x = w.x1;
       float m = -INFINITY, sum = 0.f;
       bool bad = false;
-      // causal rows: this lane's row (token r of the query span) sees keys up to len - n_q + r
-      const int see = sp.len - sp.n_q + (w.qp * kChunk + row) / G;
+      // causal rows: this lane's row (token r of the query span) sees keys up to q_pos + r
+      const int see = sp.q_pos + (w.qp * kChunk + row) / G;
       for (int b = w.b0; b < w.b1; ++b) {
         // the keys of this thread's two 32-key chunks that count; and those this lane's row sees
         if (!wait_or_abort(&bars->m_full[mi], mph, bars, pc, err, 20)) { ok = false; break; }
@@ -692,7 +693,7 @@ __global__ void lse_merge_kernel(const __grid_constant__ ScorePlan plan, const f
     const uint16_t *qr = qp + prow * 128;
     for (int d = lane; d < 128; d += 32) qv[d] = __uint_as_float(static_cast<uint32_t>(qr[d]) << 16);
     __syncwarp();
-    const int see = sp.len - sp.n_q + r;                  // causal rows: keys up to the row's position
+    const int see = sp.q_pos + r;                         // causal rows: keys up to the row's position
     float m = -INFINITY, sum = 0.f;
     for (int key = sp.t0 + lane; key < sp.t0 + sp.len; key += 32) {
       if (CAUSAL ? key - sp.t0 > see : !is_mm(modality[key])) continue;
@@ -877,8 +878,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int nch = sp.rows_pad / kChunk;
       if (nch == 0) continue;
       float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-      // causal rows: only packed rows rho >= rho_min (tokens r >= key - (len - n_q)) see this key
-      const int rho_min = CAUSAL ? max(0, w.kp * kBlock + klane - (sp.len - sp.n_q)) * G : 0;
+      // causal rows: only packed rows rho >= rho_min (tokens r >= key - q_pos) see this key
+      const int rho_min = CAUSAL ? max(0, w.kp * kBlock + klane - sp.q_pos) * G : 0;
       for (int c = 0; c < nch; ++c) {
         if (!wait_or_abort(&bars->l_full[li], lph, bars, pc, err, 30)) { ok = false; break; }
         if (!wait_or_abort(&bars->acc_full[ci], cph, bars, pc, err, 26)) { ok = false; break; }
@@ -1087,6 +1088,7 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
       sp.qp_base = static_cast<int32_t>(qp_base + qrows);
       qrows += static_cast<int64_t>(hkv) * sp.rows_pad;
       sp.nb = sp.n_q > 0 ? (sp.len + kBlock - 1) / kBlock : 0;
+      sp.q_pos = query_position(seqs, b);
       sp.flat0 = static_cast<int32_t>(flat);
       flat += pass1_items(sp, hkv);
       if (sp.nb > nb_max) nb_max = sp.nb;

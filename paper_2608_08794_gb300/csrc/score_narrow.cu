@@ -117,7 +117,7 @@ __global__ void __launch_bounds__(kThreads)
         if (in) logits[lbase + static_cast<int64_t>(rho) * sq.lstride] = y;
         // this warp's (max, sum of exp2) of the row over the keys in its denominator: the
         // multimodal keys, or (causal rows) every key up to the row's own position
-        const bool use = plan.causal ? (in && key - sq.t0 <= sq.len - sq.n_q + l / G) : mm;
+        const bool use = plan.causal ? (in && key - sq.t0 <= sq.q_pos + l / G) : mm;
         const float wm = warp_max(use ? y : -INFINITY);
         const float ws = warp_sum(use && wm != -INFINITY ? ex2_approx(y - wm) : 0.f);
         if (lane == 0) wpart[warp * R + rho] = make_float2(wm, ws);
@@ -205,8 +205,8 @@ __global__ void __launch_bounds__(kThreads)
     // eight independent sums, the loads of a block of 8 rows issued together
     const float *lp = logits + sq.logit_base + (key - sq.t0);
     float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    // causal rows: logit row rho = token * Hq + head sees this key when token >= key - (len - n_q)
-    const int rho_min = plan.causal ? max(0, key - sq.t0 - (sq.len - sq.n_q)) * plan.hq : 0;
+    // causal rows: logit row rho = token * Hq + head sees this key when token >= key - q_pos
+    const int rho_min = plan.causal ? max(0, key - sq.t0 - sq.q_pos) * plan.hq : 0;
     if (R <= 32) {
       // all rows' logits requested at once: one round trip (the paper's one query token: R = Hq)
       float x[32];
@@ -313,6 +313,7 @@ apack_status run_score_narrow(const apack_seqs *seqs, const void *q, const void 
       sq.q_off = seqs->cu_qlens_h[b];
       sq.n_q = seqs->cu_qlens_h[b + 1] - sq.q_off;
       sq.rows = hq * sq.n_q;
+      sq.q_pos = query_position(seqs, b);
       sq.unit_begin = units;
       sq.unit8_begin = units8;
       sq.lstride = (sq.len + kLogitPad - 1) / kLogitPad * kLogitPad;

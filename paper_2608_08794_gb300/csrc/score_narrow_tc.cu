@@ -229,7 +229,7 @@ __global__ void __launch_bounds__(tc_threads<HKV>(), 1)
           const int rho = (j / G) * plan.hq + h * G + j % G;
           if (valid) logits[sq.logit_base + static_cast<int64_t>(rho) * sq.lstride + key] = y;
           // the row's denominator: multimodal keys, or (causal rows) every key up to its position
-          if (plan.causal ? (valid && key <= sq.len - sq.n_q + j / G) : mm) {
+          if (plan.causal ? (valid && key <= sq.q_pos + j / G) : mm) {
             const float mn = fmaxf(m[hh][j], y);
             sum[hh][j] = sum[hh][j] * ex2_approx(m[hh][j] - mn) + ex2_approx(y - mn);
             m[hh][j] = mn;

@@ -61,9 +61,9 @@ def random_batch(rng, lens, nqs, hq, hkv, p_other=0.05, scale_k=1.0, scale_q=1.0
     return mod, cu, cuq, k, q, na, nv
 
 
-def gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv, softmax_domain=0):
+def gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv, softmax_domain=0, q_start=None):
     mod_d = dev(mod)
-    seqs = ap.Seqs(cu, cuq, na, nv, mod_d, hq, hkv, softmax_domain=softmax_domain)
+    seqs = ap.Seqs(cu, cuq, na, nv, mod_d, hq, hkv, softmax_domain=softmax_domain, q_start=q_start)
     ws = aligned_ws(ap, seqs)
     T = int(cu[-1])
     scores = torch.full((max(T, 1),), float("nan"), dtype=torch.float32, device="cuda")
@@ -166,6 +166,56 @@ def test_causal_row_scores_match_oracle(ap, lens, nqs, hq, hkv, query_text):
     for s in range(len(lens)):      # the causal row spends mass outside S: never more than the S domain's 1
         if nqs[s]:
             assert got[cu[s]:cu[s + 1]].astype(np.float64).sum() <= mm[cu[s]:cu[s + 1]].astype(np.float64).sum() + 1e-4
+
+
+@pytest.mark.parametrize("lens,nqs,hq,hkv", [CAUSAL_SHAPES[i] for i in (0, 1, 4, 6, 7, 10)])
+def test_causal_row_scores_with_the_query_span_inside_the_sequence(ap, lens, nqs, hq, hkv):
+    """apack_seqs.q_start_h places each sequence's query rows at a chosen position (text query
+    followed by more tokens): row r sees the tokens up to q_start + r, later tokens get nothing
+    from any row.  Both scoring paths (tensor-core passes and the few-row path)."""
+    rng = np.random.default_rng(sum(lens) * 7 + hq)
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, lens, nqs, hq, hkv, scale_k=1.3)
+    q_start = np.array([int(rng.integers(0, L - n + 1)) for L, n in zip(lens, nqs)], np.int32)
+    got = gpu_scores(ap, mod, cu, cuq, k, q, na, nv, hq, hkv, softmax_domain=ap.APACK_SOFTMAX_CAUSAL_ROW,
+                     q_start=q_start)
+    ref = oracle.relevance_scores(q, k, cu, cuq, mod, hq, hkv, softmax_domain=oracle.SOFTMAX_CAUSAL_ROW,
+                                  q_start=q_start)
+    check_scores(got, ref)
+    for s in range(len(lens)):
+        if nqs[s]:
+            assert not got[cu[s] + q_start[s] + nqs[s]:cu[s + 1]].any()
+    # a span that does not fit its sequence is refused before any device work
+    bad = q_start.copy()
+    bad[-1] = lens[-1] - nqs[-1] + 1
+    seqs = ap.Seqs(cu, cuq, na, nv, dev(mod), hq, hkv, softmax_domain=ap.APACK_SOFTMAX_CAUSAL_ROW, q_start=bad)
+    with pytest.raises(ap.ApackError) as e:
+        ap.apack_workspace_size(seqs)
+    assert e.value.status == ap.APACK_EINVAL
+
+
+def test_select_from_keep_ratios_equals_select_from_counts(ap):
+    """apack_select takes the keep ratios of Eq. inner directly (keep_count_h NULL): the same
+    kept indices as with the counts apack_keep_counts derives from those ratios."""
+    rng = np.random.default_rng(123)
+    lens = [3000, 700, 5000]
+    mod, cu, cuq, k, q, na, nv = random_batch(rng, lens, [3, 2, 5], 28, 4)
+    scores = rng.random(int(cu[-1])).astype(np.float32)
+    scores[(mod != 1) & (mod != 2)] = 0
+    mod_d = dev(mod)
+    seqs = ap.Seqs(cu, cuq, na, nv, mod_d, 28, 4)
+    ratios = np.array([[0.5, 0.25], [0.7, 0.4], [0.33, 0.123]], np.float32)
+    counts, new_cu = ap.apack_keep_counts(seqs, ratios)
+    ws = aligned_ws(ap, seqs)
+    out = []
+    for kc, kr in ((counts, None), (None, ratios)):
+        keep = torch.full((int(new_cu[-1]),), -1, dtype=torch.int32, device="cuda")
+        ap.apack_select(seqs, dev(scores), kc, keep, ws, keep_ratio=kr)
+        torch.cuda.synchronize()
+        out.append(keep.cpu().numpy())
+    np.testing.assert_array_equal(out[0], out[1])
+    np.testing.assert_array_equal(out[0], oracle.select_keep(scores, mod, cu, [tuple(c) for c in counts]))
+    with pytest.raises(ap.ApackError):
+        ap.apack_select(seqs, dev(scores), None, keep, ws, keep_ratio=np.full((3, 2), 1.5, np.float32))
 
 
 def test_causal_row_domain_rejects_more_rows_than_tokens(ap):

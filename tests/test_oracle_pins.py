@@ -321,10 +321,11 @@ def test_compaction_row_by_row_and_progressive_composition():
 
 # ---------------------------------------------------------------- causal-row softmax domain
 
-def brute_scores_causal(q_bits, k_bits, cu, cuq, mod, Hq, Hkv):
+def brute_scores_causal(q_bits, k_bits, cu, cuq, mod, Hq, Hkv, q_start=None):
     """Arbitrary-precision reference of the causal-row domain: query row r of a
-    sequence of length L is token L - n_q + r; its softmax runs over tokens
-    0..L - n_q + r of the sequence (every modality), explicit loops at 40 digits."""
+    sequence of length L is token p = q_start + r (q_start = L - n_q when not
+    given); its softmax runs over tokens 0..p of the sequence (every modality),
+    explicit loops at 40 digits."""
     mpmath.mp.dps = 40
     q = oracle.bf16_to_f64(q_bits)
     k = oracle.bf16_to_f64(k_bits)
@@ -338,7 +339,7 @@ def brute_scores_causal(q_bits, k_bits, cu, cuq, mod, Hq, Hkv):
             continue
         for h in range(Hq):
             for r in range(nq):
-                pos = t1 - t0 - nq + r
+                pos = (t1 - t0 - nq if q_start is None else int(q_start[s])) + r
                 vis = range(t0, t0 + pos + 1)
                 logits = {i: mpmath.fsum(mpmath.mpf(float(a)) * mpmath.mpf(float(b))
                                          for a, b in zip(q[cuq[s] + r, h], k[i, h // g])) / mpmath.sqrt(D)
@@ -367,6 +368,32 @@ def test_causal_scores_match_arbitrary_precision_brute_force(Hq, Hkv, nq):
     ref = brute_scores_causal(q, k, cu, cuq, modality, Hq, Hkv)
     np.testing.assert_allclose(got, ref, rtol=1e-12, atol=1e-15)
     assert np.all(got[modality == 0] == 0)
+
+
+@pytest.mark.parametrize("Hq,Hkv,nq", [(4, 2, 3), (6, 1, 4)])
+def test_causal_scores_with_the_query_span_inside_the_sequence(Hq, Hkv, nq):
+    # the query rows start at a given position (tokens after the span are seen by no row)
+    rng = np.random.default_rng(300 + Hq + nq)
+    mod = np.array([0, 0, 1, 2, 2, 1, 2, 2, 2, 1, 0, 2, 1, 1, 0, 0], np.uint8)
+    mod2 = np.array([0, 2, 2, 1, 2, 1, 0, 2, 0, 1], np.uint8)
+    modality = np.concatenate([mod, mod2])
+    cu = np.array([0, mod.size, modality.size], np.int32)
+    cuq = np.array([0, nq, 2 * nq], np.int32)
+    q_start = np.array([5, 2], np.int32)
+    k = rand_bf16(rng, (modality.size, Hkv, D))
+    q = rand_bf16(rng, (2 * nq, Hq, D), 0.3)
+    got = oracle.relevance_scores(q, k, cu, cuq, modality, Hq, Hkv, softmax_domain=oracle.SOFTMAX_CAUSAL_ROW,
+                                  q_start=q_start)
+    ref = brute_scores_causal(q, k, cu, cuq, modality, Hq, Hkv, q_start=q_start)
+    np.testing.assert_allclose(got, ref, rtol=1e-12, atol=1e-15)
+    # tokens after the last row's position get nothing
+    assert np.all(got[q_start[0] + nq:mod.size] == 0)
+    assert np.all(got[mod.size + q_start[1] + nq:] == 0)
+    # the default is the span at the end of each sequence
+    end = oracle.relevance_scores(q, k, cu, cuq, modality, Hq, Hkv, softmax_domain=oracle.SOFTMAX_CAUSAL_ROW,
+                                  q_start=np.diff(cu) - nq)
+    np.testing.assert_array_equal(end, oracle.relevance_scores(q, k, cu, cuq, modality, Hq, Hkv,
+                                                               softmax_domain=oracle.SOFTMAX_CAUSAL_ROW))
 
 
 def test_causal_identical_keys_closed_form():
