@@ -166,8 +166,8 @@ apack_status apack_select(const apack_seqs *seqs, const float *scores, const flo
    so each store waits (bounded) until every load that reads the rows it
    overwrites is done; the rows must be 16-byte multiples of at most 32 KB,
    16-byte aligned (APACK_EUNSUPPORTED otherwise), planes must not overlap,
-   and ws is required: the launch keeps per-CTA progress words in its bytes
-   256..1023 (the workspace of apack_workspace_size has them).
+   and ws is required: the launch keeps its progress words or wave counter
+   in bytes 256..1023 (the workspace of apack_workspace_size has them).
    Host source: a group whose src is pinned host memory (cudaHostAlloc or
    cudaHostRegister) is gathered over the host link by plain loads (zero
    copy): only the kept rows cross the link.  Its dst must be device memory,

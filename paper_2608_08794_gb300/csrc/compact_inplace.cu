@@ -2,13 +2,20 @@
 // "slice their KV-cache entries"): the first n_out rows of every plane become dst row j = src row
 // keep_idx[j].
 //
-// Output row j reads row keep_idx[j] >= j, so the store of output rows [r0, r0 + n) of a plane may
-// only start once every load of that plane that reads a row in [r0, r0 + n) is done.  Those loads
-// belong to output rows below r0 + n: earlier items of the same plane.  The kernel runs two CTAs
-// per SM (cooperative launch, so all are resident), items in (chunk, plane) order dealt
-// round-robin; each CTA publishes how many of its items' loads are complete and waits (bounded)
-// for the owners of those earlier items before each store.  Loads never wait on stores of later
-// items, so the waits always end.
+// Output row j reads row keep_idx[j] >= j.  Rows below A0, the first j with keep_idx[j] > j, stay
+// where they are.  Two schedules, both on a cooperative launch of two CTAs per SM:
+//  * Waves (when few are needed).  Wave k holds the output rows [A_k, B_k) with A_0 = A0,
+//    B_k = min(keep_idx[A_k], n_out) and A_(k+1) = B_k: its rows read sources >= B_k, above every
+//    row it writes, and no later wave reads a row below B_k.  So within a wave any order is safe,
+//    and a store of wave k only has to wait until every CTA has seen its loads of wave k - 1
+//    complete (one counter per launch).  Loads never wait.  The waves grow by about
+//    1 / (keep ratio) each, so a low keep ratio needs a handful of them.
+//  * Item dependencies (otherwise).  The store of output rows [r0, r0 + n) of a plane may only
+//    start once every load of that plane that reads a row in [r0, r0 + n) is done; those loads
+//    belong to earlier items of the same plane.  Items in (chunk, plane) order are dealt
+//    round-robin; each CTA publishes how many of its items' loads are complete and waits
+//    (bounded) for the owners of those earlier items before each store.
+// Loads never wait on stores of later work, so every wait ends.
 #include "compact_plan.cuh"
 
 namespace apack {
@@ -63,17 +70,10 @@ __device__ __forceinline__ uint32_t warp_count_below(const int32_t *__restrict__
   return lo + __reduce_add_sync(0xffffffffu, cnt);
 }
 
-__global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constant__ TmaPlan plan,
-                                                            const int32_t *__restrict__ keep_idx,
-                                                            uint16_t *progress, DeviceError *err) {
-  extern __shared__ __align__(1024) uint8_t slots[];
-  __shared__ __align__(8) uint64_t full[kInSlots];
+// The item-dependency schedule.
+__device__ void inplace_by_items(const TmaPlan &plan, const int32_t *__restrict__ keep_idx, uint16_t *progress,
+                                 DeviceError *err, uint8_t *slots, uint64_t *full, int lane) {
   __shared__ uint16_t seen[kMaxInCtas];          // last progress read of every CTA
-  const int lane = threadIdx.x;
-  if (lane == 0) {
-    for (int i = 0; i < kInSlots; ++i) mbar_init(&full[i], 1);
-    fence_mbar_init();
-  }
   for (int i = lane; i < kMaxInCtas; i += 32) seen[i] = 0;
   __syncwarp();
   const uint32_t me = blockIdx.x, P = gridDim.x;
@@ -198,6 +198,205 @@ __global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constan
     // loads issued but not observed may still be in flight: wait for them (bounded)
     for (uint32_t k = waited; k < issued; ++k) mbar_wait(&full[k % kInSlots], (k / kInSlots) & 1u, kWaitLimitNs / 4);
   }
+}
+
+// ---------------------------------------------------------------- waves
+// First output row whose source row is above it (n when none): keep_idx[j] > j holds from there
+// on, since keep_idx is strictly increasing.  Rounds of 32 evenly spaced probes.
+__device__ uint32_t warp_first_moved(const int32_t *__restrict__ a, uint32_t n, int lane) {
+  uint32_t lo = 0, hi = n;                         // the answer lies in [lo, hi]
+  while (hi - lo > 32) {
+    const uint32_t step = (hi - lo + 31) / 32;
+    const uint32_t p = lo + lane * step;
+    const uint32_t b = __ballot_sync(0xffffffffu, p < hi && a[p] > static_cast<int32_t>(p));
+    if (b) {
+      const int f = __ffs(b) - 1;
+      const uint32_t lo0 = lo;
+      hi = lo0 + f * step;
+      if (f > 0) lo = lo0 + (f - 1) * step + 1;
+    } else {
+      lo += ((hi - lo - 1) / step) * step + 1;       // past the last probe inside [lo, hi)
+    }
+  }
+  const uint32_t p = lo + lane;
+  const uint32_t b = __ballot_sync(0xffffffffu, p < hi && a[p] > static_cast<int32_t>(p));
+  return b ? lo + (__ffs(b) - 1) : hi;
+}
+
+// One wave: output rows [A, B), its items [base, base + n) of the concatenated item list.
+struct Wave {
+  uint32_t k, A, B, base, n;
+};
+
+__device__ __forceinline__ uint32_t wave_items(const TmaPlan &p, uint32_t A, uint32_t B) {
+  uint32_t n = 0;
+  for (int gi = 0; gi < p.ngroups; ++gi) n += p.g[gi].num_planes * ((B - A + p.g[gi].rows_per_slot - 1) / p.g[gi].rows_per_slot);
+  return n;
+}
+
+__device__ __forceinline__ void wave_open(const TmaPlan &p, const int32_t *__restrict__ keep_idx, Wave &w,
+                                          bool &bad) {
+  if (w.A >= p.n_out) {
+    w.B = w.A;
+    w.n = 0;
+    return;
+  }
+  const int64_t s = keep_idx[w.A];
+  if (s <= static_cast<int64_t>(w.A)) {            // not strictly increasing: stop, report
+    bad = true;
+    w.A = w.B = p.n_out;
+    w.n = 0;
+    return;
+  }
+  w.B = s < static_cast<int64_t>(p.n_out) ? static_cast<uint32_t>(s) : p.n_out;
+  w.n = wave_items(p, w.A, w.B);
+}
+
+// Moves w forward to the wave that holds item g (w.A == n_out past the last wave).
+__device__ __forceinline__ void wave_seek(const TmaPlan &p, const int32_t *__restrict__ keep_idx, uint32_t g,
+                                          Wave &w, bool &bad) {
+  while (w.A < p.n_out && g >= w.base + w.n) {
+    w.base += w.n;
+    w.A = w.B;
+    ++w.k;
+    wave_open(p, keep_idx, w, bad);
+  }
+}
+
+// Item g of wave w: (group, plane, chunk) order; chunks of rows_per_slot rows from A.
+__device__ __forceinline__ Item wave_item(const TmaPlan &p, const Wave &w, uint32_t g) {
+  uint32_t local = g - w.base;
+  int gi = 0;
+  uint32_t chunks = 0;
+  for (;; ++gi) {
+    chunks = (w.B - w.A + p.g[gi].rows_per_slot - 1) / p.g[gi].rows_per_slot;
+    const uint32_t items = p.g[gi].num_planes * chunks;
+    if (local < items || gi + 1 == p.ngroups) break;
+    local -= items;
+  }
+  const TmaGroup &G = p.g[gi];
+  Item it;
+  it.grp = &G;
+  it.plane = local / chunks;
+  const uint32_t chunk = local - it.plane * chunks;
+  it.r0 = w.A + chunk * G.rows_per_slot;
+  it.nrows = min(G.rows_per_slot, w.B - it.r0);
+  return it;
+}
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t *p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Barrier b of the launch is complete once every CTA has arrived at it: arrivals are made in
+// order, each after the previous barrier completed, so the counter then reads (b + 1) P.
+__device__ __forceinline__ bool wave_barrier_wait(const uint32_t *ctr, uint32_t b, uint32_t P) {
+  const uint32_t target = (b + 1) * P;
+  if (ld_acquire(ctr) >= target) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (ld_acquire(ctr) < target)
+    if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+  return true;
+}
+
+// The wave schedule; every lane runs it (lane 0 issues the counter operations).
+__device__ void inplace_by_waves(const TmaPlan &plan, const int32_t *__restrict__ keep_idx, uint32_t A0,
+                                 uint32_t *ctr, DeviceError *err, uint8_t *slots, uint64_t *full, int lane) {
+  const uint32_t me = blockIdx.x, P = gridDim.x;
+  bool bad = false;
+  Wave wl{0, A0, A0, 0, 0};                         // cursor of the loads
+  wave_open(plan, keep_idx, wl, bad);
+  Wave ws = wl;                                     // cursor of the stores
+  uint32_t arrived = 0;                             // barriers this CTA has arrived at
+  bool ok = true;
+  // arrive at every barrier below `upto` (each after the previous one completed)
+  auto arrive_below = [&](uint32_t upto) -> bool {
+    while (arrived < upto) {
+      bool fine = true;
+      if (lane == 0) {
+        fine = arrived == 0 || wave_barrier_wait(ctr, arrived - 1, P);
+        if (fine) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+      }
+      if (!__shfl_sync(0xffffffffu, fine, 0)) return false;
+      ++arrived;
+    }
+    return true;
+  };
+  uint32_t issued = 0;
+  for (; issued < kInSlots; ++issued) {
+    const uint32_t g = me + issued * P;
+    wave_seek(plan, keep_idx, g, wl, bad);
+    if (wl.A >= plan.n_out) break;
+    load_item(wave_item(plan, wl, g), slots + issued * kSlotBytes, &full[issued], keep_idx, lane);
+  }
+  uint32_t j = 0;
+  for (;; ++j) {
+    const uint32_t g = me + j * P;
+    wave_seek(plan, keep_idx, g, ws, bad);
+    if (ws.A >= plan.n_out) break;
+    const int slot = j % kInSlots;
+    if (!mbar_wait(&full[slot], (j / kInSlots) & 1u, kWaitLimitNs)) {
+      if (lane == 0 && err) raise_device_error(err, APACK_ETIMEOUT, 44);
+      ok = false;
+      break;
+    }
+    // every load of this CTA in the waves before this item's has been seen complete
+    if (!arrive_below(ws.k)) { ok = false; break; }
+    bool fine = true;
+    if (lane == 0 && ws.k > 0) fine = wave_barrier_wait(ctr, ws.k - 1, P);
+    if (!__shfl_sync(0xffffffffu, fine, 0)) {
+      ok = false;
+      break;
+    }
+    asm volatile("fence.proxy.async.global;" ::: "memory");   // the other CTAs' loads before the bulk store
+    fence_proxy_async_smem();
+    store_item(wave_item(plan, ws, g), slots + slot * kSlotBytes, lane);
+    // refill the slot whose store was issued one item ago, once that store has read it
+    if (j >= 1 && j - 1 + kInSlots == issued) {
+      const uint32_t k = issued;
+      const uint32_t gk = me + k * P;
+      wave_seek(plan, keep_idx, gk, wl, bad);
+      if (wl.A < plan.n_out) {
+        bulk_wait_read<1>();
+        load_item(wave_item(plan, wl, gk), slots + (k % kInSlots) * kSlotBytes, &full[k % kInSlots], keep_idx, lane);
+        issued = k + 1;
+      }
+    }
+  }
+  if (ok && !arrive_below(ws.k)) ok = false;        // the waves this CTA had no more items in
+  if (!ok) {
+    if (lane == 0 && err) raise_device_error(err, APACK_ETIMEOUT, 45);
+    for (uint32_t k = j; k < issued; ++k) mbar_wait(&full[k % kInSlots], (k / kInSlots) & 1u, kWaitLimitNs / 4);
+  }
+  if (bad && lane == 0 && err) raise_device_error(err, APACK_EDEVICE, 46);
+}
+
+constexpr float kMaxWaves = 16.f;
+
+__global__ void __launch_bounds__(32) gather_inplace_kernel(const __grid_constant__ TmaPlan plan,
+                                                            const int32_t *__restrict__ keep_idx,
+                                                            uint16_t *progress, DeviceError *err) {
+  extern __shared__ __align__(1024) uint8_t slots[];
+  __shared__ __align__(8) uint64_t full[kInSlots];
+  const int lane = threadIdx.x;
+  if (lane == 0) {
+    for (int i = 0; i < kInSlots; ++i) mbar_init(&full[i], 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  const uint32_t n = plan.n_out;
+  const uint32_t A0 = warp_first_moved(keep_idx, n, lane);   // the same in every CTA
+  if (A0 < n) {
+    // waves needed: they grow by about (last source row + 1) / n_out each, from A0
+    const float grow = (static_cast<float>(keep_idx[n - 1]) + 1.f) / static_cast<float>(n);
+    const float waves = 1.f + log2f(static_cast<float>(n) / static_cast<float>(A0 > 0 ? A0 : 1)) / log2f(grow);
+    if (grow > 1.f && waves <= kMaxWaves)
+      inplace_by_waves(plan, keep_idx, A0, reinterpret_cast<uint32_t *>(progress), err, slots, full, lane);
+    else
+      inplace_by_items(plan, keep_idx, progress, err, slots, full, lane);
+  }
   bulk_wait_all();
 }
 
@@ -235,7 +434,8 @@ apack_status launch_inplace(const TmaPlan &ip_in, uint32_t blocks, const int32_t
     return APACK_ECUDA;
   TmaPlan ip = ip_in;
   uint16_t *progress = reinterpret_cast<uint16_t *>(reinterpret_cast<uint8_t *>(err) + kProgressOff);
-  if (check_cuda(cudaMemsetAsync(progress, 0, blocks * sizeof(uint16_t), stream)) != APACK_OK) return APACK_ECUDA;
+  // the progress words (item schedule) or the barrier counter (wave schedule): bytes 256..1023
+  if (check_cuda(cudaMemsetAsync(progress, 0, 1024 - kProgressOff, stream)) != APACK_OK) return APACK_ECUDA;
   void *args[] = {&ip, const_cast<int32_t **>(&keep_idx), &progress, &err};
   if (check_cuda(cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(gather_inplace_kernel), dim3(blocks),
                                              dim3(32), args, kInSmem, stream)) != APACK_OK)

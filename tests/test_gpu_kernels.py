@@ -400,6 +400,8 @@ IN_PLACE_CASES = [
     (20000, 7000, 7168, 1, "random"),         # hidden-state rows, 4 per 32 KB slot
     (40000, 30000, 2048, 3, "tail"),          # a few early rows, then the whole tail: long dependency ranges
     (135272, 58772, 1024, 4, "random"),       # the 10-minute 7B step: thousands of items on every CTA
+    (10000, 5000, 1024, 2, "even"),           # every other row: waves of 1, 2, 4, ... rows
+    (60000, 51000, 1024, 2, "random"),        # keep ratio 0.85: the item-dependency schedule
 ]
 
 
@@ -413,6 +415,8 @@ def test_compact_in_place_is_bitexact(ap, T, n_keep, row_bytes, planes, pattern)
         keep = np.arange(T, dtype=np.int32)
     elif pattern == "last":
         keep = np.array([T - 1], np.int32)
+    elif pattern == "even":
+        keep = np.arange(0, 2 * n_keep, 2, dtype=np.int32)
     elif pattern == "tail":
         head = np.sort(rng.choice(T // 2, n_keep - (T - T // 2), replace=False))
         keep = np.concatenate([head, np.arange(T // 2, T)]).astype(np.int32)
