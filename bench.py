@@ -60,6 +60,8 @@ def parse():
     p.add_argument("--part", default="all", choices=["all", "decode", "compact"],
                    help="decode: time only the decode-step attention on a synthetic cache; compact: only "
                         "the first step's compaction of the 10-minute 7B cache, out of place and in place")
+    p.add_argument("--compact-planes", type=int, default=48,
+                   help="compact: planes of 135272 rows (48 = K and V of layers 4..27)")
     p.add_argument("--decode-tokens", type=int, default=135272)
     p.add_argument("--decode-layers", type=int, default=8)
     return p.parse_args()
@@ -923,12 +925,13 @@ def decode_only(args):
 
 def compact_only(args):
     """The first prune step's compaction of the 10-minute 7B sequence alone: K and V of layers
-    4..27 (48 planes of 135272 rows of 1024 B, 58772 kept), out of place (ping-pong buffers)
-    and in place (src == dst), through apack_compact.  Prints one JSON line."""
+    4..27 (48 planes of 135272 rows of 1024 B, 58772 kept; --compact-planes sets the plane count
+    for a smaller profiling case), out of place (ping-pong buffers) and in place (src == dst),
+    through apack_compact.  Prints one JSON line."""
     import numpy as np
     import torch
     import paper_2608_08794_gb300 as ap
-    T, n_keep, planes, rb = 135272, 58772, 48, 1024
+    T, n_keep, planes, rb = 135272, 58772, args.compact_planes, 1024
     rng = np.random.default_rng(4)
     keep = torch.from_numpy(np.sort(rng.choice(T, n_keep, replace=False)).astype(np.int32)).cuda()
     src = torch.empty((planes, T, rb), dtype=torch.uint8, device="cuda")
