@@ -94,6 +94,7 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     decode_chunk_kernel(const __grid_constant__ DecPlan plan, const uint16_t *__restrict__ q,
                         const uint8_t *__restrict__ k, const uint8_t *__restrict__ v, int64_t kv_stride,
                         float *__restrict__ opart, float2 *__restrict__ mlpart, DeviceError *err) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");   // the combine may be scheduled
   extern __shared__ __align__(1024) uint8_t dsmem[];
   uint8_t *stage_base = dsmem;                                               // [kDecStages][K | V]
   uint64_t *full = reinterpret_cast<uint64_t *>(dsmem + kDecStages * 2 * kStageBytes);
@@ -286,11 +287,13 @@ __global__ void __launch_bounds__(kDecCombineThreads)
                           const float2 *__restrict__ mlpart, float *__restrict__ out) {
   __shared__ __align__(16) float wo[kDecCombineWarps][128];
   __shared__ float2 wml[kDecCombineWarps];
+  pdl_wait_and_release();                   // the chunk kernel's partials are complete and visible
   const int s = blockIdx.x / plan.hq, hh = blockIdx.x % plan.hq;
   const DecSeq &sq = plan.seq[s];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   float m = -INFINITY, l = 0.f, o[4] = {0.f, 0.f, 0.f, 0.f};
-  constexpr int kBatch = 4;                 // chunk partials loaded before they are merged
+  constexpr int kBatch = 10;                // chunk partials loaded before they are merged (one
+                                            // round for up to 160 chunks)
   for (int c0 = warp; c0 < sq.nchunks; c0 += kDecCombineWarps * kBatch) {
     float2 ml[kBatch];
     float4 a[kBatch];
@@ -445,10 +448,13 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
       }
       count_launches(1);
     }
-    decode_combine_kernel<<<ns * num_q_heads, kDecCombineThreads, 0, s>>>(
-        P, op, mp, out + static_cast<int64_t>(s0) * num_q_heads * 128);
+    // programmatic dependent launch: the combine's CTAs are scheduled while the chunk kernel
+    // drains and wait (griddepcontrol.wait) for its completion before reading the partials
+    if (check_cuda(launch_pdl(decode_combine_kernel, dim3(ns * num_q_heads), dim3(kDecCombineThreads), 0, s, P,
+                              static_cast<const float *>(op), static_cast<const float2 *>(mp),
+                              out + static_cast<int64_t>(s0) * num_q_heads * 128)) != APACK_OK)
+      return APACK_ECUDA;
     count_launches(1);
-    if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     chunk_base += chunks;
   }
   return APACK_OK;

@@ -120,6 +120,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
                      const __grid_constant__ DecPlan plan, const uint16_t *__restrict__ q, float *__restrict__ opart,
                      float2 *__restrict__ mlpart, DeviceError *err) {
   using Lay = DLay<HKV>;
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");   // the combine may be scheduled
   extern __shared__ __align__(1024) uint8_t smem[];
   if ((smem_u32(smem) & 1023u) != 0) {
     if (threadIdx.x == 0) raise_device_error(err, APACK_EDEVICE, 90);
