@@ -32,6 +32,7 @@ namespace {
 
 constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;
+static_assert(kWarps == 32, "the keep-offset scan gives one lane to each warp of a CTA");
 constexpr int kMaxCached = 40960;               // tokens per CTA slice cached in shared memory (200 KB)
 constexpr size_t kCacheBytes = static_cast<size_t>(kMaxCached) * 5;
 
@@ -266,39 +267,44 @@ __global__ void __cluster_dims__(CL, 1, 1) __launch_bounds__(kThreads)
   cluster_sync();
   if (tid < CL * 5) rcnt[tid / 5][tid % 5] = ld_shared_cluster_u32(map_shared_rank(&cnt[tid % 5], tid / 5));
   __syncthreads();
-  if (tid == 0) {
-    // Walk the CTAs of the cluster, then the warps of this CTA, in token order:
-    // ties are granted until the quota runs out.
-    uint32_t kept_before = 0, kept_all = 0, seg_dev[2] = {0, 0};
-    uint32_t eq_prefix[2] = {0, 0}, eqb[2] = {0, 0};
-    for (int r = 0; r < CL; ++r) {
-      const uint32_t *c = rcnt[r];
-      uint32_t kept = c[0] + c[1] + c[2];
-      for (int s = 0; s < 2; ++s) {
-        const uint32_t ties = c[3 + s];
-        const uint32_t avail = quota[s] > eq_prefix[s] ? quota[s] - eq_prefix[s] : 0u;
-        kept += ties < avail ? ties : avail;
-        seg_dev[s] += c[1 + s] + ties;
-        if (r == static_cast<int>(crank)) eqb[s] = eq_prefix[s];
-        eq_prefix[s] += ties;
+  if (warp == 0) {
+    // Token order runs over the CTAs of the cluster, then over the warps of this CTA: ties are
+    // granted in that order until each segment's quota runs out.  Lane r stands for CTA r, then
+    // for warp r; exclusive prefix sums over the lanes replace a walk in order.
+    auto excl_scan = [&](uint32_t v) -> uint32_t {
+      uint32_t x = v;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, x, off);
+        if (lane >= off) x += y;
       }
-      if (r < static_cast<int>(crank)) kept_before += kept;
-      kept_all += kept;
+      return x - v;
+    };
+    auto granted = [](uint32_t ties, uint32_t before, uint32_t q) -> uint32_t {
+      const uint32_t avail = q > before ? q - before : 0u;
+      return ties < avail ? ties : avail;
+    };
+    // the cluster's CTAs
+    uint32_t c[5] = {0u, 0u, 0u, 0u, 0u};
+    if (lane < CL) {
+#pragma unroll
+      for (int i = 0; i < 5; ++i) c[i] = rcnt[lane][i];
     }
-    uint32_t run = kept_before;
-    for (int w = 0; w < kWarps; ++w) {
-      wbase[w] = run;
-      uint32_t kept = wcnt[w][0] + wcnt[w][1] + wcnt[w][2];
-      for (int s = 0; s < 2; ++s) {
-        weqb[w][s] = eqb[s];
-        const uint32_t ties = wcnt[w][3 + s];
-        const uint32_t avail = quota[s] > eqb[s] ? quota[s] - eqb[s] : 0u;
-        kept += ties < avail ? ties : avail;
-        eqb[s] += ties;
-      }
-      run += kept;
-    }
-    if (crank == 0) {
+    const uint32_t eqp0 = excl_scan(c[3]), eqp1 = excl_scan(c[4]);   // ties of the CTAs before
+    const uint32_t kept = c[0] + c[1] + c[2] + granted(c[3], eqp0, quota[0]) + granted(c[4], eqp1, quota[1]);
+    const uint32_t kept_excl = excl_scan(kept);
+    const uint32_t kept_all = __shfl_sync(0xffffffffu, kept_excl + kept, 31);
+    const uint32_t kept_before = __shfl_sync(0xffffffffu, kept_excl, static_cast<int>(crank));
+    const uint32_t eqb0 = __shfl_sync(0xffffffffu, eqp0, static_cast<int>(crank));
+    const uint32_t eqb1 = __shfl_sync(0xffffffffu, eqp1, static_cast<int>(crank));
+    // this CTA's warps (kWarps == 32: one lane each)
+    const uint32_t *wc = wcnt[lane];
+    const uint32_t we0 = eqb0 + excl_scan(wc[3]), we1 = eqb1 + excl_scan(wc[4]);
+    const uint32_t wk = wc[0] + wc[1] + wc[2] + granted(wc[3], we0, quota[0]) + granted(wc[4], we1, quota[1]);
+    wbase[lane] = kept_before + excl_scan(wk);
+    weqb[lane][0] = we0;
+    weqb[lane][1] = we1;
+    if (crank == 0 && lane == 0) {
       // Device-side consistency with the host counts.
       bool bad = kept_all != static_cast<uint32_t>(sq.out_len);
       for (int s = 0; s < nsegs; ++s)   // segment sizes seen by the first radix pass
