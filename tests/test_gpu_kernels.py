@@ -94,6 +94,7 @@ NARROW_SHAPES = [
     ([5000, 333], [1, 1], 16, 2),           # 3B heads, 8 rows per group
     ([4100], [2], 8, 4),                    # two query tokens, 4 rows per group
     ([777, 1500], [2, 2], 8, 2),            # two query tokens, 8 rows per group
+    ([140000], [1], 28, 4),                 # the paper's query row over a 140k-token sequence (8 tiles per CTA)
     # more rows per group: the general logits kernel
     ([3000, 700, 1, 0, 90], [1, 4, 2, 1, 0], 28, 4),
     ([5000], [2], 16, 2),                   # 16 rows per group
