@@ -49,10 +49,15 @@ namespace apack {
 
 namespace {
 
-constexpr int kEpiWG = 4;                         // epilogue warpgroups, one column range each
+constexpr int kEpiWG = 4;                         // epilogue warpgroups
 constexpr int kEpiWarps = 4 * kEpiWG;
-constexpr int kCols = 256 / kEpiWG;               // accumulator columns per epilogue thread and stage
-static_assert(kCols == 64, "the epilogues read 64 columns per thread and stage");
+// Warpgroups 2b and 2b + 1 own accumulator buffer b (the tiles of one parity): each reads half of
+// the buffer's 256 columns, in two loads of kCols, so that one pair computes while the other waits
+// for its next tile.
+constexpr int kPairWarps = kEpiWarps / 2;        // epilogue warps that read one buffer
+constexpr int kSpan = 128;                       // columns of a tile per warpgroup of the owning pair
+constexpr int kCols = 64;                        // columns per TMEM load
+static_assert(2 * kSpan == 256 && 2 * kCols == kSpan, "two warpgroups x two loads cover a 256-column tile");
 // warp 0: TMA, warp 1: TMEM (+ MMA on the even CTA), then the epilogue warps, then (pass 1) the
 // key-mask warp.  Nineteen warps take the same registers per thread as eighteen.
 constexpr int kMaskWarp = 2 + kEpiWarps;
@@ -241,13 +246,13 @@ __device__ PairCtx init_pair(uint8_t *smem, Bars *bars, int warp) {
       mbar_init(&bars->b_full[i], 1);
       mbar_init(&bars->b_empty[i], 1);
       mbar_init(&bars->l_full[i], 1);
-      mbar_init(&bars->l_empty[i], kEpiWarps);
+      mbar_init(&bars->l_empty[i], kPairWarps);    // stage i is read by the pair owning buffer i % 2
       mbar_init(&bars->m_full[i], 1);
-      mbar_init(&bars->m_empty[i], kEpiWarps);
+      mbar_init(&bars->m_empty[i], kPairWarps);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->acc_full[i], 1);
-      mbar_init(&bars->acc_empty[i], 2 * kEpiWarps);   // the epilogue warps of both CTAs
+      mbar_init(&bars->acc_empty[i], 2 * kPairWarps);  // the owning pair's warps in both CTAs
       mbar_init(&bars->comb_full[i], (kEpiWG - 1) * 4);
       mbar_init(&bars->comb_empty[i], 4);
     }
@@ -517,9 +522,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
     }
   } else {
-    // Epilogue: warpgroup q reads columns q*kCols.. (keys of the block) for the CTA's 128 rows;
-    // warp w reads TMEM lanes 32*(w%4)..
+    // Epilogue: warpgroup q reads the blocks of accumulator buffer q / 2 (every other block), its
+    // columns (q % 2) * 128.. (keys of the block) for the CTA's 128 rows; warp w reads TMEM lanes
+    // 32*(w%4)..
     const int q = (warp - 2) >> 2;
+    const int own = q >> 1;                                  // accumulator buffer of this warpgroup
+    const int col_base = (q & 1) * kSpan;
     const int quad = warp & 3;
     const int row = row_half + quad * 32 + lane;            // row of the 256-row pair
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
@@ -539,33 +547,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       // causal rows: this lane's row (token r of the query span) sees keys up to q_pos + r
       const int see = sp.q_pos + (w.qp * kChunk + row) / G;
       for (int b = w.b0; b < w.b1; ++b) {
-        // the keys of this thread's two 32-key chunks that count; and those this lane's row sees
-        if (!wait_or_abort(&bars->m_full[mi], mph, bars, pc, err, 20)) { ok = false; break; }
-        const uint2 mk = *reinterpret_cast<const uint2 *>(masks + mi * (kBlock / 32) + q * 2);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->m_empty[mi]);
+        if (ci == own) {   // blocks alternate between the buffers (mask slot mi % 2 == ci)
+          // the keys of this thread's four 32-key words that count; and those this lane's row sees
+          if (!wait_or_abort(&bars->m_full[mi], mph, bars, pc, err, 20)) { ok = false; break; }
+          const uint4 mk = *reinterpret_cast<const uint4 *>(masks + mi * (kBlock / 32) + (q & 1) * 4);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars->m_empty[mi]);
+          uint32_t rm[4] = {mk.x, mk.y, mk.z, mk.w};
+          if (CAUSAL) {        // keys at local index <= see
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int lim = see - (b * kBlock + col_base + 32 * i);
+              rm[i] &= lim >= 31 ? 0xffffffffu : (lim < 0 ? 0u : (2u << lim) - 1u);
+            }
+          }
+          if (!wait_or_abort(&bars->acc_full[ci], cph, bars, pc, err, 16)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const bool any = (h == 0 ? (mk.x | mk.y) : (mk.z | mk.w)) != 0u;   // uniform over the warp
+            uint32_t rr[kCols];
+            if (any) tmem_load_cols(bars->tmem_base + lane_off + ci * 256 + col_base + h * kCols, rr);
+            if (h == 1) {     // both halves are in registers: release the buffer
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);
+            }
+            if (any) online_block(rr, rm[2 * h], rm[2 * h + 1], c2, m, sum, bad);
+          }
+        }
         if (++mi == kBStages) { mi = 0; mph ^= 1; }
-        uint32_t rmask0 = mk.x, rmask1 = mk.y;
-        if (CAUSAL) {        // keys at local index <= see
-          const int lim0 = see - (b * kBlock + q * kCols), lim1 = lim0 - 32;
-          rmask0 &= lim0 >= 31 ? 0xffffffffu : (lim0 < 0 ? 0u : (2u << lim0) - 1u);
-          rmask1 &= lim1 >= 31 ? 0xffffffffu : (lim1 < 0 ? 0u : (2u << lim1) - 1u);
-        }
-        if (!wait_or_abort(&bars->acc_full[ci], cph, bars, pc, err, 16)) { ok = false; break; }
-        tc_fence_after();
-        if (mk.x | mk.y) {
-          const uint32_t tcol = bars->tmem_base + lane_off + ci * 256 + q * kCols;
-          uint32_t rr[kCols];
-          tmem_load_cols(tcol, rr);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);   // registers hold the data: release early
-          online_block(rr, rmask0, rmask1, c2, m, sum, bad);
-        } else {
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);
-        }
         if (++ci == 2) { ci = 0; cph ^= 1; }
       }
       if (!ok) break;
@@ -860,8 +871,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp < kMaskWarp) {
-    // Epilogue: warpgroup q reads columns q*kCols.. (rows of the chunk); one key per thread.
+    // Epilogue: warpgroup q reads the chunks of accumulator buffer q / 2 (every other chunk), its
+    // columns (q % 2) * 128.. (rows of the chunk); one key per thread.
     const int q = (warp - 2) >> 2;
+    const int own = q >> 1;                                  // accumulator buffer of this warpgroup
+    const int col_base = (q & 1) * kSpan;
     const int quad = warp & 3;
     const int tkey = quad * 32 + lane;
     const int klane = row_half + tkey;                  // key of the 256-key unit
@@ -881,26 +895,33 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       // causal rows: only packed rows rho >= rho_min (tokens r >= key - q_pos) see this key
       const int rho_min = CAUSAL ? max(0, w.kp * kBlock + klane - sp.q_pos) * G : 0;
       for (int c = 0; c < nch; ++c) {
-        if (!wait_or_abort(&bars->l_full[li], lph, bars, pc, err, 30)) { ok = false; break; }
-        if (!wait_or_abort(&bars->acc_full[ci], cph, bars, pc, err, 26)) { ok = false; break; }
-        tc_fence_after();
-        const float *nl = lse_s + li * kChunk + q * kCols;
-        const uint32_t tcol = bars->tmem_base + lane_off + ci * 256 + q * kCols;
-        uint32_t rr[kCols];
-        tmem_load_cols(tcol, rr);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);   // registers hold the data: release early
-        const int first = rho_min - (c * kChunk + q * kCols);
-        if (!CAUSAL || first <= 0) {
-          colsum_chunk<0>(rr, nl, c2, a);
-          colsum_chunk<32>(rr, nl + 32, c2, a);
-        } else if (first < kCols) {
-          colsum_chunk_from<0>(rr, nl, c2, first, a);
-          colsum_chunk_from<32>(rr, nl + 32, c2, first, a);
+        if (ci == own) {   // chunks alternate between the buffers (normaliser slot li % 2 == ci)
+          if (!wait_or_abort(&bars->l_full[li], lph, bars, pc, err, 30)) { ok = false; break; }
+          if (!wait_or_abort(&bars->acc_full[ci], cph, bars, pc, err, 26)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int col0 = col_base + h * kCols;
+            const float *nl = lse_s + li * kChunk + col0;
+            uint32_t rr[kCols];
+            tmem_load_cols(bars->tmem_base + lane_off + ci * 256 + col0, rr);
+            if (h == 1) {     // both halves are in registers: release the buffer
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);
+            }
+            const int first = rho_min - (c * kChunk + col0);
+            if (!CAUSAL || first <= 0) {
+              colsum_chunk<0>(rr, nl, c2, a);
+              colsum_chunk<32>(rr, nl + 32, c2, a);
+            } else if (first < kCols) {
+              colsum_chunk_from<0>(rr, nl, c2, first, a);
+              colsum_chunk_from<32>(rr, nl + 32, c2, first, a);
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars->l_empty[li]);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->l_empty[li]);
         if (++ci == 2) { ci = 0; cph ^= 1; }
         if (++li == kBStages) { li = 0; lph ^= 1; }
       }
