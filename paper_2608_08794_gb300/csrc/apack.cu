@@ -103,7 +103,12 @@ WsLayout workspace_layout(const apack_seqs *s) {
   L.qp_off = up(L.lse_off + static_cast<size_t>(qp_rows) * sizeof(float));
   L.qp_rows = qp_rows;
   L.gsum_off = up(L.qp_off + static_cast<size_t>(qp_rows) * 256);
-  L.total = up(L.gsum_off + static_cast<size_t>(s->num_kv_heads) * T * sizeof(float));
+  int64_t key_blocks = 0;   // 256-key blocks of the sequences that have query rows
+  for (int b = 0; b < s->num_seqs; ++b)
+    if (s->cu_qlens_h[b + 1] > s->cu_qlens_h[b])
+      key_blocks += (static_cast<int64_t>(s->cu_seqlens_h[b + 1]) - s->cu_seqlens_h[b] + 255) / 256;
+  L.mask_off = up(L.gsum_off + static_cast<size_t>(s->num_kv_heads) * T * sizeof(float));
+  L.total = up(L.mask_off + static_cast<size_t>(key_blocks) * 32);
   return L;
 }
 

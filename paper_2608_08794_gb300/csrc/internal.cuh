@@ -44,6 +44,7 @@ struct WsLayout {
   size_t lse_off;     // float [qp_rows]: negated log2 normaliser of every packed query row, -inf padding
   size_t qp_off;      // bf16 [qp_rows][128]: query rows repacked per KV head group, 256-row padded
   size_t gsum_off;    // float [Hkv][T]: per head group key sums of the column pass
+  size_t mask_off;    // uint32 [key blocks of the batch][8]: which keys of a block count (pass 1)
   // few query rows per head group (narrow path, used instead of the four above):
   bool narrow;
   size_t nlog_off;    // float [sum over sequences of Hq n_q len]: log2-domain logits

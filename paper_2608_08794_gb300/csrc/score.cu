@@ -34,11 +34,11 @@
 // (query rows in pass 1, keys in pass 2) is held for a run of streamed B tiles (key
 // blocks in pass 1, query chunks in pass 2), four B stages deep; two 256-column
 // accumulators alternate in TMEM.  Warp 0 issues TMA, warp 1 owns TMEM (and on the
-// even CTA issues the MMAs), warps 2..17 are four epilogue warpgroups; warpgroup w
-// reads columns 64w.. of the accumulator for the CTA's 128 lanes, 64 values per
-// thread and stage in one TMEM load.  In pass 1, warp 18 builds each key block's
-// masks once per CTA for all epilogue warps.  Operands sit in 128-byte swizzled
-// shared memory.  Persistent pairs, one CTA per SM.
+// even CTA issues the MMAs), warps 2..17 are four epilogue warpgroups; warpgroups 2b
+// and 2b + 1 read the tiles of accumulator b, 128 columns each for the CTA's 128 lanes,
+// in two TMEM loads of 64.  Pass 1 takes each key block's masks (which keys count)
+// from a bit array that the query repack kernel writes once per call.  Operands sit in
+// 128-byte swizzled shared memory.  Persistent pairs, one CTA per SM.
 #include <cmath>
 #include <cstdio>
 
@@ -60,8 +60,7 @@ constexpr int kCols = 64;                        // columns per TMEM load
 static_assert(2 * kSpan == 256 && 2 * kCols == kSpan, "two warpgroups x two loads cover a 256-column tile");
 // warp 0: TMA, warp 1: TMEM (+ MMA on the even CTA), then the epilogue warps, then (pass 1) the
 // key-mask warp.  Nineteen warps take the same registers per thread as eighteen.
-constexpr int kMaskWarp = 2 + kEpiWarps;
-constexpr int kThreads = 32 * (kMaskWarp + 1);
+constexpr int kThreads = 32 * (2 + kEpiWarps);
 constexpr uint32_t kTmemCols = 512;    // 2 accumulators x 256 fp32 columns
 constexpr int kAStages = 2, kBStages = 4;
 constexpr uint32_t kRows = 128;                // rows of A and of B per CTA (M/2, N/2 of the pair)
@@ -81,6 +80,7 @@ struct SeqPlan {
   int32_t q_pos;          // causal rows: position of query row 0 within the sequence
   int32_t unit_begin;     // pass 2: first work unit of this sequence in the launch
   int32_t flat0;          // pass 1: first flat (row group, key block) index of the sequence
+  int32_t blk0;           // pass 1: first key block of the sequence in the launch's mask array
 };
 
 struct ScorePlan {
@@ -101,21 +101,18 @@ struct __align__(8) Bars {
   uint64_t acc_full[2], acc_empty[2], drain;
   uint64_t l_full[kBStages], l_empty[kBStages];   // pass 2: normaliser slot loaded / released (this CTA)
   uint64_t comb_full[2], comb_empty[2];           // column ranges 1.. -> range 0 hand-off
-  uint64_t m_full[kBStages], m_empty[kBStages];   // pass 1: key masks of a block written / read
   uint32_t tmem_base;
   volatile int32_t abort;
 };
 
-// Shared memory: [A x2][B x4][-lse2 x4 (pass 2)][combine 2 x (kEpiWG - 1) x 128 float2]
-// [key masks 4 x 8 words (pass 1)][Bars].
+// Shared memory: [A x2][B x4][-lse2 x4 (pass 2)][combine 2 x (kEpiWG - 1) x 128 float2][Bars].
 // The dynamic shared window is declared 1024-byte aligned (the 128-byte swizzle
 // atoms of the operand tiles need it); the kernels verify it before any use.
 constexpr uint32_t kOffA = 0;
 constexpr uint32_t kOffB = kAStages * kTileBytes;
 constexpr uint32_t kOffL = kOffB + kBStages * kTileBytes;
 constexpr uint32_t kOffC = kOffL + kBStages * kChunk * sizeof(float);
-constexpr uint32_t kOffM = kOffC + 2 * (kEpiWG - 1) * kRows * sizeof(float2);
-constexpr uint32_t kOffBars = kOffM + kBStages * (kBlock / 32) * sizeof(uint32_t);
+constexpr uint32_t kOffBars = kOffC + 2 * (kEpiWG - 1) * kRows * sizeof(float2);
 constexpr uint32_t kSmemBytes = kOffBars + 512;
 static_assert(sizeof(Bars) <= 512, "barrier block");
 static_assert(kSmemBytes <= 232448, "shared memory budget");
@@ -247,8 +244,6 @@ __device__ PairCtx init_pair(uint8_t *smem, Bars *bars, int warp) {
       mbar_init(&bars->b_empty[i], 1);
       mbar_init(&bars->l_full[i], 1);
       mbar_init(&bars->l_empty[i], kPairWarps);    // stage i is read by the pair owning buffer i % 2
-      mbar_init(&bars->m_full[i], 1);
-      mbar_init(&bars->m_empty[i], kPairWarps);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->acc_full[i], 1);
@@ -389,7 +384,7 @@ __device__ __forceinline__ void online_block(uint32_t (&r)[64], uint32_t mask0, 
 template <bool CAUSAL>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     score_rowstats_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
-                          const __grid_constant__ ScorePlan plan, const uint8_t *__restrict__ modality,
+                          const __grid_constant__ ScorePlan plan, const uint32_t *__restrict__ mask_words,
                           float2 *__restrict__ part, DeviceError *err) {
   extern __shared__ __align__(1024) uint8_t smem[];
   if (!smem_aligned(smem)) {   // the same in both CTAs of the pair: both leave here
@@ -472,55 +467,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (++ai == kAStages) { ai = 0; aph ^= 1; }
       }
     }
-  } else if (warp == kMaskWarp) {
-    // Key masks: for every block, bit k of word c says whether key c*32 + k of the block counts
-    // (in the sequence and, outside the causal domain, in S); written once per CTA for all
-    // epilogue warps.  The modality bytes are loaded two blocks ahead of the block being masked.
-    uint32_t *masks = reinterpret_cast<uint32_t *>(smem + kOffM);
-    constexpr int kW = kBlock / 32;
-    // key range of flat item x: first key of its block and end of its sequence
-    auto block_keys = [&](int x, int &key_base, int &t_end) {
-      const SeqPlan &sp = plan.seq[seq_of_flat(plan, x)];
-      key_base = sp.t0 + ((x - sp.flat0) % sp.nb) * kBlock;
-      t_end = sp.t0 + sp.len;
-    };
-    auto load = [&](int x, uint8_t (&mod)[kW]) {
-      if (x >= x_end) return;
-      int kb, te;
-      block_keys(x, kb, te);
-#pragma unroll
-      for (int c = 0; c < kW; ++c) {
-        const int key = kb + c * 32 + lane;
-        mod[c] = key < te ? modality[key] : 0;
-      }
-    };
-    uint8_t m0[kW], m1[kW], m2[kW];
-    load(x_begin, m0);
-    load(x_begin + 1, m1);
-    int mi = 0;
-    uint32_t mph = 0;
-    for (int x = x_begin; x < x_end; ++x) {
-      load(x + 2, m2);
-      int kb, te;
-      block_keys(x, kb, te);
-      if (!wait_or_abort(&bars->m_empty[mi], mph ^ 1, bars, pc, err, 19)) break;
-      uint32_t word = 0;
-#pragma unroll
-      for (int c = 0; c < kW; ++c) {
-        const int key = kb + c * 32 + lane;
-        const uint32_t mk = __ballot_sync(0xffffffffu, key < te && (CAUSAL || is_mm(m0[c])));
-        if (lane == c) word = mk;
-      }
-      if (lane < kW) masks[mi * kW + lane] = word;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->m_full[mi]);
-      if (++mi == kBStages) { mi = 0; mph ^= 1; }
-#pragma unroll
-      for (int c = 0; c < kW; ++c) {
-        m0[c] = m1[c];
-        m1[c] = m2[c];
-      }
-    }
   } else {
     // Epilogue: warpgroup q reads the blocks of accumulator buffer q / 2 (every other block), its
     // columns (q % 2) * 128.. (keys of the block) for the CTA's 128 rows; warp w reads TMEM lanes
@@ -534,9 +480,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const uint32_t acc_empty0 = lead_addr(pc, bars, &bars->acc_empty[0]);
     const float c2 = plan.scale2;
     float2 *comb = reinterpret_cast<float2 *>(smem + kOffC);   // [2 parities][kEpiWG - 1 ranges][128 rows]
-    const uint32_t *masks = reinterpret_cast<const uint32_t *>(smem + kOffM);
-    int ci = 0, mi = 0;
-    uint32_t cph = 0, xph = 0, mph = 0;
+    int ci = 0;
+    uint32_t cph = 0, xph = 0;
     bool ok = true;
     for (int x = x_begin; ok && x < x_end;) {
       const Run w = next_run(plan, x, x_end, pair);
@@ -546,13 +491,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool bad = false;
       // causal rows: this lane's row (token r of the query span) sees keys up to q_pos + r
       const int see = sp.q_pos + (w.qp * kChunk + row) / G;
+      // the warpgroup's four 32-key mask words of a block (which keys count), one own block
+      // ahead: lane i < 4 holds word i, shuffled to every lane when the block is taken
+      const uint32_t *mwords = mask_words + sp.blk0 * 8 + (q & 1) * 4 + (lane & 3);
+      const int b_first = w.b0 + ((own - ci + 2) & 1);       // blocks alternate between the buffers
+      uint32_t m_next = (b_first < w.b1 && lane < 4) ? __ldg(mwords + b_first * 8) : 0u;
       for (int b = w.b0; b < w.b1; ++b) {
-        if (ci == own) {   // blocks alternate between the buffers (mask slot mi % 2 == ci)
-          // the keys of this thread's four 32-key words that count; and those this lane's row sees
-          if (!wait_or_abort(&bars->m_full[mi], mph, bars, pc, err, 20)) { ok = false; break; }
-          const uint4 mk = *reinterpret_cast<const uint4 *>(masks + mi * (kBlock / 32) + (q & 1) * 4);
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->m_empty[mi]);
+        if (ci == own) {
+          const uint32_t m_mine = m_next;
+          if (b + 2 < w.b1 && lane < 4) m_next = __ldg(mwords + (b + 2) * 8);
+          const uint4 mk = make_uint4(__shfl_sync(0xffffffffu, m_mine, 0), __shfl_sync(0xffffffffu, m_mine, 1),
+                                      __shfl_sync(0xffffffffu, m_mine, 2), __shfl_sync(0xffffffffu, m_mine, 3));
+          // the keys of this thread's words that count; and those this lane's row sees
           uint32_t rm[4] = {mk.x, mk.y, mk.z, mk.w};
           if (CAUSAL) {        // keys at local index <= see
 #pragma unroll
@@ -576,7 +526,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             if (any) online_block(rr, rm[2 * h], rm[2 * h + 1], c2, m, sum, bad);
           }
         }
-        if (++mi == kBStages) { mi = 0; mph ^= 1; }
         if (++ci == 2) { ci = 0; cph ^= 1; }
       }
       if (!ok) break;
@@ -630,9 +579,29 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 // Packed Q: for each sequence and KV head group g, rows rho = token * G + j hold
 // query head g*G + j of that token (16-byte vectors, zero padding to 256 rows).
 __global__ void q_pack_kernel(const __grid_constant__ ScorePlan plan, const uint4 *__restrict__ q,
-                              uint4 *__restrict__ qp, int64_t row_begin, int64_t n_vec) {
+                              uint4 *__restrict__ qp, int64_t row_begin, int64_t n_vec,
+                              const uint8_t *__restrict__ modality, uint32_t *__restrict__ mask_words,
+                              int64_t n_words) {
   const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (e >= n_vec) return;
+  if (e >= n_vec) {
+    // pass 1's key masks: word c of block b of a sequence has bit k set when key 32c + k of the
+    // block is in the sequence and counts in the denominator (in S; every key in the causal
+    // domain, whose per-row limit the epilogue applies)
+    const int64_t wd = e - n_vec;
+    if (wd >= n_words) return;
+    const int gb = static_cast<int>(wd >> 3), c = static_cast<int>(wd & 7);
+    int s = 0;
+    while (s + 1 < plan.nseq && plan.seq[s + 1].blk0 <= gb) ++s;
+    const SeqPlan &sp = plan.seq[s];
+    const int key0 = sp.t0 + (gb - sp.blk0) * kBlock + c * 32, t_end = sp.t0 + sp.len;
+    uint32_t word = 0;
+    for (int k = 0; k < 32; ++k) {
+      const int key = key0 + k;
+      if (key < t_end && (plan.causal || is_mm(modality[key]))) word |= 1u << k;
+    }
+    mask_words[wd] = word;
+    return;
+  }
   const int64_t prow = row_begin + e / 16;
   const int v = static_cast<int>(e % 16);
   int s = 0;
@@ -870,7 +839,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (++ai == kAStages) { ai = 0; aph ^= 1; }
       }
     }
-  } else if (warp < kMaskWarp) {
+  } else {
     // Epilogue: warpgroup q reads the chunks of accumulator buffer q / 2 (every other chunk), its
     // columns (q % 2) * 128.. (rows of the chunk); one key per thread.
     const int q = (warp - 2) >> 2;
@@ -1061,6 +1030,7 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
   float *nlse2 = reinterpret_cast<float *>(wsb + L.lse_off);
   uint8_t *qp = wsb + L.qp_off;
   float *gsum = reinterpret_cast<float *>(wsb + L.gsum_off);
+  uint32_t *mask_words = reinterpret_cast<uint32_t *>(wsb + L.mask_off);
 
   if (once_per_device(g_attr_done, [] {
         cudaError_t e = cudaFuncSetAttribute(score_rowstats_kernel<false>,
@@ -1097,7 +1067,7 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
     P.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(APACK_HEAD_DIM)));
     P.causal = seqs->softmax_domain == APACK_SOFTMAX_CAUSAL_ROW;
     int64_t qrows = 0, flat = 0, nb_max = 0;
-    int units2 = 0;
+    int units2 = 0, blocks = 0;
     for (int i = 0; i < ns; ++i) {
       const int b = s0 + i;
       SeqPlan &sp = P.seq[i];
@@ -1111,6 +1081,8 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
       sp.nb = sp.n_q > 0 ? (sp.len + kBlock - 1) / kBlock : 0;
       sp.q_pos = query_position(seqs, b);
       sp.flat0 = static_cast<int32_t>(flat);
+      sp.blk0 = blocks;
+      blocks += sp.nb;
       flat += pass1_items(sp, hkv);
       if (sp.nb > nb_max) nb_max = sp.nb;
       sp.unit_begin = units2;
@@ -1128,20 +1100,22 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
       if (pairs1 < 1) pairs1 = 1;
     }
     P.pairs = static_cast<int32_t>(pairs1);
-    // repack the query rows of this launch's sequences
+    // repack the query rows of this launch's sequences and write pass 1's key masks
+    const int64_t n_words = static_cast<int64_t>(blocks) * (kBlock / 32);
     if (qrows > 0) {
       const int64_t n_vec = qrows * 16;
-      q_pack_kernel<<<static_cast<unsigned>((n_vec + 255) / 256), 256, 0, stream>>>(
-          P, static_cast<const uint4 *>(q), reinterpret_cast<uint4 *>(qp), qp_base, n_vec);
+      q_pack_kernel<<<static_cast<unsigned>((n_vec + n_words + 255) / 256), 256, 0, stream>>>(
+          P, static_cast<const uint4 *>(q), reinterpret_cast<uint4 *>(qp), qp_base, n_vec, seqs->modality, mask_words,
+          n_words);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
     if (flat > 0) {
       const unsigned grid = static_cast<unsigned>(2 * pairs1);
       if (P.causal)
-        score_rowstats_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, seqs->modality, part, err);
+        score_rowstats_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, mask_words, part, err);
       else
-        score_rowstats_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, seqs->modality, part, err);
+        score_rowstats_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, mask_words, part, err);
       count_launches(1);
       if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
