@@ -56,8 +56,10 @@ constexpr int kEpiWarps = 4 * kEpiWG;
 // for its next tile.
 constexpr int kPairWarps = kEpiWarps / 2;        // epilogue warps that read one buffer
 constexpr int kSpan = 128;                       // columns of a tile per warpgroup of the owning pair
-constexpr int kCols = 64;                        // columns per TMEM load
-static_assert(2 * kSpan == 256 && 2 * kCols == kSpan, "two warpgroups x two loads cover a 256-column tile");
+constexpr int kCols = 64;                        // columns per TMEM load, pass 1
+constexpr int kCols2 = 32;                       // columns per TMEM load, pass 2
+static_assert(2 * kSpan == 256 && 2 * kCols == kSpan && 4 * kCols2 == kSpan,
+              "two warpgroups x (two or four) loads cover a 256-column tile");
 // warp 0: TMA, warp 1: TMEM (+ MMA on the even CTA), then the epilogue warps, then (pass 1) the
 // key-mask warp.  Nineteen warps take the same registers per thread as eighteen.
 constexpr int kThreads = 32 * (2 + kEpiWarps);
@@ -299,6 +301,10 @@ __device__ void drain_loads(uint64_t *full, const bool *pending, const uint32_t 
 // kCols consecutive TMEM columns of this warp's 32 lanes -> registers, loaded and waited for
 // in one statement (the registers are defined only once the data is there).
 __device__ __forceinline__ void tmem_load_cols(uint32_t taddr, uint32_t (&r)[64]) { tmem_ld64_wait(taddr, r); }
+__device__ __forceinline__ void tmem_load_cols(uint32_t taddr, uint32_t (&r)[32]) {
+  tmem_ld32(taddr, r);
+  tmem_wait32(r);
+}
 
 // The eight K=16 steps of one 256 x 256 x 128 product into accumulator `ci`.
 __device__ __forceinline__ void issue_mma(uint32_t tmem, int ci, uint32_t a_base, uint32_t b_base) {
@@ -716,30 +722,27 @@ __device__ __forceinline__ Unit2 decode_unit2(const ScorePlan &p, int u) {
   return w;
 }
 
-// a[0..3] += 2^(x c2 + nl[col]) over 32 columns (four independent partial sums).
-template <int OFF>
-__device__ __forceinline__ void colsum_chunk(const uint32_t (&r)[kCols], const float *nl, float c2, float2 (&a)[4]) {
+// a[0..3] += 2^(x c2 + nl[col]) over the 32 columns of one load (four independent partial sums).
+__device__ __forceinline__ void colsum_word(const uint32_t (&r)[kCols2], const float *nl, float c2, float2 (&a)[4]) {
   const float2 cc = make_float2(c2, c2);
 #pragma unroll
   for (int i = 0; i < 32; i += 4) {
     const float4 L = *reinterpret_cast<const float4 *>(nl + i);
-    const float2 y0 = ffma2(make_float2(__uint_as_float(r[OFF + i]), __uint_as_float(r[OFF + i + 1])), cc,
-                            make_float2(L.x, L.y));
-    const float2 y1 = ffma2(make_float2(__uint_as_float(r[OFF + i + 2]), __uint_as_float(r[OFF + i + 3])), cc,
-                            make_float2(L.z, L.w));
+    const float2 y0 = ffma2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), cc, make_float2(L.x, L.y));
+    const float2 y1 =
+        ffma2(make_float2(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])), cc, make_float2(L.z, L.w));
     a[(i >> 2) & 3] = fadd2(a[(i >> 2) & 3], make_float2(ex2_approx(y0.x), ex2_approx(y0.y)));
     a[(i >> 2) & 3] = fadd2(a[(i >> 2) & 3], make_float2(ex2_approx(y1.x), ex2_approx(y1.y)));
   }
 }
 
-// The same over the columns OFF + i >= first only (causal rows that cannot see the key drop out;
+// The same over the columns i >= first only (causal rows that cannot see the key drop out;
 // taken only by keys inside the query span).
-template <int OFF>
-__device__ __forceinline__ void colsum_chunk_from(const uint32_t (&r)[kCols], const float *nl, float c2, int first,
-                                                  float2 (&a)[4]) {
+__device__ __forceinline__ void colsum_word_from(const uint32_t (&r)[kCols2], const float *nl, float c2, int first,
+                                                 float2 (&a)[4]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i)
-    if (OFF + i >= first) a[i & 3].x += ex2_approx(fmaf(__uint_as_float(r[OFF + i]), c2, nl[i]));
+    if (i >= first) a[i & 3].x += ex2_approx(fmaf(__uint_as_float(r[i]), c2, nl[i]));
 }
 
 // Work unit = (256 keys, KV head group g): 128 keys per CTA of the pair; writes the group's
@@ -869,24 +872,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (!wait_or_abort(&bars->acc_full[ci], cph, bars, pc, err, 26)) { ok = false; break; }
           tc_fence_after();
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int col0 = col_base + h * kCols;
+          for (int h = 0; h < kSpan / kCols2; ++h) {
+            const int col0 = col_base + h * kCols2;
             const float *nl = lse_s + li * kChunk + col0;
-            uint32_t rr[kCols];
+            uint32_t rr[kCols2];
             tmem_load_cols(bars->tmem_base + lane_off + ci * 256 + col0, rr);
-            if (h == 1) {     // both halves are in registers: release the buffer
+            if (h == kSpan / kCols2 - 1) {     // every column is in registers: release the buffer
               tc_fence_before();
               __syncwarp();
               if (lane == 0) arrive_cluster(acc_empty0 + ci * 8);
             }
             const int first = rho_min - (c * kChunk + col0);
-            if (!CAUSAL || first <= 0) {
-              colsum_chunk<0>(rr, nl, c2, a);
-              colsum_chunk<32>(rr, nl + 32, c2, a);
-            } else if (first < kCols) {
-              colsum_chunk_from<0>(rr, nl, c2, first, a);
-              colsum_chunk_from<32>(rr, nl + 32, c2, first, a);
-            }
+            if (!CAUSAL || first <= 0)
+              colsum_word(rr, nl, c2, a);
+            else if (first < kCols2)
+              colsum_word_from(rr, nl, c2, first, a);
           }
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->l_empty[li]);
