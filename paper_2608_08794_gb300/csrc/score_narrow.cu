@@ -155,8 +155,21 @@ __global__ void __launch_bounds__(kThreads)
   const int rho = static_cast<int>(e - acc);
   const int ctas = sq.nparts;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // up to kHold partials per thread are loaded once, together, and kept for the sum
+  constexpr int kHold = 8;
+  const bool held = ctas <= kHold * kThreads;
+  float2 v[kHold];
   float m = -INFINITY;
-  for (int c = tid; c < ctas; c += kThreads) m = fmaxf(m, part[sq.part_base + static_cast<int64_t>(c) * sq.rows + rho].x);
+  if (held) {
+#pragma unroll
+    for (int i = 0; i < kHold; ++i) {
+      const int c = tid + i * kThreads;
+      v[i] = c < ctas ? part[sq.part_base + static_cast<int64_t>(c) * sq.rows + rho] : make_float2(-INFINITY, 0.f);
+      m = fmaxf(m, v[i].x);
+    }
+  } else {
+    for (int c = tid; c < ctas; c += kThreads) m = fmaxf(m, part[sq.part_base + static_cast<int64_t>(c) * sq.rows + rho].x);
+  }
   m = warp_max(m);
   if (lane == 0) red[warp] = m;
   __syncthreads();
@@ -168,11 +181,18 @@ __global__ void __launch_bounds__(kThreads)
   __syncthreads();
   m = mshared;
   float sum = 0.f;
-  if (m != -INFINITY)
-    for (int c = tid; c < ctas; c += kThreads) {
-      const float2 v = part[sq.part_base + static_cast<int64_t>(c) * sq.rows + rho];
-      if (v.x != -INFINITY) sum += v.y * exp2f(v.x - m);
+  if (m != -INFINITY) {
+    if (held) {
+#pragma unroll
+      for (int i = 0; i < kHold; ++i)   // the same partials in the same order as the loop below
+        if (v[i].x != -INFINITY) sum += v[i].y * exp2f(v[i].x - m);
+    } else {
+      for (int c = tid; c < ctas; c += kThreads) {
+        const float2 w = part[sq.part_base + static_cast<int64_t>(c) * sq.rows + rho];
+        if (w.x != -INFINITY) sum += w.y * exp2f(w.x - m);
+      }
     }
+  }
   sum = warp_sum(sum);
   __syncthreads();
   if (lane == 0) red[warp] = sum;
@@ -195,24 +215,32 @@ __global__ void __launch_bounds__(kThreads)
   const int s = find_unit_seq(plan, blockIdx.x);
   const NSeq &sq = plan.seq[s];
   const int R = sq.rows;
-  for (int i = threadIdx.x; i < R; i += kThreads) ls[i] = lse2[sq.lse_base + i];
-  __syncthreads();
   const int kt = blockIdx.x - sq.unit_begin;
   const int key = sq.t0 + kt * kThreads + threadIdx.x;
-  if (key >= sq.t0 + sq.len) return;
+  const bool in = key < sq.t0 + sq.len;
+  const float *lp = logits + sq.logit_base + (key - sq.t0);
+  // the key's own loads (modality, and up to 32 rows' logits) are issued before the normalisers
+  // arrive: one round trip for all of them
+  const uint8_t mod = in ? modality[key] : static_cast<uint8_t>(0);
+  float raw[32];
+  if (R <= 32) {
+#pragma unroll
+    for (int u = 0; u < 32; ++u) raw[u] = (in && u < R) ? lp[static_cast<int64_t>(u) * sq.lstride] : 0.f;
+  }
+  for (int i = threadIdx.x; i < R; i += kThreads) ls[i] = lse2[sq.lse_base + i];
+  __syncthreads();
+  if (!in) return;
   float out = 0.f;
-  if (sq.n_q > 0 && is_mm(modality[key])) {
+  if (sq.n_q > 0 && is_mm(mod)) {
     // eight independent sums, the loads of a block of 8 rows issued together
-    const float *lp = logits + sq.logit_base + (key - sq.t0);
     float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     // causal rows: logit row rho = token * Hq + head sees this key when token >= key - q_pos
     const int rho_min = plan.causal ? max(0, key - sq.t0 - sq.q_pos) * plan.hq : 0;
     if (R <= 32) {
-      // all rows' logits requested at once: one round trip (the paper's one query token: R = Hq)
+      // all rows (the paper's one query token: R = Hq)
       float x[32];
 #pragma unroll
-      for (int u = 0; u < 32; ++u)
-        x[u] = (u < R && u >= rho_min) ? lp[static_cast<int64_t>(u) * sq.lstride] - ls[u] : -INFINITY;
+      for (int u = 0; u < 32; ++u) x[u] = (u < R && u >= rho_min) ? raw[u] - ls[u] : -INFINITY;
 #pragma unroll
       for (int u = 0; u < 32; ++u) a[u & 7] += ex2_approx(x[u]);
     } else {
