@@ -14,7 +14,9 @@
 //                zeroed by the pool kernel) computes c-bar, min/max of d, the min-max
 //                normalised distance and the gated score s_f of Eq. gate (blend when
 //                c-bar < tau) over the whole clip.
-// All reductions run in a fixed order: results are deterministic.  Two launches per call.
+// All reductions run in a fixed order: results are deterministic.  Two launches per call; the
+// CKA kernel is a programmatic dependent of the pool kernel (scheduled while the pool drains,
+// waiting for its completion before any read).
 #include <algorithm>
 #include <cmath>
 
@@ -41,6 +43,7 @@ __global__ void __launch_bounds__(kPoolMaxThreads, 2)
     frame_pool_kernel(const uint4 *__restrict__ visual, const uint4 *__restrict__ audio, int n_frames, int tpf,
                       int n_audio, int64_t dim, float *__restrict__ v_out, float *__restrict__ a_out,
                       unsigned int *done) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");   // the CKA kernel may be scheduled
   const int f = blockIdx.x;
   if (f == 0 && blockIdx.y == 0 && threadIdx.x == 0) *done = 0u;   // CTA counter of the CKA kernel
   const int64_t fi = (static_cast<int64_t>(blockIdx.y) * blockDim.x + threadIdx.x) * 8;
@@ -76,6 +79,7 @@ __global__ void __launch_bounds__(kCkaThreads)
                           float tau, float beta, unsigned int *done, float *__restrict__ c_out,
                           float *__restrict__ d_out, float *__restrict__ s_out, float *__restrict__ dn_out,
                           float *__restrict__ cbar_out) {
+  pdl_wait_and_release();   // the pooled rows (and the zeroed counter) of the pool kernel are visible
   constexpr int kG = W * (W + 1) / 2;
   constexpr int kN = 2 * kG + 1;
   constexpr int kWarps = kCkaThreads / 32;
@@ -264,26 +268,28 @@ apack_status apack_frame_alignment(const void *visual, const void *audio, int32_
                                               n_frames, tokens_per_frame, n_audio, dim, vbuf, abuf, done);
   count_launches(1);
   if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+  // programmatic dependent launch: the CKA kernel's CTAs are scheduled while the pool kernel drains
+  cudaError_t e = cudaSuccess;
   switch (window) {
     case 1:
-      frame_cka_gate_kernel<1><<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, tau, beta, done, c_out,
-                                                                dbuf, s_out, dnorm_out, cbar_out);
+      e = launch_pdl(frame_cka_gate_kernel<1>, dim3(n_frames), dim3(kCkaThreads), 0, s, vbuf, abuf, n_frames, dim,
+                     tau, beta, done, c_out, dbuf, s_out, dnorm_out, cbar_out);
       break;
     case 3:
-      frame_cka_gate_kernel<3><<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, tau, beta, done, c_out,
-                                                                dbuf, s_out, dnorm_out, cbar_out);
+      e = launch_pdl(frame_cka_gate_kernel<3>, dim3(n_frames), dim3(kCkaThreads), 0, s, vbuf, abuf, n_frames, dim,
+                     tau, beta, done, c_out, dbuf, s_out, dnorm_out, cbar_out);
       break;
     case 5:
-      frame_cka_gate_kernel<5><<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, tau, beta, done, c_out,
-                                                                dbuf, s_out, dnorm_out, cbar_out);
+      e = launch_pdl(frame_cka_gate_kernel<5>, dim3(n_frames), dim3(kCkaThreads), 0, s, vbuf, abuf, n_frames, dim,
+                     tau, beta, done, c_out, dbuf, s_out, dnorm_out, cbar_out);
       break;
     default:
-      frame_cka_gate_kernel<7><<<n_frames, kCkaThreads, 0, s>>>(vbuf, abuf, n_frames, dim, tau, beta, done, c_out,
-                                                                dbuf, s_out, dnorm_out, cbar_out);
+      e = launch_pdl(frame_cka_gate_kernel<7>, dim3(n_frames), dim3(kCkaThreads), 0, s, vbuf, abuf, n_frames, dim,
+                     tau, beta, done, c_out, dbuf, s_out, dnorm_out, cbar_out);
       break;
   }
   count_launches(1);
-  if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+  if (check_cuda(e) != APACK_OK) return APACK_ECUDA;
   return APACK_OK;
 }
 
