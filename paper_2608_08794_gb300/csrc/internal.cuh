@@ -61,14 +61,15 @@ int device_sm_count();
 void count_launches(uint64_t n);
 apack_status check_cuda(cudaError_t e);
 
-// Programmatic dependent launch.  The kernels of the few-row scoring path are launched with
+// Programmatic dependent launch.  The scoring kernels (both paths) are launched with
 // programmatic stream serialization: a kernel may be scheduled while its predecessor on the
 // stream drains, and it waits (griddepcontrol.wait, first statement of the kernel) until that
 // predecessor has completed and its memory is visible, before any global access.  Each such
 // kernel lets its own successor launch early (griddepcontrol.launch_dependents) right after that
-// wait.  Measured on GB300, per-step calls with one query row: scoring 0.541 -> 0.487 ms summed
-// over 14 steps.  The wide scoring chain got slower with it (0.796 -> 0.849 ms) and selection and
-// compaction did not gain, so those launch plainly.
+// wait.  Measured on GB300, per-step calls: few-row scoring 0.541 -> 0.487 ms summed over the
+// paper's 14 steps; the tensor-core scoring chain 0.697 -> 0.675 ms over the 3-step 10-minute
+// schedule (a captured graph of the schedule gains nothing: it has no launch gaps to hide).
+// Selection and compaction did not gain, so those launch plainly.
 __device__ __forceinline__ void pdl_wait_and_release() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");

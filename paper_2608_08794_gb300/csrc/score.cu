@@ -392,6 +392,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     score_rowstats_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                           const __grid_constant__ ScorePlan plan, const uint32_t *__restrict__ mask_words,
                           float2 *__restrict__ part, DeviceError *err) {
+  pdl_wait_and_release();
   extern __shared__ __align__(1024) uint8_t smem[];
   if (!smem_aligned(smem)) {   // the same in both CTAs of the pair: both leave here
     if (threadIdx.x == 0) raise_device_error(err, APACK_EDEVICE, 10);
@@ -588,6 +589,7 @@ __global__ void q_pack_kernel(const __grid_constant__ ScorePlan plan, const uint
                               uint4 *__restrict__ qp, int64_t row_begin, int64_t n_vec,
                               const uint8_t *__restrict__ modality, uint32_t *__restrict__ mask_words,
                               int64_t n_words) {
+  pdl_wait_and_release();
   const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
   if (e >= n_vec) {
     // pass 1's key masks: word c of block b of a sequence has bit k set when key 32c + k of the
@@ -639,6 +641,7 @@ __global__ void lse_merge_kernel(const __grid_constant__ ScorePlan plan, const f
                                  const uint16_t *__restrict__ qp, const uint8_t *__restrict__ k,
                                  int64_t k_stride, const uint8_t *__restrict__ modality, float *__restrict__ nlse2,
                                  int64_t row_begin, int64_t n_rows) {
+  pdl_wait_and_release();
   __shared__ float qsh[8][128];                           // the query row of each warp (fallback only)
   const int64_t e = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
@@ -752,6 +755,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     score_colsum_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                         const __grid_constant__ ScorePlan plan, const float *__restrict__ nlse2,
                         float *__restrict__ gsum, DeviceError *err) {
+  pdl_wait_and_release();
   extern __shared__ __align__(1024) uint8_t smem[];
   if (!smem_aligned(smem)) {   // the same in both CTAs of the pair: both leave here
     if (threadIdx.x == 0) raise_device_error(err, APACK_EDEVICE, 10);
@@ -925,6 +929,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 __global__ void score_finalize_kernel(const __grid_constant__ ScorePlan plan, const uint8_t *__restrict__ modality,
                                       const float *__restrict__ gsum, float *__restrict__ scores, int64_t t_begin,
                                       int64_t n) {
+  pdl_wait_and_release();
   const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
   if (e >= n) return;
   const int64_t i = t_begin + e;
@@ -1104,53 +1109,58 @@ apack_status run_score(const apack_seqs *seqs, const void *q, const void *k, int
     const int64_t n_words = static_cast<int64_t>(blocks) * (kBlock / 32);
     if (qrows > 0) {
       const int64_t n_vec = qrows * 16;
-      q_pack_kernel<<<static_cast<unsigned>((n_vec + n_words + 255) / 256), 256, 0, stream>>>(
-          P, static_cast<const uint4 *>(q), reinterpret_cast<uint4 *>(qp), qp_base, n_vec, seqs->modality, mask_words,
-          n_words);
+      if (check_cuda(launch_pdl(q_pack_kernel, dim3(static_cast<unsigned>((n_vec + n_words + 255) / 256)), dim3(256), 0,
+                                stream, P, static_cast<const uint4 *>(q), reinterpret_cast<uint4 *>(qp), qp_base, n_vec,
+                                seqs->modality, mask_words, n_words)) != APACK_OK)
+        return APACK_ECUDA;
       count_launches(1);
-      if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
     if (flat > 0) {
       const unsigned grid = static_cast<unsigned>(2 * pairs1);
-      if (P.causal)
-        score_rowstats_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, mask_words, part, err);
-      else
-        score_rowstats_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, mask_words, part, err);
+      const uint32_t *mw = mask_words;
+      const cudaError_t e = P.causal ? launch_pdl(score_rowstats_kernel<true>, dim3(grid), dim3(kThreads), kSmemBytes,
+                                                  stream, qmap, kmap, P, mw, part, err)
+                                     : launch_pdl(score_rowstats_kernel<false>, dim3(grid), dim3(kThreads), kSmemBytes,
+                                                  stream, qmap, kmap, P, mw, part, err);
       count_launches(1);
-      if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+      if (check_cuda(e) != APACK_OK) return APACK_ECUDA;
     }
     if (qrows > 0) {
       const unsigned blocks = static_cast<unsigned>((qrows * 32 + 255) / 256);   // one warp per packed row
       const uint16_t *qp16 = reinterpret_cast<const uint16_t *>(qp);
       const uint8_t *k8 = static_cast<const uint8_t *>(k);
-      if (P.causal)
-        lse_merge_kernel<true><<<blocks, 256, 0, stream>>>(P, part, qp16, k8, k_token_stride, seqs->modality, nlse2,
-                                                           qp_base, qrows);
-      else
-        lse_merge_kernel<false><<<blocks, 256, 0, stream>>>(P, part, qp16, k8, k_token_stride, seqs->modality, nlse2,
-                                                            qp_base, qrows);
+      const float2 *pc = part;
+      const int64_t qb = qp_base;
+      const cudaError_t e =
+          P.causal ? launch_pdl(lse_merge_kernel<true>, dim3(blocks), dim3(256), 0, stream, P, pc, qp16, k8,
+                                k_token_stride, static_cast<const uint8_t *>(seqs->modality), nlse2, qb, qrows)
+                   : launch_pdl(lse_merge_kernel<false>, dim3(blocks), dim3(256), 0, stream, P, pc, qp16, k8,
+                                k_token_stride, static_cast<const uint8_t *>(seqs->modality), nlse2, qb, qrows);
       count_launches(1);
-      if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+      if (check_cuda(e) != APACK_OK) return APACK_ECUDA;
     }
     // Pass 2 units: (256 keys, head group), dealt round-robin to the pairs.
     P.total_units = units2;
     if (units2 > 0) {
       const int pairs2 = units2 < max_pairs ? units2 : max_pairs;
       const unsigned grid = static_cast<unsigned>(2 * pairs2);
-      if (P.causal)
-        score_colsum_kernel<true><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, nlse2, gsum, err);
-      else
-        score_colsum_kernel<false><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, P, nlse2, gsum, err);
+      const float *nl = nlse2;
+      const cudaError_t e = P.causal ? launch_pdl(score_colsum_kernel<true>, dim3(grid), dim3(kThreads), kSmemBytes,
+                                                  stream, qmap, kmap, P, nl, gsum, err)
+                                     : launch_pdl(score_colsum_kernel<false>, dim3(grid), dim3(kThreads), kSmemBytes,
+                                                  stream, qmap, kmap, P, nl, gsum, err);
       count_launches(1);
-      if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
+      if (check_cuda(e) != APACK_OK) return APACK_ECUDA;
     }
     const int64_t t_begin = P.seq[0].t0;
     const int64_t n_tok = static_cast<int64_t>(P.seq[ns - 1].t0) + P.seq[ns - 1].len - t_begin;
     if (n_tok > 0) {
-      score_finalize_kernel<<<static_cast<unsigned>((n_tok + 255) / 256), 256, 0, stream>>>(P, seqs->modality, gsum,
-                                                                                            scores, t_begin, n_tok);
+      const float *gs = gsum;
+      if (check_cuda(launch_pdl(score_finalize_kernel, dim3(static_cast<unsigned>((n_tok + 255) / 256)), dim3(256), 0,
+                                stream, P, static_cast<const uint8_t *>(seqs->modality), gs, scores, t_begin,
+                                n_tok)) != APACK_OK)
+        return APACK_ECUDA;
       count_launches(1);
-      if (check_cuda(cudaGetLastError()) != APACK_OK) return APACK_ECUDA;
     }
     qp_base += qrows;
   }
