@@ -124,3 +124,53 @@ def test_random_prune_step_matches_oracle(ap, seed):
         np.testing.assert_array_equal(ko[li, :n_out].cpu().numpy(), oracle.compact_rows(kn[li], got_keep))
         np.testing.assert_array_equal(vo[li, :n_out].cpu().numpy(), oracle.compact_rows(vn[li], got_keep))
     np.testing.assert_array_equal(ho[:n_out].cpu().numpy(), oracle.compact_rows(hn, got_keep))
+
+
+def draw_keep(rng, T, n_keep):
+    """Strictly increasing kept rows of one of four shapes (uniform, kept prefix, kept tail, runs)."""
+    kind = int(rng.integers(4))
+    if kind == 0 or n_keep in (0, T):
+        return np.sort(rng.choice(T, n_keep, replace=False))
+    if kind == 1:      # a prefix that stays in place, then a uniform choice
+        head = int(rng.integers(0, n_keep + 1))
+        rest = np.sort(rng.choice(np.arange(head, T), n_keep - head, replace=False))
+        return np.concatenate([np.arange(head), rest])
+    if kind == 2:      # a uniform choice, then the whole tail
+        tail = int(rng.integers(0, n_keep + 1))
+        head = np.sort(rng.choice(T - tail, n_keep - tail, replace=False))
+        return np.concatenate([head, np.arange(T - tail, T)])
+    starts = np.sort(rng.choice(T, min(T, max(1, n_keep // 37)), replace=False))   # runs of kept rows
+    keep = np.unique(np.concatenate([np.arange(s, min(T, s + 64)) for s in starts]))
+    if keep.size >= n_keep:
+        return np.sort(rng.choice(keep, n_keep, replace=False))
+    extra = rng.choice(np.setdiff1d(np.arange(T), keep), n_keep - keep.size, replace=False)
+    return np.sort(np.concatenate([keep, extra]))
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_random_in_place_compaction_matches_oracle(ap, seed):
+    """apack_compact with src == dst on random keep lists of every density (the wave schedule for
+    low keep ratios, the per-item one near 1), one to three groups of various row sizes."""
+    rng = np.random.default_rng(5000 + seed)
+    T = int(rng.integers(1, 40000))
+    n_keep = int(rng.integers(0, T + 1)) if rng.random() < 0.8 else int(T * rng.uniform(0.8, 1.0))
+    keep = draw_keep(rng, T, n_keep).astype(np.int32)
+    assert keep.size == n_keep
+    shapes = [(int(rng.integers(1, 4)), int(rng.choice([16, 256, 1024, 2048, 7168])))
+              for _ in range(int(rng.integers(1, 4)))]
+    while T * sum(pl * rb for pl, rb in shapes) > 400_000_000:      # a few hundred MB per case
+        shapes = shapes[:-1] if len(shapes) > 1 else [(1, shapes[0][1])]
+    srcs = [rng.integers(0, 256, (pl, T, rb), dtype=np.uint8) for pl, rb in shapes]
+    bufs = [dev(s) for s in srcs]
+    ws = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+    groups = [ap.make_plane(b, b, rb, pl, src_plane_stride=T * rb, dst_plane_stride=T * rb)
+              for b, (pl, rb) in zip(bufs, shapes)]
+    if n_keep:
+        ap.apack_compact(dev(keep), n_keep, groups, ws=ws)
+    torch.cuda.synchronize()
+    assert ap.apack_device_error(ws) == ap.APACK_OK
+    for b, s in zip(bufs, srcs):
+        got = b.cpu().numpy()
+        for pl in range(s.shape[0]):
+            np.testing.assert_array_equal(got[pl, :n_keep], oracle.compact_rows(s[pl], keep))
+            np.testing.assert_array_equal(got[pl, n_keep:], s[pl, n_keep:])
