@@ -1095,13 +1095,17 @@ def main():
     # (ProgressivePrune.host_step): each step scores and selects on the device and gathers over
     # the host link, at the composed indices, only the layers that end at its level (and the keys
     # the next step scores), so every layer's rows cross the link once.  The result (the last
-    # step's layers, the hidden states, the indices) is read back.  Two device buffer sets let
+    # step's layers, the hidden states, the indices) is read back.  Three device buffer sets let
     # iteration i+1's upload and first selection run while iteration i's gathers hold the link,
-    # and iteration i-1's result is read back on a third stream: the link carries both directions.
+    # and iteration i-1's result is read back on a third stream (the link carries both
+    # directions) without holding up iteration i+2's upload: with two sets, the gather queue
+    # stood idle while one iteration's read-back, the next upload and its first selection ran.
+    # Each step waits only for its own schedule's previous gather (not for gathers of the next
+    # iteration queued meanwhile), so its scoring overlaps them.
     e2e_steps = args.e2e_steps or max(3, min(args.steps, 20))
-    pp2 = ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
-                           wl.prune_layers, counts, select_mode=mode)
-    sets = [pp, pp2]
+    pp2, pp3 = (ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
+                                 wl.prune_layers, counts, select_mode=mode) for _ in range(2))
+    sets = [pp, pp2, pp3]
     h_k = torch.empty(pp.k_in.shape, dtype=pp.k_in.dtype, pin_memory=True)
     h_v = torch.empty_like(h_k, pin_memory=True)
     h_h = torch.empty(pp.hidden_in.shape, dtype=pp.hidden_in.dtype, pin_memory=True)
@@ -1147,7 +1151,7 @@ def main():
 
     def front(j):
         """Upload, score, select and start the host-source compaction of iteration j."""
-        b = j % 2
+        b = j % len(sets)
         p = sets[b]
         with torch.cuda.stream(s_up):          # upload once the set's last result was read back
             s_up.wait_event(ev_down[b])
@@ -1161,7 +1165,7 @@ def main():
 
     def back(j):
         """The later steps and the read-back of iteration j."""
-        b = j % 2
+        b = j % len(sets)
         p = sets[b]
         for i in range(1, nsteps):
             p.host_step(i, h_k, h_v, h_h, stream=stream, gather_stream=s_gather)
@@ -1185,7 +1189,7 @@ def main():
                 front(j + 1)
             back(j)
 
-    e2e_run(2)
+    e2e_run(len(sets))
     torch.cuda.synchronize()
     barrier()
     if clocks:
@@ -1204,7 +1208,7 @@ def main():
     link = link_rates(h_k, h_v, pp2, s_up, s_down)
     stream_dev.wait_stream(stream)
     stream = stream_dev
-    del pp2, sets
+    del pp2, pp3, sets
 
     # the paper's own setting (last query token, joint top-k, 14 steps), when the headline is the
     # workloads' schedule
@@ -1268,7 +1272,7 @@ def main():
                                 "the layers that end at its level plus the keys the next step scores, so each "
                                 "layer's rows cross the link once; the result is every layer's final cache on the "
                                 "device, of which the last step's layers, the hidden states and the indices are read "
-                                "back; two device buffer sets let the next iteration's upload and first selection "
+                                "back; three device buffer sets let the next iteration's upload and first selection "
                                 "and the previous read-back run while the current gathers hold the link",
                     "h2d_note": "h2d_bytes_per_step counts the copies and the kept rows read from host memory",
                     "h2d_gbs": h2d / (e2e_ms / 1e3) / 1e9, "link": link,

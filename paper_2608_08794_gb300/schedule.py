@@ -248,6 +248,7 @@ class ProgressivePrune:
         self.k_score = [None] + [torch.empty((max(1, self.t_out[i - 1]), self.hkv, APACK_HEAD_DIM),
                                              dtype=torch.bfloat16, device=self.dev) for i in range(1, n)]
         self.comp = [None] + [torch.empty(max(1, t), dtype=torch.int32, device=self.dev) for t in self.t_out[1:]]
+        self.gather_done = [torch.cuda.Event() for _ in range(n)]
 
     def run_from_host(self, k_host, v_host, hidden_host=None, stream=None, gather_stream=None):
         """The whole schedule with the K/V caches of layers [l_0, L) and the hidden states in pinned
@@ -281,7 +282,9 @@ class ProgressivePrune:
         t = self.t_out[i]
         k_sc = self.k_in.view(-1) if i == 0 else self.k_score[i]
         if i > 0 and gs is not stream:
-            _wait(stream, gs)                  # the scored keys came over the link
+            # the scored keys (and at step 1 the step-0 hidden rows) came over the link in step
+            # i-1's gather; later gathers queued on gs meanwhile (another schedule's) need not end
+            (stream or torch.cuda.current_stream()).wait_event(self.gather_done[i - 1])
         apack_score(seqs, self.q[i], k_sc, row, self.scores, self.ws, stream=stream)
         apack_select(seqs, self.scores, self.counts[i], self.keep_idx[i], self.ws, select_mode=self.mode,
                      modality_out=self.mod_out[i % 2], stream=stream)
@@ -306,12 +309,12 @@ class ProgressivePrune:
         if gs is not stream:
             _wait(gs, stream)
         apack_compact(comp, t, planes, ws=self.ws, stream=gs)
+        if gs is not stream:
+            self.gather_done[i].record(gs)
         if i > 0:                              # device-side: the scored keys and the hidden states
             dev_planes = [_plane(self.k_score[i].data_ptr(), kf, 0, 0, row, 1)]
             h_prev, h_new = self.h_out[(i - 1) % 2], self.h_out[i % 2]
             if h_prev is not None and hidden_host is not None:
-                if i == 1 and gs is not stream:
-                    _wait(stream, gs)          # the step-0 hidden rows came over the link
                 dev_planes.append(make_plane(h_prev, h_new, self.H * 2, 1))
             apack_compact(self.keep_idx[i], t, dev_planes, ws=self.ws, stream=stream)
         k = self.counts[i]
@@ -319,7 +322,7 @@ class ProgressivePrune:
         cu[1:] = np.cumsum(other + k[:, 0] + k[:, 1])
         self.new_cu[i] = cu
         if i + 1 == n and gs is not stream:
-            _wait(stream, gs)
+            (stream or torch.cuda.current_stream()).wait_event(self.gather_done[i])
 
     def final_kv(self, i):
         """run_from_host's caches of layers [l_i, l_(i+1)) (the last step: [l_i, L)) at their final
