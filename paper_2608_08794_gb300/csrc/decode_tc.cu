@@ -3,7 +3,8 @@
 //
 //   out[b, h] = sum_j softmax_j(q[b, h] . k[j, g(h)] / sqrt(128)) v[j, g(h)]
 //
-// One CTA per chunk of a sequence's keys (whole 128-key tiles), all KV heads.  A stage is one
+// One CTA per chunk of a sequence's keys, all KV heads; the sequence's 128-key tiles are dealt
+// round-robin over its chunks (CTA c of n takes tiles c, c + n, c + 2n, ...).  A stage is one
 // KV head of one tile; its K rows and its V rows (TMA boxes of 64 features x 1 head x 128 keys,
 // 128-byte swizzle, 32 KB each) are separate items of a 6-slot shared-memory ring, loaded in
 // the order K0 K1 V0 K2 V1 K3 V2 ...: the keys of a stage arrive one stage ahead of its values,
@@ -137,9 +138,10 @@ __global__ void __launch_bounds__(kDThreads, 1)
   const DecSeq &sq = plan.seq[s];
   const int G = plan.group;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tb = (c - sq.chunk_begin) * plan.chunk;
-  const int te = min(sq.len, tb + plan.chunk);
-  const int ntiles = (te - tb + kDM - 1) / kDM;
+  // this CTA's tiles: lc, lc + nch, lc + 2 nch, ... of the sequence's 128-key tiles (lc < nch <=
+  // the tile count, so every CTA has one at least)
+  const int lc = c - sq.chunk_begin, nch = sq.nchunks;
+  const int ntiles = ((sq.len + kDM - 1) / kDM - lc + nch - 1) / nch;
   const int nstage = ntiles * HKV;
 
   // query tiles: rows j < G of head group h, 128-byte swizzled K-major layout
@@ -204,7 +206,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
         uint8_t *dst = ring + slot * kDSlotBytes;
         const CUtensorMap *map = is_v ? &vmap : &kmap;
         mbar_arrive_expect_tx(&bars->full[slot], kDSlotBytes);
-        const int key0 = sq.t0 + tb + t * kDM;
+        const int key0 = sq.t0 + (lc + t * nch) * kDM;
         tma_load_3d(dst, map, &bars->full[slot], 0, h, key0);
         tma_load_3d(dst + kDHalf, map, &bars->full[slot], 64, h, key0);
         pend[slot] = true;
@@ -281,8 +283,8 @@ __global__ void __launch_bounds__(kDThreads, 1)
         bool ok = __all_sync(0xffffffffu, d_wait(&bars->s_full[buf], (n >> 1) & 1u, bars, err, 95));
         if (ok && t >= 1)   // the head's previous O^T MMAs are done: its P tile and O^T are free
           ok = __all_sync(0xffffffffu, d_wait(&bars->p_empty[h], (t - 1) & 1u, bars, err, 96));
-        const int key = tb + t * kDM + kt;
-        const bool valid = key < te;
+        const int key = (lc + t * nch) * kDM + kt;
+        const bool valid = key < sq.len;
         const float *m_old = msm + ((t & 1) ^ 1) * HKV * kDRows + h * kDRows;
         float *m_new = msm + (t & 1) * HKV * kDRows + h * kDRows;
         float x[kDRows], m[kDRows];
