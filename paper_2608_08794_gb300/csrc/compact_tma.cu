@@ -23,6 +23,7 @@ __global__ void __launch_bounds__(32) gather_tma_kernel(const __grid_constant__ 
                                                         const int32_t *__restrict__ keep_idx, DeviceError *err) {
   extern __shared__ __align__(1024) uint8_t slots[];
   __shared__ __align__(8) uint64_t full[kSlots];
+  pdl_wait_and_release();   // keep_idx and the source rows are complete; the next launch may be scheduled
   const int lane = threadIdx.x;
   if (lane == 0) {
     for (int i = 0; i < kSlots; ++i) mbar_init(&full[i], 1);
@@ -74,9 +75,10 @@ apack_status launch_out_of_place(const TmaPlan &tp, const int32_t *keep_idx, Dev
     return APACK_ECUDA;
   uint64_t blocks = static_cast<uint64_t>(device_sm_count()) * kCtasPerSm;
   if (blocks > tp.total_items) blocks = tp.total_items;
-  gather_tma_kernel<<<static_cast<unsigned>(blocks), 32, kTmaSmem, stream>>>(tp, keep_idx, err);
+  const cudaError_t e = launch_pdl(gather_tma_kernel, dim3(static_cast<unsigned>(blocks)), dim3(32), kTmaSmem, stream,
+                                   tp, keep_idx, err);
   count_launches(1);
-  return check_cuda(cudaGetLastError());
+  return check_cuda(e);
 }
 
 }  // namespace gather

@@ -144,17 +144,6 @@ __global__ void __launch_bounds__(kDThreads, 1)
   const int ntiles = ((sq.len + kDM - 1) / kDM - lc + nch - 1) / nch;
   const int nstage = ntiles * HKV;
 
-  // query tiles: rows j < G of head group h, 128-byte swizzled K-major layout
-  for (int idx = threadIdx.x; idx < HKV * kDN * 16; idx += kDThreads) {
-    const int h = idx / (kDN * 16), rem = idx % (kDN * 16);
-    const int row = rem / 16, ch = rem % 16;
-    const int half = ch >> 3, cc = ch & 7;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (row < G)
-      v = __ldg(reinterpret_cast<const uint4 *>(q + (static_cast<int64_t>(s) * plan.hq + h * G + row) * 128) + ch);
-    *reinterpret_cast<uint4 *>(qs + h * 2 * kDQHalf + half * kDQHalf + (row >> 3) * 1024 + (row & 7) * 128 +
-                               ((cc ^ (row & 7)) << 4)) = v;
-  }
   if (threadIdx.x == 0) {
     for (int i = 0; i < kDSlots; ++i) {
       mbar_init(&bars->full[i], 1);
@@ -174,11 +163,26 @@ __global__ void __launch_bounds__(kDThreads, 1)
     for (int i = 0; i < 2 * HKV * kDRows; ++i) msm[i] = -INFINITY;
     fence_mbar_init();
   }
-  fence_proxy_async_smem();
   if (warp == 1) {
     tmem_alloc(&bars->tmem_base, kDTmemCols);
     tc_fence_before();
   }
+  // Launched as a programmatic dependent: the set-up above runs beside the previous launch on
+  // the stream; q, the cache and the partials (which the previous call's combine reads) are
+  // touched only once that launch has completed.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // query tiles: rows j < G of head group h, 128-byte swizzled K-major layout
+  for (int idx = threadIdx.x; idx < HKV * kDN * 16; idx += kDThreads) {
+    const int h = idx / (kDN * 16), rem = idx % (kDN * 16);
+    const int row = rem / 16, ch = rem % 16;
+    const int half = ch >> 3, cc = ch & 7;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (row < G)
+      v = __ldg(reinterpret_cast<const uint4 *>(q + (static_cast<int64_t>(s) * plan.hq + h * G + row) * 128) + ch);
+    *reinterpret_cast<uint4 *>(qs + h * 2 * kDQHalf + half * kDQHalf + (row >> 3) * 1024 + (row & 7) * 128 +
+                               ((cc ^ (row & 7)) << 4)) = v;
+  }
+  fence_proxy_async_smem();
   __syncthreads();
   tc_fence_after();
 
@@ -442,7 +446,8 @@ cudaError_t launch_decode_tc(int grid, cudaStream_t stream, const CUtensorMap &k
                                   static_cast<int>(DLay<4>::kBytes));
     });
     if (e != cudaSuccess) return e;
-    decode_tc_kernel<4><<<grid, kDThreads, DLay<4>::kBytes, stream>>>(kmap, vmap, P, q, opart, mlpart, err);
+    return launch_pdl(decode_tc_kernel<4>, dim3(grid), dim3(kDThreads), DLay<4>::kBytes, stream, kmap, vmap, P, q,
+                      opart, mlpart, err);
   } else {
     static std::atomic<uint64_t> attr{0};
     const cudaError_t e = once_per_device(attr, [] {
@@ -450,9 +455,9 @@ cudaError_t launch_decode_tc(int grid, cudaStream_t stream, const CUtensorMap &k
                                   static_cast<int>(DLay<2>::kBytes));
     });
     if (e != cudaSuccess) return e;
-    decode_tc_kernel<2><<<grid, kDThreads, DLay<2>::kBytes, stream>>>(kmap, vmap, P, q, opart, mlpart, err);
+    return launch_pdl(decode_tc_kernel<2>, dim3(grid), dim3(kDThreads), DLay<2>::kBytes, stream, kmap, vmap, P, q,
+                      opart, mlpart, err);
   }
-  return cudaGetLastError();
 }
 
 }  // namespace apack

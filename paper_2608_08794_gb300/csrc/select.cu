@@ -111,6 +111,7 @@ __global__ void __cluster_dims__(CL, 1, 1) __launch_bounds__(kThreads)
   __shared__ uint32_t cnt[5];                 // per CTA (read by the cluster)
   __shared__ uint32_t wbase[kWarps], weqb[kWarps][2];
   extern __shared__ __align__(16) uint8_t cache_raw[];
+  pdl_wait_and_release();                     // the scores are complete; the compaction may be scheduled
 
   const SelSeq &sq = plan.seq[blockIdx.y];
   const uint32_t crank = cluster_ctarank();
@@ -359,9 +360,8 @@ template <int CL>
 cudaError_t launch_select(const SelectPlan &P, int ns, size_t smem, const float *scores, const uint8_t *modality,
                           int32_t *keep_idx, uint8_t *modality_out, int32_t *dst_of_src, int32_t *new_cu,
                           DeviceError *err, cudaStream_t stream) {
-  select_kernel<CL><<<dim3(CL, ns, 1), kThreads, smem, stream>>>(P, scores, modality, keep_idx, modality_out,
-                                                                   dst_of_src, new_cu, err);
-  return cudaGetLastError();
+  return launch_pdl(select_kernel<CL>, dim3(CL, ns, 1), dim3(kThreads), smem, stream, P, scores, modality, keep_idx,
+                    modality_out, dst_of_src, new_cu, err);
 }
 
 // Cluster size per sequence: 8 CTAs, or 16 for sequences longer than kWideFrom tokens where such
