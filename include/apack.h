@@ -321,13 +321,18 @@ apack_status apack_graph_destroy(apack_graph graph);
    a multiple of 16, >= Hkv*256); out: fp32 [num_seqs][Hq][128] (16-byte
    aligned, device).  cu_seqlens_h: host [num_seqs+1], starting at 0; an
    empty sequence gives zeros.  Supported: Hq / Hkv <= 8 and Hkv in
-   {1, 2, 4, 8} (APACK_EUNSUPPORTED otherwise).  fp32 accumulation, fixed
-   merge order (deterministic).  ws: 256-byte aligned,
-   apack_decode_workspace_size bytes (the size depends on the device's SM
-   count: query it on the device that runs the call); its first 16 bytes are
-   a device error word read by apack_device_error, zeroed by the caller once.
-   A device-side wait that runs out records APACK_ETIMEOUT there.  Two kernel
-   launches per 64 sequences; no allocation, no synchronisation. */
+   {1, 2, 4, 8} (APACK_EUNSUPPORTED otherwise).  fp32 accumulation.  With
+   Hkv 2 or 4 and at most 8 query heads per KV head (the tensor-core path) the
+   CTAs of a sequence claim its 128-key tiles from a counter as they go, so
+   the grouping of keys into partial sums, and with it the last bits of out,
+   can differ from call to call; the other head layouts merge in a fixed
+   order.  ws: 256-byte aligned, apack_decode_workspace_size bytes (the size
+   depends on the device's SM count: query it on the device that runs the
+   call), zeroed by the caller once before its first use: its first 16 bytes
+   are a device error word read by apack_device_error, and it holds the
+   claim counters, which every call leaves at zero.  A device-side wait that
+   runs out records APACK_ETIMEOUT there.  Two kernel launches per 64
+   sequences; no allocation, no synchronisation. */
 apack_status apack_decode_workspace_size(int32_t num_seqs, const int32_t *cu_seqlens_h, int32_t num_q_heads,
                                          int32_t num_kv_heads, size_t *bytes);
 apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_h, const void *q, const void *k,

@@ -281,14 +281,17 @@ __global__ void __launch_bounds__(kDecThreads, 1)
 
 // One CTA per (sequence, query head): merge the sequence's chunks.  Warp w folds chunks
 // w, w + 16, w + 32, ... in that order (lane: features [4 lane, 4 lane + 4)); the warps
-// then merge in warp order.  A sequence with no cached token gets zeros.
+// then merge in warp order.  A sequence with no cached token gets zeros.  The CTA of query
+// head 0 also zeroes the sequence's stage-claim counter for the next call (the chunk kernel,
+// the counter's only user, is complete here).
 __global__ void __launch_bounds__(kDecCombineThreads)
     decode_combine_kernel(const __grid_constant__ DecPlan plan, const float *__restrict__ opart,
-                          const float2 *__restrict__ mlpart, float *__restrict__ out) {
+                          const float2 *__restrict__ mlpart, float *__restrict__ out, unsigned int *claims) {
   __shared__ __align__(16) float wo[kDecCombineWarps][128];
   __shared__ float2 wml[kDecCombineWarps];
   pdl_wait_and_release();                   // the chunk kernel's partials are complete and visible
   const int s = blockIdx.x / plan.hq, hh = blockIdx.x % plan.hq;
+  if (hh == 0 && threadIdx.x == 0) claims[s] = 0u;
   const DecSeq &sq = plan.seq[s];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   float m = -INFINITY, l = 0.f, o[4] = {0.f, 0.f, 0.f, 0.f};
@@ -371,9 +374,11 @@ apack_status apack_decode_workspace_size(int32_t num_seqs, const int32_t *cu_seq
   const int chunk = decode_chunk_keys(total, num_kv_heads);
   int64_t chunks = 0;
   for (int b = 0; b < num_seqs; ++b) chunks += (cu_seqlens_h[b + 1] - cu_seqlens_h[b] + chunk - 1) / chunk;
-  // device error word, chunk partials o [chunks][Hq][128] and (max, sum) [chunks][Hq]
+  // device error word, chunk partials o [chunks][Hq][128] and (max, sum) [chunks][Hq], one
+  // stage-claim counter per sequence
   *bytes = 256 + up256(static_cast<size_t>(chunks) * num_q_heads * 128 * sizeof(float)) +
-           up256(static_cast<size_t>(chunks) * num_q_heads * sizeof(float2));
+           up256(static_cast<size_t>(chunks) * num_q_heads * sizeof(float2)) +
+           up256(static_cast<size_t>(num_seqs) * sizeof(unsigned int));
   return APACK_OK;
 }
 
@@ -401,6 +406,8 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
   float *opart = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + 256);
   float2 *mlpart = reinterpret_cast<float2 *>(static_cast<uint8_t *>(ws) + 256 +
                                               up256(static_cast<size_t>(chunks_all) * num_q_heads * 128 * sizeof(float)));
+  unsigned int *claims = reinterpret_cast<unsigned int *>(
+      reinterpret_cast<uint8_t *>(mlpart) + up256(static_cast<size_t>(chunks_all) * num_q_heads * sizeof(float2)));
   static std::atomic<uint64_t> attr_done{0};
   if (once_per_device(attr_done, [] {
         return cudaFuncSetAttribute(decode_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -439,7 +446,8 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
     const uint16_t *qs = q16 + static_cast<int64_t>(s0) * num_q_heads * 128;
     if (chunks > 0) {
       if (tc) {
-        if (check_cuda(launch_decode_tc(chunks, s, kmap, vmap, P, qs, op, mp, err)) != APACK_OK) return APACK_ECUDA;
+        if (check_cuda(launch_decode_tc(chunks, s, kmap, vmap, P, qs, op, mp, claims + s0, err)) != APACK_OK)
+          return APACK_ECUDA;
       } else {
         decode_chunk_kernel<<<chunks, kDecThreads, kDecSmem, s>>>(P, qs, static_cast<const uint8_t *>(k),
                                                                   static_cast<const uint8_t *>(v), kv_token_stride,
@@ -452,7 +460,7 @@ apack_status apack_decode_attention(int32_t num_seqs, const int32_t *cu_seqlens_
     // drains and wait (griddepcontrol.wait) for its completion before reading the partials
     if (check_cuda(launch_pdl(decode_combine_kernel, dim3(ns * num_q_heads), dim3(kDecCombineThreads), 0, s, P,
                               static_cast<const float *>(op), static_cast<const float2 *>(mp),
-                              out + static_cast<int64_t>(s0) * num_q_heads * 128)) != APACK_OK)
+                              out + static_cast<int64_t>(s0) * num_q_heads * 128, claims + s0)) != APACK_OK)
       return APACK_ECUDA;
     count_launches(1);
     chunk_base += chunks;

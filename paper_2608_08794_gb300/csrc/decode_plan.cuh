@@ -25,9 +25,12 @@ __device__ __forceinline__ int find_chunk_seq(const DecPlan &p, int c) {
   return s;
 }
 
-// Tensor-core chunk kernel (decode_tc.cu): Hkv = 2 or 4, at most 8 query heads per KV head,
-// P.chunk a multiple of 128.  Writes the same chunk partials as the CUDA-core kernel.
+// Tensor-core chunk kernel (decode_tc.cu): Hkv = 2 or 4, at most 8 query heads per KV head.
+// The CTAs of sequence i claim its 128-key stages from claims[i] (zero before the launch; the
+// combine kernel zeroes it again); each writes one partial per query head, in the layout of
+// the CUDA-core kernel's chunk partials.
 cudaError_t launch_decode_tc(int grid, cudaStream_t stream, const CUtensorMap &kmap, const CUtensorMap &vmap,
-                             const DecPlan &P, const uint16_t *q, float *opart, float2 *mlpart, DeviceError *err);
+                             const DecPlan &P, const uint16_t *q, float *opart, float2 *mlpart, unsigned int *claims,
+                             DeviceError *err);
 
 }  // namespace apack

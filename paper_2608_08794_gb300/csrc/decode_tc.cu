@@ -3,14 +3,20 @@
 //
 //   out[b, h] = sum_j softmax_j(q[b, h] . k[j, g(h)] / sqrt(128)) v[j, g(h)]
 //
-// One CTA per chunk of a sequence's keys, all KV heads; the sequence's 128-key tiles are dealt
-// round-robin over its chunks (CTA c of n takes tiles c, c + n, c + 2n, ...).  A stage is one
-// KV head of one tile; its K rows and its V rows (TMA boxes of 64 features x 1 head x 128 keys,
-// 128-byte swizzle, 32 KB each) are separate items of a 6-slot shared-memory ring, loaded in
-// the order K0 K1 V0 K2 V1 K3 V2 ...: the keys of a stage arrive one stage ahead of its values,
-// so its logits and probabilities are ready when V lands, and each item holds its slot only
-// until its own contraction is done (K: S, V: O^T).
-//   warp 0, one lane:  TMA loads of the items
+// About one CTA per SM (each sequence gets CTAs in proportion to its length), all KV heads.  A
+// stage is one KV head of one 128-key tile; the CTAs of a sequence claim its stages in order
+// from a counter in the workspace (tile-major, heads within a tile), so that CTAs on SMs that
+// stream faster take more of them and all finish together.  Each CTA folds every stage it
+// claims into its running per-head state, so it still writes one partial per query head;
+// which CTA takes which stage varies from call to call, and with it the last bits of the
+// result.  The combine kernel resets the counter for the next call.  A stage's K rows and V
+// rows (TMA boxes of 64 features x 1 head x 128 keys, 128-byte swizzle, 32 KB each) are
+// separate items of a 6-slot shared-memory ring, loaded in the order K0 K1 V0 K2 V1 K3 V2 ...:
+// the keys of a stage arrive one stage ahead of its values, so its logits and probabilities
+// are ready when V lands, and each item holds its slot only until its own contraction is done
+// (K: S, V: O^T).  The producer publishes each claimed stage (or the end of the claims) in a
+// small ring of stage records with their own barriers, which every other role reads in order.
+//   warp 0, one lane:  stage claims and TMA loads of the items
 //   warp 1, one lane:  TMEM allocation; S = K q^T of every stage: keys as M = 128, the head
 //                      group's <= 8 query rows (zero-padded) as N = 16; S[key][row] in TMEM
 //   warp 6, one lane:  O^T += V^T P^T of every stage: features as M = 128 (V read as an MN-major
@@ -23,7 +29,8 @@
 //                      tile's logits exceed it by more than 2^8 (then O^T's columns of that row
 //                      and the partial sums are rescaled once), p written as the bf16 pair into
 //                      the head's P tile; at the end they read O^T back (one feature per thread).
-// The result per query head is the chunk partial (m, l = sum p, o = sum p v) in log2 units,
+// The result per query head is the CTA's partial (m, l = sum p, o = sum p v) in log2 units
+// (m = -inf, l = 0, o = 0 for a head of which it claimed no stage),
 // merged by the combine kernel with the CUDA-core kernel's partials' rules.  hi + lo carries p
 // to about 2^-17 relative, so o matches fp32 arithmetic.  Every wait is bounded.
 #include <cmath>
@@ -52,10 +59,13 @@ constexpr float kDLazy = 8.f;                      // the reference maximum lags
 constexpr uint32_t kDIdescS = idesc_bf16_f32(kDM, kDN);
 constexpr uint32_t kDIdescO = idesc_bf16_f32(128, kDN) | (1u << 15);   // A (V^T) MN-major
 constexpr uint32_t kDTmemCols = 128;               // S [2][16] at 0, O^T of head h at 32 + 16 h
+constexpr int kDInfo = 8;                          // stage records in flight (the producer leads by <= 5)
 
 struct __align__(8) DBars {
   uint64_t full[kDSlots], empty[kDSlots], s_full[2], s_empty[2], drain[2];   // drain: per issuing warp
-  uint64_t p_full[4], p_empty[4];                  // one pair per KV head: their phases are its tiles
+  uint64_t p_full[4], p_empty[4];                  // one pair per KV head: their phases are its stages
+  uint64_t info_full[kDInfo];                      // stage record n % kDInfo written (phase n / kDInfo)
+  volatile int32_t info[kDInfo];                   // claimed unit (tile * HKV + head), or -1: no more
   uint32_t tmem_base;
   volatile int32_t abort;
 };
@@ -67,8 +77,9 @@ struct DLay {
   static constexpr uint32_t kOffT = kOffP + HKV * kDPBytes;                      // tile maxima [2][4][8]
   static constexpr uint32_t kOffM = kOffT + 2 * kDSoftWarps * kDRows * 4;        // reference max [2][HKV][8]
   static constexpr uint32_t kOffBars = (kOffM + 2 * HKV * kDRows * 4 + 7) & ~7u;
-  static constexpr uint32_t kBytes = kOffBars + 256;
+  static constexpr uint32_t kBytes = kOffBars + 512;
 };
+static_assert(sizeof(DBars) <= 512, "barrier block");
 
 __device__ __forceinline__ bool d_wait(uint64_t *bar, uint32_t parity, DBars *bars, DeviceError *err, int where) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -105,12 +116,12 @@ __device__ __forceinline__ uint32_t p_off(int row, int key) {
   return half * 2048 + (row >> 3) * 1024 + (row & 7) * 128 + ((ch ^ (row & 7)) << 4) + (key & 7) * 2;
 }
 
-// Load order of the ring's items: K0, K1, V0, K2, V1, ..., K(N-1), V(N-2), V(N-1) for N stages.
+// Load order of the ring's items: K0, K1, V0, K2, V1, K3, V2, ...  With N claimed stages the
+// position of K(N) carries no load (the end of the claims) and V(N-1) is the last item.
 __device__ __forceinline__ int item_of_k(int n) { return n == 0 ? 0 : 2 * n - 1; }
-__device__ __forceinline__ int item_of_v(int n, int N) { return n == N - 1 ? 2 * N - 1 : 2 * n + 2; }
-__device__ __forceinline__ void item_stage(int i, int N, bool *is_v, int *n) {
+__device__ __forceinline__ int item_of_v(int n) { return 2 * n + 2; }
+__device__ __forceinline__ void item_stage(int i, bool *is_v, int *n) {
   if (i == 0) { *is_v = false; *n = 0; }
-  else if (i == 2 * N - 1) { *is_v = true; *n = N - 1; }
   else if (i & 1) { *is_v = false; *n = (i + 1) >> 1; }
   else { *is_v = true; *n = (i >> 1) - 1; }
 }
@@ -119,7 +130,7 @@ template <int HKV>
 __global__ void __launch_bounds__(kDThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ DecPlan plan, const uint16_t *__restrict__ q, float *__restrict__ opart,
-                     float2 *__restrict__ mlpart, DeviceError *err) {
+                     float2 *__restrict__ mlpart, unsigned int *claims, DeviceError *err) {
   using Lay = DLay<HKV>;
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");   // the combine may be scheduled
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -138,11 +149,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
   const DecSeq &sq = plan.seq[s];
   const int G = plan.group;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // this CTA's tiles: lc, lc + nch, lc + 2 nch, ... of the sequence's 128-key tiles (lc < nch <=
-  // the tile count, so every CTA has one at least)
-  const int lc = c - sq.chunk_begin, nch = sq.nchunks;
-  const int ntiles = ((sq.len + kDM - 1) / kDM - lc + nch - 1) / nch;
-  const int nstage = ntiles * HKV;
+  const int units = (sq.len + kDM - 1) / kDM * HKV;   // the sequence's stages
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kDSlots; ++i) {
@@ -159,6 +166,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
     }
     mbar_init(&bars->drain[0], 1);
     mbar_init(&bars->drain[1], 1);
+    for (int i = 0; i < kDInfo; ++i) mbar_init(&bars->info_full[i], 1);
     bars->abort = 0;
     for (int i = 0; i < 2 * HKV * kDRows; ++i) msm[i] = -INFINITY;
     fence_mbar_init();
@@ -192,41 +200,88 @@ __global__ void __launch_bounds__(kDThreads, 1)
 #pragma unroll
     for (int j = 0; j < kDRows; ++j) l_run[h][j] = 0.f;
   bool stop = false;
+  uint32_t par = 0, seen = 0;                      // softmax threads, per KV head: stage-count parity, any stage
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+    // ------------------------------------------------------------ claims and TMA producer
     if (lane == 0) {
       tma_prefetch_desc(&kmap);
       tma_prefetch_desc(&vmap);
+      // claims run two stages ahead of the loads (an atomic's round trip is about a stage's
+      // time); one thread's claims on one counter return increasing units
+      unsigned int *claim = claims + s;
+      int next = static_cast<int>(atomicAdd(claim, 1u));   // stage 0's unit
+      int next2 = static_cast<int>(atomicAdd(claim, 1u));  // stage 1's
+      int unit[2] = {0, 0};                       // units of the last two claimed stages (by n & 1)
+      int n_end = -1;                             // the number of claimed stages, once known
+      int last = -1;                              // the last item issued with a load
       bool pend[kDSlots] = {};
       uint32_t pend_par[kDSlots] = {};
-      for (int i = 0; i < 2 * nstage; ++i) {
-        const int slot = i % kDSlots;
-        if (i >= kDSlots && !d_wait(&bars->empty[slot], ((i / kDSlots) - 1) & 1u, bars, err, 91)) break;
+      for (int i = 0;; ++i) {
         bool is_v;
         int n;
-        item_stage(i, nstage, &is_v, &n);
-        const int t = n / HKV, h = n % HKV;
+        item_stage(i, &is_v, &n);
+        if (n_end >= 0 && (!is_v || n >= n_end)) break;
+        const int slot = i % kDSlots;
+        if (!is_v) {
+          // publish stage n's record (its unit, or the end of the claims) before its K load
+          const int u = next;
+          const int r = n % kDInfo;
+          if (u >= units) {
+            bars->info[r] = -1;
+            mbar_arrive(&bars->info_full[r]);
+            n_end = n;
+            continue;                              // no load: V(n - 1) is the last item
+          }
+          next = next2;
+          next2 = static_cast<int>(atomicAdd(claim, 1u));  // stage n + 2's unit
+          unit[n & 1] = u;
+          bars->info[r] = u;
+          mbar_arrive(&bars->info_full[r]);
+        }
+        if (i >= kDSlots && !d_wait(&bars->empty[slot], ((i / kDSlots) - 1) & 1u, bars, err, 91)) break;
+        const int u = unit[n & 1];
+        const int t = u / HKV, h = u % HKV;
         uint8_t *dst = ring + slot * kDSlotBytes;
         const CUtensorMap *map = is_v ? &vmap : &kmap;
         mbar_arrive_expect_tx(&bars->full[slot], kDSlotBytes);
-        const int key0 = sq.t0 + (lc + t * nch) * kDM;
+        const int key0 = sq.t0 + t * kDM;
         tma_load_3d(dst, map, &bars->full[slot], 0, h, key0);
         tma_load_3d(dst + kDHalf, map, &bars->full[slot], 64, h, key0);
         pend[slot] = true;
         pend_par[slot] = (i / kDSlots) & 1u;
+        last = i;
       }
-      if (bars->abort)
+      if (bars->abort) {
         for (int i = 0; i < kDSlots; ++i)
           if (pend[i]) mbar_wait(&bars->full[i], pend_par[i], kWaitLimitNs / 4);
+      } else {
+        // every loaded item's slot is released by a commit after its MMAs; the last loaded item
+        // of each slot is awaited here (earlier ones were, before their slots were reloaded), so
+        // that no commit arrives after the CTA has left.  The end marker loads nothing and no
+        // item after it shares its slot; the kDSlots + 2 latest positions cover every slot.
+        const int k_end = n_end >= 0 ? item_of_k(n_end) : -1;
+        uint32_t waited = 0;
+        for (int k = last; k >= 0 && k >= last - kDSlots - 1; --k) {
+          const int sl = k % kDSlots;
+          if (k == k_end || ((waited >> sl) & 1u)) continue;
+          waited |= 1u << sl;
+          d_wait(&bars->empty[sl], (k / kDSlots) & 1u, bars, err, 89);
+        }
+      }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ S issuer
     if (lane == 0) {
       const uint32_t tmem = bars->tmem_base;
       const uint32_t q_base = smem_u32(qs);
-      for (int n = 0; n < nstage; ++n) {
-        const int item = item_of_k(n), slot = item % kDSlots, buf = n & 1, h = n % HKV;
+      bool issued = false;
+      for (int n = 0;; ++n) {
+        const int r = n % kDInfo;
+        if (!d_wait(&bars->info_full[r], (n / kDInfo) & 1u, bars, err, 99)) break;
+        const int u = bars->info[r];
+        if (u < 0) break;
+        const int item = item_of_k(n), slot = item % kDSlots, buf = n & 1, h = u % HKV;
         if (n >= 2 && !d_wait(&bars->s_empty[buf], ((n >> 1) - 1) & 1u, bars, err, 92)) break;
         if (!d_wait(&bars->full[slot], (item / kDSlots) & 1u, bars, err, 93)) break;
         tc_fence_after();
@@ -241,35 +296,48 @@ __global__ void __launch_bounds__(kDThreads, 1)
                       kk > 0 ? 1u : 0u);
         }
         tc_commit(&bars->s_full[buf]);
-        if (item + kDSlots < 2 * nstage) tc_commit(&bars->empty[slot]);   // K is free once S is done
+        tc_commit(&bars->empty[slot]);              // K is free once S is done
+        issued = true;
       }
-      tc_commit(&bars->drain[0]);                   // every MMA of this thread done before teardown
-      mbar_wait(&bars->drain[0], 0, kWaitLimitNs / 4);
+      if (issued) {                                 // every MMA of this thread done before teardown
+        tc_commit(&bars->drain[0]);
+        mbar_wait(&bars->drain[0], 0, kWaitLimitNs / 4);
+      }
     }
   } else if (warp == kDPvWarp) {
     // ------------------------------------------------------------ O^T issuer
     if (lane == 0) {
       const uint32_t tmem = bars->tmem_base;
       const uint32_t p_base = smem_u32(ps);
-      for (int n = 0; n < nstage; ++n) {
-        const int item = item_of_v(n, nstage), slot = item % kDSlots, t = n / HKV, h = n % HKV;
-        if (!d_wait(&bars->p_full[h], t & 1u, bars, err, 94)) break;
+      uint32_t opar = 0, oseen = 0;                 // per KV head: stage-count parity, any stage
+      for (int n = 0;; ++n) {
+        const int r = n % kDInfo;
+        if (!d_wait(&bars->info_full[r], (n / kDInfo) & 1u, bars, err, 99)) break;
+        const int u = bars->info[r];
+        if (u < 0) break;
+        const int item = item_of_v(n), slot = item % kDSlots, h = u % HKV;
+        if (!d_wait(&bars->p_full[h], (opar >> h) & 1u, bars, err, 94)) break;
         if (!d_wait(&bars->full[slot], (item / kDSlots) & 1u, bars, err, 98)) break;
         tc_fence_after();
         // O^T[feature][col] += sum_key V[key][feature] P^T[col][key]: 16 keys per MMA
         const uint32_t v_base = smem_u32(ring + slot * kDSlotBytes);
         const uint32_t b_base = p_base + h * kDPBytes;
+        const bool acc = (oseen >> h) & 1u;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t bo = (kk >> 2) * (kDPBytes / 2) + (kk & 3) * 32;
           tc_mma_bf16(tmem + 32 + h * kDN, smem_desc_sw128_mn(v_base + kk * 2048, kDHalf, 1024),
-                      smem_desc_sw128(b_base + bo), kDIdescO, (t > 0 || kk > 0) ? 1u : 0u);
+                      smem_desc_sw128(b_base + bo), kDIdescO, (acc || kk > 0) ? 1u : 0u);
         }
         tc_commit(&bars->p_empty[h]);
-        if (item + kDSlots < 2 * nstage) tc_commit(&bars->empty[slot]);   // only slots that are reloaded
+        tc_commit(&bars->empty[slot]);
+        opar ^= 1u << h;
+        oseen |= 1u << h;
       }
-      tc_commit(&bars->drain[1]);
-      mbar_wait(&bars->drain[1], 0, kWaitLimitNs / 4);
+      if (oseen) {
+        tc_commit(&bars->drain[1]);
+        mbar_wait(&bars->drain[1], 0, kWaitLimitNs / 4);
+      }
     }
   } else {
     // ------------------------------------------------------------ softmax, one key per thread (warps 2..5)
@@ -279,115 +347,138 @@ __global__ void __launch_bounds__(kDThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const float c2 = plan.scale2;
     const bool odd = lane & 1;
-    for (int t = 0; t < ntiles && !stop; ++t) {
-#pragma unroll
-      for (int h = 0; h < HKV; ++h) {         // compile-time head: the partial sums stay in registers
-        const int n = t * HKV + h, buf = n & 1;
-        // every wait of the stage comes first; the group leaves only together, at a barrier
-        bool ok = __all_sync(0xffffffffu, d_wait(&bars->s_full[buf], (n >> 1) & 1u, bars, err, 95));
-        if (ok && t >= 1)   // the head's previous O^T MMAs are done: its P tile and O^T are free
-          ok = __all_sync(0xffffffffu, d_wait(&bars->p_empty[h], (t - 1) & 1u, bars, err, 96));
-        const int key = (lc + t * nch) * kDM + kt;
-        const bool valid = key < sq.len;
-        const float *m_old = msm + ((t & 1) ^ 1) * HKV * kDRows + h * kDRows;
-        float *m_new = msm + (t & 1) * HKV * kDRows + h * kDRows;
-        float x[kDRows], m[kDRows];
-        bool raise = false;
-#pragma unroll
-        for (int j = 0; j < kDRows; ++j) x[j] = -INFINITY;
-        if (ok) {
-          tc_fence_after();
-          uint32_t r[8];
-          tmem_ld8_wait(bars->tmem_base + lane_off + buf * kDN, r);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->s_empty[buf]);
-#pragma unroll
-          for (int j = 0; j < kDRows; ++j) {
-            x[j] = (valid && j < G) ? __uint_as_float(r[j]) * c2 : -INFINITY;
-            m[j] = m_old[j];
-            raise |= x[j] > m[j] + kDLazy;           // also every finite logit against -inf
-          }
-        }
-        const bool bad = !ok || bars->abort;
-        if (bar_red_or(1, kDSoftWarps * 32, bad || raise)) {
-          // slow path (the first tile, a new maximum, or an abort): the tile's row maxima
-          float *tm = tmax + buf * kDSoftWarps * kDRows;
-#pragma unroll
-          for (int j = 0; j < kDRows; ++j) {
-            float wm = x[j];
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, off));
-            if (lane == 0) tm[sw * kDRows + j] = wm;
-          }
-          if (bar_red_or(1, kDSoftWarps * 32, bad)) {
-            stop = true;
-            break;
-          }
-          float f[kDRows];
-          bool any = false;
-#pragma unroll
-          for (int j = 0; j < kDRows; ++j) {
-            const float mt = fmaxf(fmaxf(tm[j], tm[kDRows + j]), fmaxf(tm[2 * kDRows + j], tm[3 * kDRows + j]));
-            f[j] = 1.f;
-            if (mt > m[j] + kDLazy) {               // the same decision in every thread
-              f[j] = m[j] == -INFINITY ? 0.f : ex2_approx(m[j] - mt);
-              m[j] = mt;
-              any = true;
-            }
-            l_run[h][j] *= f[j];
-          }
-          if (any && t > 0) {
-            // rescale the head's O^T columns (this thread's feature kt): hi and lo alike
-            uint32_t o[16];
-            tc_fence_after();
-            tmem_ld16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
-#pragma unroll
-            for (int j = 0; j < kDRows; ++j) {
-              o[j] = __float_as_uint(__uint_as_float(o[j]) * f[j]);
-              o[j + 8] = __float_as_uint(__uint_as_float(o[j + 8]) * f[j]);
-            }
-            tmem_st16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
-            tc_fence_before();
-          }
-        }
-        // p = exp2(s - m) as a bf16 pair into the head's P^T tile; the even lane of a key pair
-        // writes the high parts of both keys, the odd lane the low parts (rows rotated by 4 so
-        // that the two halves of the warp hit different banks)
-        uint32_t hl[kDRows];                         // (hi | lo << 16) of this key, per row
-#pragma unroll
-        for (int j = 0; j < kDRows; ++j) {
-          const float p = x[j] == -INFINITY ? 0.f : ex2_approx(x[j] - m[j]);
-          l_run[h][j] += p;
-          const __nv_bfloat16 hi = __float2bfloat16_rn(p);
-          const __nv_bfloat16 lo = __float2bfloat16_rn(p - __bfloat162float(hi));
-          hl[j] = static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
-                  (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16);
-        }
-        uint8_t *pt = ps + h * kDPBytes;
-#pragma unroll
-        for (int j = 0; j < kDRows; ++j) {
-          const int jl = (j + 4) & 7;
-          const uint32_t send = odd ? (hl[j] & 0xFFFFu) : (hl[jl] >> 16);
-          const uint32_t recv = __shfl_xor_sync(0xffffffffu, send, 1);
-          if (!odd)   // keys kt, kt + 1: high parts of row j
-            *reinterpret_cast<uint32_t *>(pt + p_off(j, kt)) = (hl[j] & 0xFFFFu) | (recv << 16);
-          else        // keys kt - 1, kt: low parts of row jl
-            *reinterpret_cast<uint32_t *>(pt + p_off(8 + jl, kt - 1)) = recv | (hl[jl] & 0xFFFF0000u);
-        }
-        if (kt == 0)
-#pragma unroll
-          for (int j = 0; j < kDRows; ++j) m_new[j] = m[j];
-        fence_proxy_async_smem();                    // the P tile is read by the tensor cores
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->p_full[h]);
+    for (int n = 0;; ++n) {
+      // the stage's record; the four warps leave together, at a barrier, at the end of the
+      // claims or when a wait gave up
+      const int r = n % kDInfo;
+      bool ok = __all_sync(0xffffffffu, d_wait(&bars->info_full[r], (n / kDInfo) & 1u, bars, err, 99));
+      const int u = ok ? bars->info[r] : -1;
+      if (bar_red_or(1, kDSoftWarps * 32, !ok || u < 0)) {
+        stop = bar_red_or(1, kDSoftWarps * 32, !ok);
+        break;
       }
+      const int t = u / HKV, h = u % HKV, buf = n & 1;
+      const bool hseen = (seen >> h) & 1u;
+      const uint32_t hpar = (par >> h) & 1u;
+      // every wait of the stage comes first; the group leaves only together, at a barrier
+      ok = __all_sync(0xffffffffu, d_wait(&bars->s_full[buf], (n >> 1) & 1u, bars, err, 95));
+      if (ok && hseen)   // the head's previous O^T MMAs are done: its P tile and O^T are free
+        ok = __all_sync(0xffffffffu, d_wait(&bars->p_empty[h], hpar ^ 1u, bars, err, 96));
+      const int key = t * kDM + kt;
+      const bool valid = key < sq.len;
+      const float *m_old = msm + (hpar ^ 1u) * HKV * kDRows + h * kDRows;
+      float *m_new = msm + hpar * HKV * kDRows + h * kDRows;
+      float x[kDRows], m[kDRows];
+      bool raise = false;
+#pragma unroll
+      for (int j = 0; j < kDRows; ++j) {
+        x[j] = -INFINITY;
+        m[j] = m_old[j];
+      }
+      if (ok) {
+        tc_fence_after();
+        uint32_t rr[8];
+        tmem_ld8_wait(bars->tmem_base + lane_off + buf * kDN, rr);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->s_empty[buf]);
+#pragma unroll
+        for (int j = 0; j < kDRows; ++j) {
+          x[j] = (valid && j < G) ? __uint_as_float(rr[j]) * c2 : -INFINITY;
+          raise |= x[j] > m[j] + kDLazy;           // also every finite logit against -inf
+        }
+      }
+      const bool bad = !ok || bars->abort;
+      if (bar_red_or(1, kDSoftWarps * 32, bad || raise)) {
+        // slow path (the head's first stage, a new maximum, or an abort): the tile's row maxima
+        float *tm = tmax + buf * kDSoftWarps * kDRows;
+#pragma unroll
+        for (int j = 0; j < kDRows; ++j) {
+          float wm = x[j];
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, off));
+          if (lane == 0) tm[sw * kDRows + j] = wm;
+        }
+        if (bar_red_or(1, kDSoftWarps * 32, bad)) {
+          stop = true;
+          break;
+        }
+        float f[kDRows];
+        bool any = false;
+#pragma unroll
+        for (int j = 0; j < kDRows; ++j) {
+          const float mt = fmaxf(fmaxf(tm[j], tm[kDRows + j]), fmaxf(tm[2 * kDRows + j], tm[3 * kDRows + j]));
+          f[j] = 1.f;
+          if (mt > m[j] + kDLazy) {               // the same decision in every thread
+            f[j] = m[j] == -INFINITY ? 0.f : ex2_approx(m[j] - mt);
+            m[j] = mt;
+            any = true;
+          }
+        }
+#pragma unroll
+        for (int hh = 0; hh < HKV; ++hh)            // register-resident sums: head selected by predicate
+          if (hh == h)
+#pragma unroll
+            for (int j = 0; j < kDRows; ++j) l_run[hh][j] *= f[j];
+        if (any && hseen) {
+          // rescale the head's O^T columns (this thread's feature kt): hi and lo alike
+          uint32_t o[16];
+          tc_fence_after();
+          tmem_ld16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
+#pragma unroll
+          for (int j = 0; j < kDRows; ++j) {
+            o[j] = __float_as_uint(__uint_as_float(o[j]) * f[j]);
+            o[j + 8] = __float_as_uint(__uint_as_float(o[j + 8]) * f[j]);
+          }
+          tmem_st16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
+          tc_fence_before();
+        }
+      }
+      // p = exp2(s - m) as a bf16 pair into the head's P^T tile; the even lane of a key pair
+      // writes the high parts of both keys, the odd lane the low parts (rows rotated by 4 so
+      // that the two halves of the warp hit different banks)
+      float pv[kDRows];
+      uint32_t hl[kDRows];                         // (hi | lo << 16) of this key, per row
+#pragma unroll
+      for (int j = 0; j < kDRows; ++j) {
+        pv[j] = x[j] == -INFINITY ? 0.f : ex2_approx(x[j] - m[j]);
+        const __nv_bfloat16 hi = __float2bfloat16_rn(pv[j]);
+        const __nv_bfloat16 lo = __float2bfloat16_rn(pv[j] - __bfloat162float(hi));
+        hl[j] = static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
+                (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16);
+      }
+#pragma unroll
+      for (int hh = 0; hh < HKV; ++hh)
+        if (hh == h)
+#pragma unroll
+          for (int j = 0; j < kDRows; ++j) l_run[hh][j] += pv[j];
+      uint8_t *pt = ps + h * kDPBytes;
+#pragma unroll
+      for (int j = 0; j < kDRows; ++j) {
+        const int jl = (j + 4) & 7;
+        const uint32_t send = odd ? (hl[j] & 0xFFFFu) : (hl[jl] >> 16);
+        const uint32_t recv = __shfl_xor_sync(0xffffffffu, send, 1);
+        if (!odd)   // keys kt, kt + 1: high parts of row j
+          *reinterpret_cast<uint32_t *>(pt + p_off(j, kt)) = (hl[j] & 0xFFFFu) | (recv << 16);
+        else        // keys kt - 1, kt: low parts of row jl
+          *reinterpret_cast<uint32_t *>(pt + p_off(8 + jl, kt - 1)) = recv | (hl[jl] & 0xFFFF0000u);
+      }
+      if (kt == 0)
+#pragma unroll
+        for (int j = 0; j < kDRows; ++j) m_new[j] = m[j];
+      fence_proxy_async_smem();                    // the P tile is read by the tensor cores
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->p_full[h]);
+      par ^= 1u << h;
+      seen |= 1u << h;
     }
-    // the head's last O^T MMAs must be complete before O^T is read
+    // each head's last O^T MMAs must be complete before O^T is read
     if (!stop)
 #pragma unroll
       for (int h = 0; h < HKV; ++h)
-        if (!__all_sync(0xffffffffu, d_wait(&bars->p_empty[h], (ntiles - 1) & 1u, bars, err, 97))) break;
+        if (((seen >> h) & 1u) &&
+            !__all_sync(0xffffffffu, d_wait(&bars->p_empty[h], ((par >> h) & 1u) ^ 1u, bars, err, 97)))
+          break;
   }
 
   // ---------------------------------------------------------------- epilogue and teardown
@@ -403,7 +494,10 @@ __global__ void __launch_bounds__(kDThreads, 1)
 #pragma unroll
     for (int h = 0; h < HKV; ++h) {
       uint32_t o[16];
-      tmem_ld16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) o[j] = 0u;
+      if ((seen >> h) & 1u)                      // uniform over the softmax warps
+        tmem_ld16_wait(bars->tmem_base + lane_off + 32 + h * kDN, o);
 #pragma unroll
       for (int j = 0; j < kDRows; ++j)           // feature kt of row j: high plus low part
         if (j < G)
@@ -412,11 +506,14 @@ __global__ void __launch_bounds__(kDThreads, 1)
 #pragma unroll
       for (int j = 0; j < kDRows; ++j) lsum[(h * kDRows + j) * kDM + kt] = l_run[h][j];
     }
-    if (kt == 0)   // the last tile's copy of the reference maximum
+    if (kt == 0)   // the reference maximum of each head's last stage (-inf: no stage)
 #pragma unroll
       for (int h = 0; h < HKV; ++h)
 #pragma unroll
-        for (int j = 0; j < kDRows; ++j) mrow[h * kDRows + j] = msm[((ntiles - 1) & 1) * HKV * kDRows + h * kDRows + j];
+        for (int j = 0; j < kDRows; ++j)
+          mrow[h * kDRows + j] = ((seen >> h) & 1u)
+                                     ? msm[(((par >> h) & 1u) ^ 1u) * HKV * kDRows + h * kDRows + j]
+                                     : -INFINITY;
   }
   tc_fence_before();
   __syncthreads();
@@ -438,7 +535,8 @@ __global__ void __launch_bounds__(kDThreads, 1)
 }  // namespace
 
 cudaError_t launch_decode_tc(int grid, cudaStream_t stream, const CUtensorMap &kmap, const CUtensorMap &vmap,
-                             const DecPlan &P, const uint16_t *q, float *opart, float2 *mlpart, DeviceError *err) {
+                             const DecPlan &P, const uint16_t *q, float *opart, float2 *mlpart, unsigned int *claims,
+                             DeviceError *err) {
   if (P.hkv == 4) {
     static std::atomic<uint64_t> attr{0};
     const cudaError_t e = once_per_device(attr, [] {
@@ -447,7 +545,7 @@ cudaError_t launch_decode_tc(int grid, cudaStream_t stream, const CUtensorMap &k
     });
     if (e != cudaSuccess) return e;
     return launch_pdl(decode_tc_kernel<4>, dim3(grid), dim3(kDThreads), DLay<4>::kBytes, stream, kmap, vmap, P, q,
-                      opart, mlpart, err);
+                      opart, mlpart, claims, err);
   } else {
     static std::atomic<uint64_t> attr{0};
     const cudaError_t e = once_per_device(attr, [] {
@@ -456,7 +554,7 @@ cudaError_t launch_decode_tc(int grid, cudaStream_t stream, const CUtensorMap &k
     });
     if (e != cudaSuccess) return e;
     return launch_pdl(decode_tc_kernel<2>, dim3(grid), dim3(kDThreads), DLay<2>::kBytes, stream, kmap, vmap, P, q,
-                      opart, mlpart, err);
+                      opart, mlpart, claims, err);
   }
 }
 

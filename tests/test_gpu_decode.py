@@ -71,9 +71,16 @@ def test_decode_attention_matches_oracle(ap, lens, hq, hkv):
     k = bits(rng, (T, hkv, 128), 1.5)        # peaky softmax
     v = bits(rng, (T, hkv, 128))
     got = run(ap, cu, q, k, v, hq, hkv)
-    check(got, oracle.decode_attention(q, k, v, cu, hq, hkv))
+    ref = oracle.decode_attention(q, k, v, cu, hq, hkv)
+    check(got, ref)
     again = run(ap, cu, q, k, v, hq, hkv)
-    assert got.tobytes() == again.tobytes()
+    if hkv in (2, 4) and hq // hkv <= 8:
+        # tensor-core path: tiles are claimed as the CTAs go, so two calls may group the keys'
+        # partial sums differently; both meet the rule and agree to fp32 rounding
+        check(again, ref)
+        np.testing.assert_allclose(again, got, rtol=1e-4, atol=1e-6)
+    else:                                    # CUDA-core path: a fixed split and merge order
+        assert got.tobytes() == again.tobytes()
 
 
 def test_decode_attention_strided_rows_and_uniform_keys(ap):
@@ -147,3 +154,30 @@ def test_decode_attention_rising_and_falling_maxima(ap, hq, hkv):
     v = bits(rng, (T, hkv, 128))
     got = run(ap, cu, q, k, v, hq, hkv)
     check(got, oracle.decode_attention(q, k, v, cu, hq, hkv))
+
+
+def test_decode_attention_repeated_calls_on_one_workspace(ap):
+    # On the tensor-core path the CTAs of a sequence claim its tiles from counters at the end of
+    # the workspace, and the combine kernel zeroes them again: after every call they must read
+    # zero, and every call must meet the rule (the tiles' split over CTAs varies between calls).
+    rng = np.random.default_rng(2024)
+    lens = [30011, 0, 4097, 1, 129]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = int(cu[-1])
+    q = bits(rng, (len(lens), 28, 128))
+    k = bits(rng, (T, 4, 128), 1.5)
+    v = bits(rng, (T, 4, 128))
+    ref = oracle.decode_attention(q, k, v, cu, 28, 4)
+    kd = torch.from_numpy(k.reshape(T, -1).view(np.int16)).cuda()
+    vd = torch.from_numpy(v.reshape(T, -1).view(np.int16)).cuda()
+    qd = torch.from_numpy(q.view(np.int16)).cuda()
+    n_ws = ap.apack_decode_workspace_size(cu, 28, 4)
+    ws = torch.zeros(n_ws, dtype=torch.uint8, device="cuda")
+    cl0 = n_ws - (len(lens) * 4 + 255) // 256 * 256          # the claim counters: the last region
+    for _ in range(12):
+        out = torch.full((len(lens), 28, 128), float("nan"), dtype=torch.float32, device="cuda")
+        ap.apack_decode_attention(cu, qd, kd, vd, 4 * 256, 28, 4, out, ws)
+        torch.cuda.synchronize()
+        assert ap.apack_device_error(ws) == ap.APACK_OK
+        assert not ws[cl0:cl0 + 4 * len(lens)].any()
+        check(out.cpu().numpy(), ref)
