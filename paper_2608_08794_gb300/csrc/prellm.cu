@@ -94,32 +94,46 @@ __global__ void __launch_bounds__(kCkaThreads)
   float ga[kG], gv[kG], dist = 0.f;
 #pragma unroll
   for (int i = 0; i < kG; ++i) ga[i] = gv[i] = 0.f;
-  for (int64_t x = threadIdx.x; x < dim; x += kCkaThreads) {
-    float av[W], vv[W], am = 0.f, vm = 0.f, dd = 0.f;
+  // four consecutive features per thread and step (16-byte loads of the pooled rows: dim is a
+  // multiple of 8 and the rows start 256-byte aligned)
+  const int64_t nv4 = dim / 4;
+  const float4 *a4 = reinterpret_cast<const float4 *>(a);
+  const float4 *v4 = reinterpret_cast<const float4 *>(v);
+  for (int64_t x = threadIdx.x; x < nv4; x += kCkaThreads) {
+    float4 a_r[W], v_r[W];
 #pragma unroll
     for (int r = 0; r < W; ++r) {
-      av[r] = r < w ? a[static_cast<int64_t>(lo + r) * dim + x] : 0.f;
-      vv[r] = r < w ? v[static_cast<int64_t>(lo + r) * dim + x] : 0.f;
-      am += av[r];
-      vm += vv[r];
-      if (r == center) dd = vv[r] - av[r];
+      a_r[r] = r < w ? a4[static_cast<int64_t>(lo + r) * nv4 + x] : make_float4(0.f, 0.f, 0.f, 0.f);
+      v_r[r] = r < w ? v4[static_cast<int64_t>(lo + r) * nv4 + x] : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    dist = fmaf(dd, dd, dist);
-    am *= inv_w;
-    vm *= inv_w;
 #pragma unroll
-    for (int r = 0; r < W; ++r) {
-      av[r] = r < w ? av[r] - am : 0.f;
-      vv[r] = r < w ? vv[r] - vm : 0.f;
-    }
-    int k = 0;
+    for (int e = 0; e < 4; ++e) {             // the four features in order
+      float av[W], vv[W], am = 0.f, vm = 0.f, dd = 0.f;
 #pragma unroll
-    for (int i = 0; i < W; ++i)
-#pragma unroll
-      for (int j = i; j < W; ++j, ++k) {
-        ga[k] = fmaf(av[i], av[j], ga[k]);
-        gv[k] = fmaf(vv[i], vv[j], gv[k]);
+      for (int r = 0; r < W; ++r) {
+        av[r] = e == 0 ? a_r[r].x : e == 1 ? a_r[r].y : e == 2 ? a_r[r].z : a_r[r].w;
+        vv[r] = e == 0 ? v_r[r].x : e == 1 ? v_r[r].y : e == 2 ? v_r[r].z : v_r[r].w;
+        am += av[r];
+        vm += vv[r];
+        if (r == center) dd = vv[r] - av[r];
       }
+      dist = fmaf(dd, dd, dist);
+      am *= inv_w;
+      vm *= inv_w;
+#pragma unroll
+      for (int r = 0; r < W; ++r) {
+        av[r] = r < w ? av[r] - am : 0.f;
+        vv[r] = r < w ? vv[r] - vm : 0.f;
+      }
+      int k = 0;
+#pragma unroll
+      for (int i = 0; i < W; ++i)
+#pragma unroll
+        for (int j = i; j < W; ++j, ++k) {
+          ga[k] = fmaf(av[i], av[j], ga[k]);
+          gv[k] = fmaf(vv[i], vv[j], gv[k]);
+        }
+    }
   }
   // fixed-order block reduction: warp trees, then one thread per sum over the warps in order
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
