@@ -57,9 +57,11 @@ def parse():
                    help="with several GPUs, run the whole batch on every rank instead of splitting its sequences")
     p.add_argument("--no-paper-setting", action="store_true",
                    help="skip the side measurement of the paper's own 14-step setting")
-    p.add_argument("--part", default="all", choices=["all", "decode", "compact"],
+    p.add_argument("--part", default="all", choices=["all", "decode", "compact", "prellm"],
                    help="decode: time only the decode-step attention on a synthetic cache; compact: only "
-                        "the first step's compaction of the 10-minute 7B cache, out of place and in place")
+                        "the first step's compaction of the 10-minute 7B cache, out of place and in place; "
+                        "prellm: only the pre-LLM frame alignment of the workload's clip")
+    p.add_argument("--window", type=int, default=3, help="prellm: the CKA window (odd, 1..7)")
     p.add_argument("--compact-planes", type=int, default=48,
                    help="compact: planes of 135272 rows (48 = K and V of layers 4..27)")
     p.add_argument("--decode-tokens", type=int, default=135272)
@@ -530,7 +532,7 @@ def prellm_cpu_baseline(wl, frames=24):
                       f"fp64 oracle (literal d x d products), {sec:.1f} s"}
 
 
-def prellm_measure(ap, wl, steps, warmup, stream, dist):
+def prellm_measure(ap, wl, steps, warmup, stream, dist, window=3):
     """Pre-LLM frame alignment (Sec. 3.1, Eq. cka and Eq. gate) of the
     workload's clip: pooled frame embeddings, windowed CKA and the gate, one
     apack_frame_alignment call per step.  The bf16 encoder tokens are read
@@ -548,7 +550,7 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
     sc = torch.empty_like(c)
 
     def call():
-        ap.apack_frame_alignment(vis, aud, F, tpf, na, dim, c, sc, ws, stream=stream)
+        ap.apack_frame_alignment(vis, aud, F, tpf, na, dim, c, sc, ws, window=window, stream=stream)
 
     for _ in range(max(3, warmup)):
         call()
@@ -574,7 +576,7 @@ def prellm_measure(ap, wl, steps, warmup, stream, dist):
     return {"metric": "frames aligned per second", "value": F / (ms / 1e3), "unit": "frames/s",
             "ms_per_clip": ms, "steps": k, "gpu_launches": int(launches),
             "config": {"workload": f"{wl.name} clip: {F} frames x {tpf} visual tokens, {na} audio tokens, d={dim}",
-                       "window": 3, "tau": 0.78, "beta": 0.90,
+                       "window": window, "tau": 0.78, "beta": 0.90,
                        "l2": "inputs larger than L2 (%.2f GB of bf16 encoder tokens)" % (token_bytes / 1e9)},
             "roofline": {"bound": "hbm", "kernel": "apack_frame_alignment call (frame_pool_kernel + "
                                                    "frame_cka_gate_kernel)",
@@ -978,6 +980,14 @@ def main():
     if args.part == "compact":
         compact_only(args)
         return
+    if args.part == "prellm":
+        import torch
+        import paper_2608_08794_gb300 as ap
+        from synth import workload
+        torch.cuda.set_device(local)
+        print(json.dumps(prellm_measure(ap, workload(args.workload), args.steps, args.warmup,
+                                        torch.cuda.current_stream(), None, window=args.window)))
+        return
 
     import numpy as np
     import torch
@@ -1101,7 +1111,9 @@ def main():
     # directions) without holding up iteration i+2's upload: with two sets, the gather queue
     # stood idle while one iteration's read-back, the next upload and its first selection ran.
     # Each step waits only for its own schedule's previous gather (not for gathers of the next
-    # iteration queued meanwhile), so its scoring overlaps them.
+    # iteration queued meanwhile), so its scoring overlaps them; the next iteration's first
+    # gather is queued before this iteration's last step, so the link never waits for a step's
+    # scoring and selection.
     e2e_steps = args.e2e_steps or max(3, min(args.steps, 20))
     pp2, pp3 = (ProgressivePrune(cu0, cuq, na, nv, wl.num_q_heads, wl.num_kv_heads, wl.num_layers, wl.hidden,
                                  wl.prune_layers, counts, select_mode=mode) for _ in range(2))
@@ -1163,12 +1175,18 @@ def main():
         stream.wait_event(ev_up[b])
         p.host_step(0, h_k, h_v, h_h, stream=stream, gather_stream=s_gather)
 
+    def middle(j):
+        """Steps 1 .. n-2 of iteration j."""
+        p = sets[j % len(sets)]
+        for i in range(1, nsteps - 1):
+            p.host_step(i, h_k, h_v, h_h, stream=stream, gather_stream=s_gather)
+
     def back(j):
-        """The later steps and the read-back of iteration j."""
+        """The last step and the read-back of iteration j."""
         b = j % len(sets)
         p = sets[b]
-        for i in range(1, nsteps):
-            p.host_step(i, h_k, h_v, h_h, stream=stream, gather_stream=s_gather)
+        if nsteps > 1:
+            p.host_step(nsteps - 1, h_k, h_v, h_h, stream=stream, gather_stream=s_gather)
         ev_comp[b].record(stream)
         with torch.cuda.stream(s_down):
             s_down.wait_event(ev_comp[b])
@@ -1181,10 +1199,12 @@ def main():
             ev_down[b].record(s_down)
 
     def e2e_run(n):
-        # software pipeline: iteration j+1's upload, scoring and selection are queued before
-        # iteration j's later steps, so that they run while iteration j's gather holds the link
+        # software pipeline: iteration j+1's upload, scoring, selection and first gather are
+        # queued before iteration j's last step, so that the link carries that gather while the
+        # last step scores and selects, and the last step's scoring runs during it
         front(0)
         for j in range(n):
+            middle(j)
             if j + 1 < n:
                 front(j + 1)
             back(j)
