@@ -5,7 +5,9 @@
 //   out[b, h] = sum_j softmax_j(q[b, h] . k[j, g(h)] / sqrt(128)) v[j, g(h)],
 //   g(h) = h / (Hq / Hkv), j over every cached token of sequence b.
 //
-// Split-KV in two launches:
+// Split-KV in two launches.  With Hkv 2 or 4 and at most 8 query rows per KV head the chunk
+// kernel is the tensor-core one of decode_tc.cu (its CTAs claim the sequence's stages from a
+// counter, so the keys' grouping into partials varies from call to call); otherwise:
 //   chunk kernel:   one CTA per (sequence, chunk of about T / #SMs keys).  K and V rows
 //                   stream into a 3-stage shared-memory ring by bulk async copies (issued
 //                   by one lane).  Each of 16 warps works on KV head
@@ -18,8 +20,9 @@
 //                   accumulated in registers.  The warps of a head merge in shared memory;
 //                   the CTA writes (max, sum, o[128]) per query head.
 //   combine kernel: one CTA per (sequence, query head) merges the chunks in order.
-// K and V are read once: the chunk kernel is HBM-bound.  All merges run in a fixed
-// order, so the output is deterministic.
+// K and V are read once: the chunk kernel is HBM-bound.  The CUDA-core path's merges run in a
+// fixed order, so its output is deterministic; the combine merges any path's partials in a
+// fixed order.
 #include <algorithm>
 #include <cmath>
 
