@@ -96,10 +96,9 @@ __global__ void __launch_bounds__(tc_threads<HKV>(), 1)
   const int te = min(sq.len, tb + plan.chunk);
   const int ntiles = (te - tb + kTcM - 1) / kTcM;
 
-  // zeroed ring; query tiles in the 128-byte-swizzled K-major layout: row r, 16-byte chunk
-  // cc of a 64-dim half sits at chunk cc ^ (r & 7) of the row's 128 bytes
-  for (uint32_t i = threadIdx.x; i < Lay::kOffQ / 16; i += tc_threads<HKV>())
-    reinterpret_cast<uint4 *>(ring)[i] = make_uint4(0, 0, 0, 0);
+  // query tiles in the 128-byte-swizzled K-major layout: row r, 16-byte chunk cc of a 64-dim
+  // half sits at chunk cc ^ (r & 7) of the row's 128 bytes (every ring stage the MMAs read is
+  // written whole by its TMA load, rows past the cache as zeros)
   for (int idx = threadIdx.x; idx < HKV * kTcN * 16; idx += tc_threads<HKV>()) {
     const int h = idx / (kTcN * 16), rem = idx % (kTcN * 16);
     const int row = rem / 16, ch = rem % 16;
