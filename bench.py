@@ -645,15 +645,15 @@ def final_levels_measure(ap, pp, nsteps, mm_per_iter, steps, warmup, stream, dis
     for i in range(nsteps):
         c, t = pp.fin_layers[i], pp.t_out[i]
         planes = 2 * c + (1 if i + 1 < nsteps else 0)
-        moved += 2 * t * (planes * pp.row + pp.H * 2) + 4 * t
+        moved += 2 * t * (planes * pp.row + (pp.H * 2 if i + 1 == nsteps else 0)) + 4 * t
     best = graph_ms if graph_ms is not None else ms
     return {"value": mm_per_iter / (best / 1e3), "unit": UNIT, "ms_per_step": best, "steps": steps,
             "eager_ms_per_step": ms, "graph_error": graph_error, "bytes_moved_per_iter": int(moved),
             "equal_to_per_step_schedule": bool(same),
             "how": "the library calls of ProgressivePrune.run_from_host captured once as a CUDA graph and replayed "
-                   "(eager_ms_per_step: direct calls); every layer's K/V written once at its final level from the "
-                   "step-0 input, the scored keys and the hidden states compacted per step; the per-step schedule "
-                   "of the headline compacts layers [l_i, L) at every step"}
+                   "(eager_ms_per_step: direct calls); every layer's K/V and the hidden states written once at their "
+                   "final level from the step-0 input, the scored keys compacted per step; the per-step schedule "
+                   "of the headline compacts layers [l_i, L) and the hidden states at every step"}
 
 
 def link_rates(h_k, h_v, pp2, s_up, s_down, reps=3):
@@ -1142,12 +1142,12 @@ def main():
     h_out = [host_outputs(p) for p in sets]
     # bytes over the link per iteration: the copies (scored keys, modality, queries) and the rows
     # the gathers read from host memory (step i: the V of its layers, their K but for its scored
-    # layer's after step 0, the next step's scored keys; step 0 also the hidden states)
+    # layer's after step 0, the next step's scored keys; the last step also the hidden states)
     h2d = h_k[0].numel() * h_k.element_size() + h_m.numel() + sum(x.numel() * x.element_size() for x in h_q)
     for i in range(nsteps):
         c = pp.fin_layers[i]
         planes = 2 * c - (1 if i > 0 else 0) + (1 if i + 1 < nsteps else 0)
-        h2d += pp.t_out[i] * (planes * pp.row + (pp.H * 2 if i == 0 else 0))
+        h2d += pp.t_out[i] * (planes * pp.row + (pp.H * 2 if i + 1 == nsteps else 0))
     d2h = sum(x.numel() * x.element_size() for x in h_out[0])
     # the device work of the e2e pipeline runs on a stream of the highest priority, so that its
     # kernels take SMs as soon as CTAs of the link-bound gather (default priority) retire
@@ -1289,8 +1289,9 @@ def main():
                     "pipeline": "caches and hidden states in pinned host memory; per iteration the scored layer's "
                                 "keys, the queries and the modality are copied; every step scores and selects on the "
                                 "device and gathers over the host link (its own stream), at the composed indices, "
-                                "the layers that end at its level plus the keys the next step scores, so each "
-                                "layer's rows cross the link once; the result is every layer's final cache on the "
+                                "the layers that end at its level plus the keys the next step scores (the last step "
+                                "also the hidden states), so each layer's rows and the hidden states cross the link "
+                                "once; the result is every layer's final cache on the "
                                 "device, of which the last step's layers, the hidden states and the indices are read "
                                 "back; three device buffer sets let the next iteration's upload and first selection "
                                 "and the previous read-back run while the current gathers hold the link",

@@ -255,8 +255,9 @@ class ProgressivePrune:
         host memory (laid out like k_in / v_in / hidden_in; the caller copies the scored keys,
         slab 0 of k_in, to the device).  Every layer's rows cross the host link once, at the level
         that layer ends at: step i gathers, at the composed indices of steps 0..i, the K and V of
-        layers [l_i, l_(i+1)) and the keys that step i+1 scores (layer l_(i+1)).  Only the scored
-        keys of step i (already on the device) and the hidden states are compacted on the device.
+        layers [l_i, l_(i+1)) and the keys that step i+1 scores (layer l_(i+1)); the last step
+        also gathers the hidden states.  Only the scored keys of step i (already on the device)
+        are compacted on the device.
         Scoring and selection are those of run_step, so keep_idx, scores and the caches equal the
         per-step schedule's bit for bit; the result is every layer's final cache (final_kv),
         output_hidden(last) and keep_idx.  gather_stream: None, or a stream for the host-link
@@ -282,8 +283,8 @@ class ProgressivePrune:
         t = self.t_out[i]
         k_sc = self.k_in.view(-1) if i == 0 else self.k_score[i]
         if i > 0 and gs is not stream:
-            # the scored keys (and at step 1 the step-0 hidden rows) came over the link in step
-            # i-1's gather; later gathers queued on gs meanwhile (another schedule's) need not end
+            # the scored keys came over the link in step i-1's gather; later gathers queued on gs
+            # meanwhile (another schedule's) need not end
             (stream or torch.cuda.current_stream()).wait_event(self.gather_done[i - 1])
         apack_score(seqs, self.q[i], k_sc, row, self.scores, self.ws, stream=stream)
         apack_select(seqs, self.scores, self.counts[i], self.keep_idx[i], self.ws, select_mode=self.mode,
@@ -304,19 +305,17 @@ class ProgressivePrune:
         if i + 1 < n:
             planes.append(_plane(kh + (self.layers[i + 1] - l0) * T0 * row, self.k_score[i + 1].data_ptr(),
                                  T0 * row, t * row, row, 1))
-        if i == 0 and hidden_host is not None and self.h_out[0] is not None:
-            planes.append(make_plane(hidden_host, self.h_out[0], self.H * 2, 1))
+        if i + 1 == n and hidden_host is not None and self.h_out[0] is not None:
+            # the hidden states cross once too, at the level they end at
+            planes.append(make_plane(hidden_host, self.h_out[i % 2], self.H * 2, 1))
         if gs is not stream:
             _wait(gs, stream)
         apack_compact(comp, t, planes, ws=self.ws, stream=gs)
         if gs is not stream:
             self.gather_done[i].record(gs)
-        if i > 0:                              # device-side: the scored keys and the hidden states
-            dev_planes = [_plane(self.k_score[i].data_ptr(), kf, 0, 0, row, 1)]
-            h_prev, h_new = self.h_out[(i - 1) % 2], self.h_out[i % 2]
-            if h_prev is not None and hidden_host is not None:
-                dev_planes.append(make_plane(h_prev, h_new, self.H * 2, 1))
-            apack_compact(self.keep_idx[i], t, dev_planes, ws=self.ws, stream=stream)
+        if i > 0:                              # device-side: layer l_i's keys, scored above
+            apack_compact(self.keep_idx[i], t, [_plane(self.k_score[i].data_ptr(), kf, 0, 0, row, 1)], ws=self.ws,
+                          stream=stream)
         k = self.counts[i]
         cu = np.zeros(self.B + 1, np.int32)
         cu[1:] = np.cumsum(other + k[:, 0] + k[:, 1])
