@@ -814,6 +814,8 @@ def paper_setting_measure(ap, steps, warmup, stream, dist, clocks=None):
                                    "peak_source": peak_kind},
            "how": "the 14-step schedule captured once by apack_prune_schedule_graph and replayed; stage times "
                   "from direct apack_prune_schedule calls with stage events"}
+    # the same 14 steps with every layer and the hidden states written once, at their final level
+    out["schedule_final_levels"] = final_levels_measure(ap, pp, nsteps, mm_per_iter, steps, warmup, stream, dist)
     del pp
     torch.cuda.empty_cache()
     return out
