@@ -181,3 +181,26 @@ def test_decode_attention_repeated_calls_on_one_workspace(ap):
         assert ap.apack_device_error(ws) == ap.APACK_OK
         assert not ws[cl0:cl0 + 4 * len(lens)].any()
         check(out.cpu().numpy(), ref)
+
+
+RANDOM_HEADS = [(28, 4), (16, 2), (12, 4), (32, 4), (8, 2), (8, 8), (8, 1), (4, 4)]
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_random_decode_matches_oracle(ap, seed):
+    # random batches: one to eight sequences of 0 to 20000 cached tokens (some empty, some shorter
+    # than one 128-key tile), every supported head layout (the tensor-core path for Hkv 2 or 4,
+    # the CUDA-core path otherwise), key scales from flat to peaky softmax, and a token-row
+    # stride wider than the heads in half the cases
+    rng = np.random.default_rng(9000 + seed)
+    hq, hkv = RANDOM_HEADS[seed % len(RANDOM_HEADS)]
+    B = int(rng.integers(1, 9))
+    lens = [0 if rng.random() < 0.1 else int(rng.choice([rng.integers(1, 130), rng.integers(1, 20000)]))
+            for _ in range(B)]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    T = int(cu[-1])
+    q = bits(rng, (B, hq, 128))
+    k = bits(rng, (T, hkv, 128), float(rng.choice([0.3, 1.0, 2.0])))
+    v = bits(rng, (T, hkv, 128))
+    got = run(ap, cu, q, k, v, hq, hkv, pad_heads=int(rng.integers(0, 2)))
+    check(got, oracle.decode_attention(q, k, v, cu, hq, hkv))
